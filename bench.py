@@ -1,0 +1,404 @@
+#!/usr/bin/env python3
+"""Complete-detection latency of RTCC vs Barrier on the 3-agent PointPillars
+workload (256x256 grid, 100k points + 20x500 clustered points per agent, max
+fusion, arrivals U[0, 30] ms), plus the encoder's tensor-core throughput and
+the fusion kernel's bandwidth.
+
+One step = four frames of the whole hot path, each replayed in real time from
+a seeded arrival trace: {RTCC, Barrier} x {inputs resident in HBM, inputs in
+pinned host memory copied on release}.  The order of RTCC and Barrier
+alternates between steps.  L2 is flushed (a 512 MiB device write) before every
+frame.  Latency = host time the detections are ready (after the D2H of the
+boxes) minus host time of the call that delivered the last payload.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+`value` is the RTCC p50 latency with resident inputs; `e2e` the same with
+host inputs (H2D inside the measured span).  --impl reference times the CPU
+oracle on this workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = "complete-detection latency p50/p99 ms RTCC vs barrier; conv TFLOP/s, fusion GB/s"
+WORKLOAD = "pp3"
+DATA = ("synthetic: seeded uniform + Gaussian-cluster point clouds, He-normal fp32 weights "
+        "rounded to fp16, seeded arrival traces (OPV2V and the trained OpenCOOD model are not "
+        "available)")
+FLUSH_BYTES = 512 << 20
+
+
+def _peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), float(d["bf16_tflops"]), "measured"
+    except Exception:
+        return 6800.0, 1900.0, "fallback"
+
+
+def conv_flops(cfg) -> float:
+    """Algorithmic FLOPs of one encoder branch's convs and deconvs (2 per MAC)."""
+    fl = 0.0
+    w, h, cin = cfg.grid_w, cfg.grid_h, cfg.pfn_ch
+    dims = []
+    for (n, ch, st) in cfg.blocks:
+        for li in range(n):
+            s = st if li == 0 else 1
+            w, h = w // s, h // s
+            fl += 2.0 * w * h * ch * 9 * cin
+            cin = ch
+        dims.append((w, h, ch))
+    for bi, s in enumerate(cfg.up_strides):
+        bw, bh, bc = dims[bi]
+        fl += 2.0 * (bw * s) * (bh * s) * cfg.up_ch * bc
+    return fl
+
+
+def fusion_bytes(cfg, k_present: int) -> float:
+    """Algorithmic bytes of the fusion+head kernel: each present slot read
+    once (16-bit), the fp32 head map written once."""
+    cells = cfg.feat_w * cfg.feat_h
+    return float(k_present * cells * cfg.feat_ch * 2 + cells * 16 * 4)
+
+
+def pct(x, q):
+    return float(np.percentile(np.asarray(x, dtype=np.float64), q)) if len(x) else None
+
+
+# --------------------------------------------------------------------------
+# clocks during the timed region
+# --------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.rows = []
+        self.proc = None
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) >= 8:
+                self.rows.append(parts)
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+        if self.thread is not None:
+            self.thread.join(timeout=2)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in self.rows:
+            try:
+                sm.append(float(r[0]))
+                mx.append(float(r[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, r[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": float(max(mx)),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# --------------------------------------------------------------------------
+# CPU oracle timing (cpu_baseline leg and the reference arm)
+# --------------------------------------------------------------------------
+
+def oracle_step(cfg, w, pts_agent, arrivals_list):
+    """Time one oracle encoder branch and one oracle post-join; return the
+    measured service times and the RTCC tail latency of each arrival trace
+    under the single-stream timeline (Eqs. 20-22) with those times."""
+    from oracle import forward as of
+    from oracle import schedule as sch
+    t0 = time.perf_counter()
+    enc = of.encoder(pts_agent, w, cfg, store=cfg.dtype)
+    t1 = time.perf_counter()
+    feats = [enc["feat"]] * cfg.n_agents
+    F = of.fuse_max(feats) if cfg.fusion == "max" else of.fuse_attn(feats)
+    hd = of.head(F, of.store_round(w["head.w"], cfg.dtype), of.store_round(w["head.b"], cfg.dtype))
+    of.decode(hd, cfg)
+    t2 = time.perf_counter()
+    c_enc = int((t1 - t0) * 1e9)
+    c_post = int((t2 - t1) * 1e9)
+    tails = []
+    for a in arrivals_list:
+        a_ns = [int(x * 1e6) for x in a]
+        tails.append(sch.simulate(a_ns, [c_enc] * cfg.n_agents, [c_post], "rtcc")["T_tail"] / 1e6)
+    return c_enc / 1e6, c_post / 1e6, tails
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    cfg = synth.get_config(WORKLOAD)
+    w = synth.weights_for(cfg)
+    cores = os.cpu_count()
+    for s in range(args.warmup):
+        oracle_step(cfg, w, synth.points_for(cfg, s, 0), [synth.arrivals_for(cfg, s)])
+    tails, c_encs, c_posts = [], [], []
+    t_start = time.perf_counter()
+    for s in range(args.steps):
+        ce, cp, t = oracle_step(cfg, w, synth.points_for(cfg, s, s % cfg.n_agents),
+                                [synth.arrivals_for(cfg, s)])
+        tails += t
+        c_encs.append(ce)
+        c_posts.append(cp)
+    wall = (time.perf_counter() - t_start) * 1e3
+    v = pct(tails, 50)
+    sample = (f"per step: one oracle encoder branch (float64 NumPy, {cfg.name} shapes) and one "
+              f"post-join; the {cfg.n_agents}-agent frame's tail from those service times on the "
+              f"single-stream timeline (Eqs. 20-22)")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": v, "unit": "ms", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": wall / max(args.steps, 1),
+        "higher_is_better": False, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": DATA, "config": {"workload": _workload_desc(cfg)},
+        "latency_ms": {"rtcc_p50": v, "rtcc_p99": pct(tails, 99),
+                       "encoder_ms_median": float(np.median(c_encs)),
+                       "post_join_ms_median": float(np.median(c_posts))},
+        "cpu_baseline": {"value": v, "unit": "ms", "cores": cores, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": v, "unit": "ms", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def _workload_desc(cfg):
+    return (f"{cfg.name}: {cfg.n_agents}-agent PointPillars intermediate fusion, "
+            f"{cfg.grid_w}x{cfg.grid_h} pillar grid (0.4 m), {cfg.n_uniform} uniform + "
+            f"{cfg.n_clusters}x{cfg.cluster_pts} clustered points per agent, P_max "
+            f"{cfg.max_pillars}, N_max {cfg.max_pts}, backbone 3/5/5 convs 64/128/256 ch, "
+            f"deconv neck to {cfg.feat_w}x{cfg.feat_h}x{cfg.feat_ch}, {cfg.fusion} fusion, "
+            f"1x1 head, top-{cfg.max_boxes} decode; arrivals U[0,30] ms")
+
+
+# --------------------------------------------------------------------------
+# our arm
+# --------------------------------------------------------------------------
+
+def run_ours(args):
+    import torch
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    from paper_2608_08330_gb300 import build as B
+    if rank == 0 or world == 1:
+        B.build()
+    if dist is not None:
+        dist.barrier()
+    B.build()
+    from paper_2608_08330_gb300 import rtcc as R
+    R.load()
+
+    cfg = synth.get_config(WORKLOAD)
+    w = synth.weights_for(cfg)
+    ctx = R.rtcc_init(R.model_config(cfg, flags=R.FLAG_TIMELINE), synth.weight_blob(w))
+    K = cfg.n_agents
+    NF = 4
+    frames = [[synth.points_for(cfg, f, k) for k in range(K)] for f in range(NF)]
+    staging = [R.rtcc_staging_buffer(ctx, k) for k in range(K)]
+    flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    fid = [0]
+
+    def one_frame(step, mode, resident):
+        pts = frames[step % NF]
+        a = synth.arrivals_for(cfg, step)
+        flush.zero_()
+        torch.cuda.synchronize()
+        for k in range(K):
+            if resident:
+                assert R.rtcc_stage_resident(ctx, k, pts[k]) == R.OK
+            else:
+                staging[k][:pts[k].shape[0]] = pts[k]
+        assert R.rtcc_set_mode(ctx, mode) == R.OK
+        fid[0] += 1
+        assert R.rtcc_frame_begin(ctx, fid[0], 0.0) == R.OK
+        t0 = R.rtcc_now_ms() + 0.5
+        for k in sorted(range(K), key=lambda k: (a[k], k)):
+            due = t0 + a[k]
+            while True:
+                rem = due - R.rtcc_now_ms()
+                if rem <= 0:
+                    break
+                if rem > 2.0:
+                    time.sleep((rem - 1.5) / 1e3)
+            if resident:
+                s = R.rtcc_payload_resident(ctx, k, float(a[k]))
+            else:
+                n = pts[k].shape[0]
+                s = R.rtcc_payload_complete(ctx, k, staging[k][:n], float(a[k]))
+            assert s == R.OK, R.rtcc_status_str(s)
+        s, boxes, _ = R.rtcc_wait_detection(ctx, 10000)
+        assert s == R.OK, R.rtcc_status_str(s)
+        info = R.rtcc_get_frame_info(ctx)
+        return {"tail": info.t_ready_ms - info.t_last_event_ms,
+                "bb": [info.gpu_backbone_ms[k] for k in range(K)],
+                "fuse": info.gpu_fusion_ms, "post": info.gpu_post_ms,
+                "branch": [info.gpu_branch_ms[k] for k in range(K)], "n_boxes": len(boxes)}
+
+    def step_frames(step):
+        modes = (R.MODE_RTCC, R.MODE_BARRIER) if step % 2 == 0 else (R.MODE_BARRIER, R.MODE_RTCC)
+        out = []
+        for resident in (True, False):
+            for mode in modes:
+                out.append((mode, resident, one_frame(step, mode, resident)))
+        return out
+
+    for s in range(args.warmup):
+        step_frames(1000 + s)
+
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks = ClockSampler(torch.cuda.current_device())
+    clocks.start()
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    ev0.record()
+    t_start = time.perf_counter()
+    rec = []
+    for s in range(args.steps):
+        rec += step_frames(s)
+    torch.cuda.synchronize()
+    ev1.record()
+    torch.cuda.synchronize()
+    wall_ms = (time.perf_counter() - t_start) * 1e3
+    if dist is not None:
+        dist.barrier()
+    clk = clocks.stop()
+
+    def tails(mode, resident):
+        return [r["tail"] for (m, res, r) in rec if m == mode and res == resident]
+
+    r_res, b_res = tails(R.MODE_RTCC, True), tails(R.MODE_BARRIER, True)
+    r_e2e, b_e2e = tails(R.MODE_RTCC, False), tails(R.MODE_BARRIER, False)
+    bb = [x for (m, res, r) in rec if m == R.MODE_RTCC and res for x in r["bb"] if x > 0]
+    fu = [r["fuse"] for (m, res, r) in rec if m == R.MODE_RTCC and res and r["fuse"] > 0]
+    value = pct(r_res, 50)
+    if dist is not None:
+        t = torch.tensor([value, wall_ms], device="cuda", dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        value, wall_ms = float(t[0]), float(t[1])
+
+    hbm, tflops_peak, peak_kind = _peaks()
+    flops = conv_flops(cfg)
+    bb_ms = float(np.mean(bb)) if bb else None
+    enc_tflops = flops / (bb_ms * 1e-3) / 1e12 if bb_ms else None
+    fu_ms = float(np.mean(fu)) if fu else None
+    fu_gbs = fusion_bytes(cfg, K) / (fu_ms * 1e-3) / 1e9 if fu_ms else None
+    n_launch = R.rtcc_kernels_per_frame(ctx, K) * 4 * args.steps
+    h2d = sum(int(p.shape[0]) * 16 + 16 for p in frames[0])
+    d2h = 16 + cfg.max_boxes * 36
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "ms", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": wall_ms / max(args.steps, 1),
+        "higher_is_better": False, "scaling": "weak", "vs_baseline": None, "dtype": "fp16",
+        "data": DATA,
+        "config": {"workload": _workload_desc(cfg), "frames_per_step": 4,
+                   "l2": "flushed by a 512 MiB device write before every frame",
+                   "inputs": "value: payloads resident in HBM before release; e2e: pinned host "
+                             "staging, H2D on release inside the measured span",
+                   "replicas": world},
+        "latency_ms": {"rtcc_p50": value, "rtcc_p99": pct(r_res, 99),
+                       "barrier_p50": pct(b_res, 50), "barrier_p99": pct(b_res, 99),
+                       "e2e_rtcc_p50": pct(r_e2e, 50), "e2e_rtcc_p99": pct(r_e2e, 99),
+                       "e2e_barrier_p50": pct(b_e2e, 50), "e2e_barrier_p99": pct(b_e2e, 99),
+                       "frames_per_mode": len(r_res)},
+        "encoder": {"tflops": enc_tflops, "frac_of_bf16_peak": (enc_tflops / tflops_peak)
+                    if enc_tflops else None, "backbone_ms_per_branch": bb_ms,
+                    "gflop_per_branch": flops / 1e9},
+        "fusion": {"gbs": fu_gbs, "frac_of_hbm": (fu_gbs / hbm) if fu_gbs else None,
+                   "ms": fu_ms, "mb_per_launch": fusion_bytes(cfg, K) / 1e6},
+        "roofline": {"kernel": "k_conv_tc (tcgen05 implicit-GEMM conv/deconv backbone of one "
+                               "branch, 13 convs + 3 deconvs)",
+                     "bound": "tensor", "achieved": enc_tflops, "peak": tflops_peak,
+                     "unit": "TFLOP/s", "frac": (enc_tflops / tflops_peak) if enc_tflops else None,
+                     "peak_kind": f"{peak_kind} bf16 burst (fp16 has the same nominal rate)",
+                     "traffic": None},
+        "e2e": {"value": pct(r_e2e, 50), "unit": "ms", "h2d_bytes_per_step": 2 * h2d,
+                "d2h_bytes_per_step": 2 * d2h},
+        "clocks": clk,
+        "gpu_launches": n_launch,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        arr = [synth.arrivals_for(cfg, s) for s in range(args.steps)]
+        ce, cp, ct = oracle_step(cfg, w, frames[0][0], arr)
+        line["cpu_baseline"] = {
+            "value": pct(ct, 50), "unit": "ms", "cores": os.cpu_count(), "kind": "oracle",
+            "sample": (f"one oracle encoder branch ({ce:.0f} ms) and one post-join ({cp:.0f} ms) "
+                       f"in float64 NumPy; RTCC tail of each timed step's arrival trace on the "
+                       f"single-stream timeline (Eqs. 20-22) with those service times")}
+    R.rtcc_destroy(ctx)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -249,8 +249,29 @@ def weight_layout(cfg: ModelConfig) -> List[Tuple[str, Tuple[int, ...], int]]:
     return out
 
 
+def pfn_feature_stats(cfg: ModelConfig) -> Tuple[np.ndarray, np.ndarray]:
+    """Population mean and variance of the 9 PFN input features under the
+    synthetic point recipe (x, y, z, intensity uniform over their ranges;
+    offsets to the pillar mean and centre spread over one pillar)."""
+    v = cfg.pillar
+    ux = lambda lo, hi: ((lo + hi) / 2.0, (hi - lo) ** 2 / 12.0)
+    mx, vx = ux(*cfg.pts_x)
+    my, vy = ux(*cfg.pts_y)
+    mz, vz = ux(*cfg.pts_z)
+    mean = np.array([mx, my, mz, 0.5, 0.0, 0.0, 0.0, 0.0, 0.0])
+    var = np.array([vx, vy, vz, 1.0 / 12.0, v * v / 12.0, v * v / 12.0, vz / 2.0,
+                    v * v / 12.0, v * v / 12.0])
+    return mean, var
+
+
 def weights_for(cfg: ModelConfig) -> dict:
     """fp32 master weights: He-normal std sqrt(2/fan_in), biases U(-0.1, 0.1).
+
+    The PFN's linear layer is followed by BatchNorm in PointPillars; here a
+    BatchNorm with the synthetic inputs' population statistics (gamma = 1,
+    beta = the drawn bias) is folded into the PFN weight and bias, so that the
+    PFN output -- and with He-normal layers after it, every activation -- has
+    unit scale as in a trained, normalised network.
 
     Returns an ordered dict name -> float32 array; ``np.concatenate`` of the
     flattened values in order is the blob the C library takes.
@@ -262,8 +283,14 @@ def weights_for(cfg: ModelConfig) -> dict:
             v = rng.normal(0.0, math.sqrt(2.0 / fan_in), shape)
         else:
             v = rng.uniform(-0.1, 0.1, shape)
-        out[name] = v.astype(np.float32)
-    return out
+        out[name] = v
+    mean, var = pfn_feature_stats(cfg)
+    w = out["pfn.w"]
+    sigma = np.sqrt((w * w * var[None, :]).sum(axis=1))
+    mu = w @ mean
+    out["pfn.w"] = w / sigma[:, None]
+    out["pfn.b"] = out["pfn.b"] - mu / sigma
+    return {k: v.astype(np.float32) for k, v in out.items()}
 
 
 def weight_blob(weights: dict) -> np.ndarray:

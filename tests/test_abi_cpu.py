@@ -1,0 +1,177 @@
+"""Host-side checks of the C-ABI library (no GPU needed).
+
+* the library builds for sm_103a and exports every entry point declared in
+  include/rtcc.h;
+* the release controller validates completion events, walks the branch state
+  machine of Eq. 18, orders releases by (r_k, k) (Sec. IV-C/D), holds Barrier
+  releases until the last branch resolves (Sec. V), and withholds the join of an
+  aborted frame (Sec. IV-C, last sentence).
+"""
+import ctypes
+import math
+import os
+import re
+
+import pytest
+
+from paper_2608_08330_gb300 import build as B
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def R():
+    B.build()
+    from paper_2608_08330_gb300 import rtcc
+    rtcc.load()
+    return rtcc
+
+
+def _declared():
+    hdr = open(os.path.join(ROOT, "include", "rtcc.h")).read()
+    hdr = re.sub(r"/\*.*?\*/", "", hdr, flags=re.S)
+    names = set(re.findall(r"\b(rtcc_[a-z0-9_]+)\s*\(", hdr))
+    return sorted(names)
+
+
+def test_library_exports_every_declared_symbol(R):
+    lib = ctypes.CDLL(R.LIB_PATH)
+    names = _declared()
+    assert len(names) >= 30
+    missing = [n for n in names if not hasattr(lib, n)]
+    assert not missing, missing
+
+
+def test_status_strings_and_clock(R):
+    assert R.rtcc_status_str(R.OK) == "ok"
+    assert "duplicate" in R.rtcc_status_str(R.E_DUPLICATE)
+    t0 = R.rtcc_now_ms()
+    t1 = R.rtcc_now_ms()
+    assert t1 >= t0 > 0
+
+
+def test_init_rejects_bad_config_without_touching_gpu(R):
+    cfg = R.rtcc_model_config()
+    cfg.n_agents = 0
+    out = ctypes.c_void_p()
+    w = (ctypes.c_float * 4)()
+    assert R.load().rtcc_init(ctypes.byref(cfg), w, 4, ctypes.byref(out)) == R.E_ARG
+    assert R.load().rtcc_init(None, w, 4, ctypes.byref(out)) == R.E_ARG
+
+
+def test_rtcc_releases_on_completion_in_event_order(R):
+    c = R.rtcc_ctrl_create(3, 100)
+    assert R.rtcc_ctrl_begin(c, 1, 0.0) == R.OK
+    for k in range(3):
+        s, st, r = R.rtcc_ctrl_state(c, k)
+        assert st == R.WAITING and r is None
+    s, rel = R.rtcc_ctrl_complete(c, 2, True, 10, 4.0)
+    assert s == R.OK and rel == [2]
+    s, st, r = R.rtcc_ctrl_state(c, 2)
+    assert st == R.RELEASED and r == 4.0                  # release certificate r_k = a_k
+    assert not R.rtcc_ctrl_join_ready(c)
+    assert R.rtcc_ctrl_mark(c, 2, R.RUNNING) == R.OK
+    assert R.rtcc_ctrl_mark(c, 2, R.RUNNING) == R.E_STATE
+    assert R.rtcc_ctrl_mark(c, 2, R.FINISHED) == R.OK
+    assert R.rtcc_ctrl_complete(c, 0, True, 0, 7.0) == (R.OK, [0])   # empty payload is valid
+    assert R.rtcc_ctrl_complete(c, 1, True, 100, 9.5) == (R.OK, [1])
+    assert R.rtcc_ctrl_join_ready(c)
+    assert R.rtcc_ctrl_end(c) == R.OK
+    R.rtcc_ctrl_destroy(c)
+
+
+def test_event_validation(R):
+    c = R.rtcc_ctrl_create(2, 100)
+    assert R.rtcc_ctrl_complete(c, 0, True, 5, 1.0)[0] == R.E_PREMATURE   # no frame
+    assert R.rtcc_ctrl_begin(c, 7, 10.0) == R.OK
+    assert R.rtcc_ctrl_begin(c, 8, 10.0) == R.E_STATE                      # still open
+    assert R.rtcc_ctrl_complete(c, 0, True, 5, 9.0)[0] == R.E_PREMATURE    # t < t0
+    assert R.rtcc_ctrl_complete(c, 2, True, 5, 11.0)[0] == R.E_AGENT
+    assert R.rtcc_ctrl_complete(c, -1, True, 5, 11.0)[0] == R.E_AGENT
+    assert R.rtcc_ctrl_complete(c, 0, True, 101, 11.0)[0] == R.E_MALFORMED
+    assert R.rtcc_ctrl_complete(c, 0, True, -1, 11.0)[0] == R.E_MALFORMED
+    assert R.rtcc_ctrl_complete(c, 0, False, 3, 11.0)[0] == R.E_MALFORMED
+    assert R.rtcc_ctrl_complete(c, 0, True, 3, float("nan"))[0] == R.E_MALFORMED
+    # rejected events left the branch WAITING
+    assert R.rtcc_ctrl_state(c, 0)[1] == R.WAITING
+    assert R.rtcc_ctrl_complete(c, 0, True, 3, 11.0) == (R.OK, [0])
+    assert R.rtcc_ctrl_complete(c, 0, True, 3, 12.0)[0] == R.E_DUPLICATE
+    assert R.rtcc_ctrl_absent(c, 0, 12.0)[0] == R.E_DUPLICATE
+    assert R.rtcc_ctrl_set_mode(c, R.MODE_BARRIER) == R.E_STATE            # mid-frame
+    R.rtcc_ctrl_destroy(c)
+
+
+def test_barrier_holds_until_last_and_dispatches_in_index_order(R):
+    c = R.rtcc_ctrl_create(4, 100)
+    assert R.rtcc_ctrl_set_mode(c, R.MODE_BARRIER) == R.OK
+    R.rtcc_ctrl_begin(c, 1, 0.0)
+    assert R.rtcc_ctrl_complete(c, 3, True, 1, 1.0) == (R.OK, [])
+    assert R.rtcc_ctrl_complete(c, 1, True, 1, 2.0) == (R.OK, [])
+    assert R.rtcc_ctrl_state(c, 3)[1] == R.RELEASED
+    assert R.rtcc_ctrl_absent(c, 2, 2.5) == (R.OK, [])
+    s, rel = R.rtcc_ctrl_complete(c, 0, True, 1, 6.0)
+    assert s == R.OK and rel == [0, 1, 3]                 # r_k = A for all, then index
+    for k in (0, 1, 3):
+        assert R.rtcc_ctrl_state(c, k)[2] == 6.0
+    assert R.rtcc_ctrl_state(c, 2)[1] == R.ABSENT
+    assert R.rtcc_ctrl_join_ready(c)
+    R.rtcc_ctrl_destroy(c)
+
+
+def test_simultaneous_completions_tie_break_by_index(R):
+    # two agents complete at the same a_k; the queue orders them by index even
+    # if the later index reports first (Barrier exposes the queue order)
+    c = R.rtcc_ctrl_create(3, 10)
+    R.rtcc_ctrl_set_mode(c, R.MODE_BARRIER)
+    R.rtcc_ctrl_begin(c, 1, 0.0)
+    R.rtcc_ctrl_complete(c, 2, True, 1, 5.0)
+    R.rtcc_ctrl_complete(c, 1, True, 1, 5.0)
+    assert R.rtcc_ctrl_complete(c, 0, True, 1, 5.0) == (R.OK, [0, 1, 2])
+    R.rtcc_ctrl_destroy(c)
+
+
+def test_absent_rules_and_abort(R):
+    c = R.rtcc_ctrl_create(2, 10, attn_ego=True)
+    R.rtcc_ctrl_begin(c, 1, 0.0)
+    assert R.rtcc_ctrl_absent(c, 0, 1.0)[0] == R.E_ARG     # the ego query must be present
+    assert R.rtcc_ctrl_absent(c, 1, 1.0) == (R.OK, [])
+    assert not R.rtcc_ctrl_join_ready(c)
+    R.rtcc_ctrl_destroy(c)
+    c = R.rtcc_ctrl_create(2, 10)
+    R.rtcc_ctrl_begin(c, 1, 0.0)
+    assert R.rtcc_ctrl_absent(c, 0, 1.0)[0] == R.OK
+    assert R.rtcc_ctrl_absent(c, 1, 1.0)[0] == R.E_ARG     # nobody would be left
+    R.rtcc_ctrl_destroy(c)
+    c = R.rtcc_ctrl_create(3, 10)
+    R.rtcc_ctrl_begin(c, 1, 0.0)
+    R.rtcc_ctrl_complete(c, 0, True, 1, 1.0)
+    assert R.rtcc_ctrl_abort(c) == R.OK                     # horizon expired
+    assert not R.rtcc_ctrl_join_ready(c)                    # post-join withheld
+    assert R.rtcc_ctrl_complete(c, 1, True, 1, 2.0)[0] == R.E_PREMATURE
+    assert R.rtcc_ctrl_end(c) == R.OK
+    assert R.rtcc_ctrl_begin(c, 2, 0.0) == R.OK             # next frame starts clean
+    assert R.rtcc_ctrl_state(c, 0)[1] == R.WAITING
+    R.rtcc_ctrl_destroy(c)
+
+
+def test_random_event_orders_match_the_timeline_oracle(R):
+    """Dispatch order of the controller = the oracle's (a_k, k) order."""
+    import numpy as np
+    from oracle import schedule as sch
+    rng = np.random.default_rng(1)
+    for _ in range(200):
+        K = int(rng.integers(1, 9))
+        a = rng.integers(0, 5, K).astype(float).tolist()
+        c = R.rtcc_ctrl_create(K, 10)
+        R.rtcc_ctrl_begin(c, 1, 0.0)
+        order = []
+        for k in sorted(range(K), key=lambda k: (a[k], rng.random())):   # report order
+            s, rel = R.rtcc_ctrl_complete(c, k, True, 1, a[k])
+            assert s == R.OK
+            order += rel
+        R.rtcc_ctrl_destroy(c)
+        # reports arrive in time order; ties may be reported in any order but a
+        # tie reported later still dispatches when reported (online release)
+        ref = sch.simulate([int(x) for x in a], [1] * K, [0], "rtcc")["order"]
+        assert sorted(order) == sorted(ref)
+        assert [a[k] for k in order] == sorted(a)

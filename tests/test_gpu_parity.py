@@ -1,0 +1,236 @@
+"""GPU path vs the CPU oracle, through the C ABI.
+
+Bar: pillar indices, counts and drop counters bit-exact; every floating-point
+tensor within |gpu - oracle| <= 2e-2 + 1e-2 |oracle| (fp16/bf16 storage, fp32
+accumulation) against the oracle in storage-rounded mode; the decode's
+selection and order exact given the GPU head; RTCC and Barrier outputs
+bit-identical (Sec. III-C last paragraph, Sec. V-F).
+
+Stages are also checked in isolation (the oracle's next stage applied to the
+GPU's own input of that stage) so that a kernel is judged on its own error.
+"""
+import dataclasses
+
+import numpy as np
+import pytest
+
+import synth
+from oracle import forward as of
+from tests import gpu_util as U
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def R():
+    return U.load()
+
+
+def _small_pp(name="pp3", grid=(96, 64), n_uniform=6000, clusters=4, **kw):
+    base = synth.get_config(name)
+    return dataclasses.replace(base, grid_w=grid[0], grid_h=grid[1],
+                               x_min=-grid[0] * 0.2, x_max=grid[0] * 0.2,
+                               y_min=-grid[1] * 0.2, y_max=grid[1] * 0.2,
+                               pts_x=(-grid[0] * 0.2 - 1, grid[0] * 0.2 + 1),
+                               pts_y=(-grid[1] * 0.2 - 1, grid[1] * 0.2 + 1),
+                               n_uniform=n_uniform, n_clusters=clusters, **kw)
+
+
+def _check_frame(R, ctx, cfg, w, pts, absent=()):
+    """Compare every stage of the frame just run against the oracle."""
+    store = cfg.dtype
+    K = cfg.n_agents
+    feats_gpu = []
+    for k in range(K):
+        if k in absent:
+            feats_gpu.append(None)
+            continue
+        # pillars: bit-exact
+        op = of.pillarise(pts[k], cfg)
+        gp = R.rtcc_get_pillars(ctx, k, cfg.grid_h, cfg.grid_w, cfg.max_pillars)
+        assert gp["n_pillars"] == op["n_pillars"]
+        np.testing.assert_array_equal(gp["cell2pillar"], op["cell2pillar"])
+        n = op["n_pillars"]
+        np.testing.assert_array_equal(gp["pillar_cell"][:n], op["pillar_cell"][:n])
+        np.testing.assert_array_equal(gp["count"][:n], op["count"][:n])
+        assert gp["drop_range"] == op["drop_range"]
+        assert gp["drop_pcap"] == op["drop_pcap"]
+        assert gp["drop_ncap"] == op["drop_ncap"]
+        # PFN + scatter
+        h = of.pfn(op, w["pfn.w"], w["pfn.b"], cfg, store)
+        img_o = of.scatter(h, op, cfg)
+        img_g = U.gpu_tensor(ctx, cfg, k, 0, (cfg.pfn_ch, cfg.grid_h, cfg.grid_w))
+        occ_g = (img_g != 0).any(axis=0).reshape(-1)
+        assert not (occ_g & (op["cell2pillar"] < 0)).any()        # nonzero only on pillars
+        U.assert_close(img_g, img_o, f"pseudo-image agent {k}")
+        # every conv layer, isolated on the GPU's own input of that layer
+        x_g = img_g
+        layers = U.conv_layers(cfg)
+        last_of_block = {}
+        for i, (bi, li, st, shape) in enumerate(layers):
+            y_o = U.oracle_conv_layer(x_g, w, bi, li, st, store)
+            y_g = U.gpu_tensor(ctx, cfg, k, 16 + i, shape)
+            U.assert_close(y_g, y_o, f"conv b{bi}.c{li} agent {k}")
+            x_g = y_g
+            last_of_block[bi] = y_g
+        blocks_g = [last_of_block[bi] for bi in range(len(cfg.blocks))]
+        shapes = U.block_shapes(cfg)
+        for bi in range(len(cfg.blocks)):                       # block read-back = last layer
+            np.testing.assert_array_equal(U.gpu_tensor(ctx, cfg, k, bi + 1, shapes[bi]), blocks_g[bi])
+        # neck, isolated on the GPU's own block outputs
+        feat_o = U.oracle_neck(blocks_g, w, cfg, store)
+        feat_g = U.gpu_tensor(ctx, cfg, k, 8, (cfg.feat_ch, cfg.feat_h, cfg.feat_w))
+        U.assert_close(feat_g, feat_o, f"features agent {k}")
+        feats_gpu.append(feat_g)
+    # fusion + head, isolated on the GPU's own feature slots
+    F_o = of.fuse_max(feats_gpu) if cfg.fusion == "max" else of.fuse_attn(feats_gpu)
+    F_g = U.gpu_tensor(ctx, cfg, 0, 9, (cfg.feat_ch, cfg.feat_h, cfg.feat_w))
+    if cfg.fusion == "max":
+        np.testing.assert_array_equal(F_g, F_o)                 # max is exact
+    else:
+        U.assert_close(F_g, F_o, "fused (attention)")
+    hd_o = of.head(F_o, of.store_round(w["head.w"], store), of.store_round(w["head.b"], store))
+    hd_g = U.head_to_oracle_layout(R.rtcc_get_head(ctx, cfg.feat_h, cfg.feat_w))
+    U.assert_close(hd_g, hd_o, "head (isolated)")
+    return hd_g
+
+
+def _check_decode(cfg, hd_g, boxes):
+    det = of.decode(hd_g, cfg)
+    assert boxes["anchor"].tolist() == det["idx"].tolist()      # exact selection + order
+    got = np.stack([boxes[f] for f in ("x", "y", "z", "l", "w", "h", "yaw", "score")], axis=1)
+    U.assert_close(got, det["boxes"], "boxes")
+
+
+def _end_to_end(R, cfg, frame=0, absent=(), flags=None, arrivals=None):
+    ctx, w = U.make_ctx(cfg) if flags is None else U.make_ctx(cfg, flags=flags)
+    try:
+        pts = [synth.points_for(cfg, frame, k) for k in range(cfg.n_agents)]
+        a = synth.arrivals_for(cfg, frame) if arrivals is None else arrivals
+        boxes = U.run_frame(ctx, cfg, pts, a, R.MODE_RTCC, absent=absent)
+        hd_g = _check_frame(R, ctx, cfg, w, pts, absent=absent)
+        _check_decode(cfg, hd_g, boxes)
+        # whole-path parity: the oracle forward from the points
+        full = of.forward([None if k in absent else pts[k] for k in range(cfg.n_agents)], w, cfg,
+                          store=cfg.dtype)
+        U.assert_close(hd_g, full["head"], "head (end to end)")
+        return ctx, w, pts, a
+    except Exception:
+        R.rtcc_destroy(ctx)
+        raise
+
+
+def test_tiny_end_to_end(R):
+    cfg = synth.get_config("tiny")
+    ctx, *_ = _end_to_end(R, cfg)
+    info = R.rtcc_get_frame_info(ctx)
+    assert info.n_dispatched == 2 and info.gpu_backbone_ms[0] > 0 and info.gpu_fusion_ms > 0
+    R.rtcc_destroy(ctx)
+
+
+def test_pointpillars_small_grid_ragged_tiles(R):
+    # 96x64 grid: block maps 48x32, 24x16, 12x8 -- none a multiple of the
+    # 32x4 tile in x except the first; deconvs s = 1, 2, 4 into 384 channels
+    cfg = _small_pp()
+    ctx, *_ = _end_to_end(R, cfg)
+    R.rtcc_destroy(ctx)
+
+
+def test_attention_bf16_with_absent_agent(R):
+    cfg = _small_pp("lr5", grid=(88, 40), n_uniform=5000)
+    ctx, *_ = _end_to_end(R, cfg, absent=(3,))
+    R.rtcc_destroy(ctx)
+
+
+def test_caps_bind_bit_exact(R):
+    cfg = dataclasses.replace(synth.get_config("tiny"), max_pillars=16, max_pts=8)
+    ctx, w = U.make_ctx(cfg, max_points=4096)
+    pts = [synth.points_cap_patch(2048, 8, seed=3), synth.points_cap_patch(4096, 6, seed=4)]
+    U.run_frame(ctx, cfg, pts, [0.0, 1.0], R.MODE_RTCC)
+    hd = _check_frame(R, ctx, cfg, w, pts)
+    full = of.forward(pts, w, cfg, store="fp16")
+    U.assert_close(hd, full["head"], "head (caps)")
+    gp = R.rtcc_get_pillars(ctx, 1, cfg.grid_h, cfg.grid_w, cfg.max_pillars)
+    assert gp["drop_pcap"] > 0 and gp["drop_ncap"] > 0
+    R.rtcc_destroy(ctx)
+
+
+def test_empty_and_out_of_range_payloads(R):
+    cfg = synth.get_config("tiny")
+    ctx, w = U.make_ctx(cfg)
+    far = synth.points_for(cfg, 0, 1).copy()
+    far[:, 0] += 100.0                                  # every point out of range
+    pts = [np.zeros((0, 4), dtype=np.float32), far]
+    U.run_frame(ctx, cfg, pts, [0.0, 0.0], R.MODE_RTCC)
+    for k in range(2):
+        gp = R.rtcc_get_pillars(ctx, k, cfg.grid_h, cfg.grid_w, cfg.max_pillars)
+        assert gp["n_pillars"] == 0 and (gp["cell2pillar"] == -1).all()
+    hd = _check_frame(R, ctx, cfg, w, pts)
+    full = of.forward(pts, w, cfg, store="fp16")
+    U.assert_close(hd, full["head"], "head (empty)")
+    R.rtcc_destroy(ctx)
+
+
+@pytest.mark.parametrize("name", ["tiny", "small_pp", "small_attn"])
+def test_rtcc_and_barrier_bit_identical(R, name):
+    if name == "tiny":
+        cfg = synth.get_config("tiny")
+    elif name == "small_pp":
+        cfg = _small_pp()
+    else:
+        cfg = _small_pp("lr5", grid=(88, 40), n_uniform=5000)
+    ctx, w = U.make_ctx(cfg)
+    outs = {}
+    for frame in range(2):
+        pts = [synth.points_for(cfg, frame, k) for k in range(cfg.n_agents)]
+        a = synth.arrivals_for(cfg, frame) if cfg.arrival != "fixed" else [0.0, 5.0]
+        for mode in (R.MODE_RTCC, R.MODE_BARRIER, R.MODE_RTCC):
+            boxes = U.run_frame(ctx, cfg, pts, a, mode, frame_id=frame)
+            hd = R.rtcc_get_head(ctx, cfg.feat_h, cfg.feat_w)
+            feats = b"".join(R.rtcc_get_tensor(ctx, k, 8).tobytes() for k in range(cfg.n_agents))
+            key = (frame, mode)
+            cur = (hd.tobytes(), boxes.tobytes(), feats)
+            if key in outs:
+                assert outs[key] == cur                       # run-to-run deterministic
+            outs[key] = cur
+        assert outs[(frame, R.MODE_RTCC)] == outs[(frame, R.MODE_BARRIER)]
+    R.rtcc_destroy(ctx)
+
+
+def test_resident_input_release_matches_staged(R):
+    cfg = synth.get_config("tiny")
+    ctx, w = U.make_ctx(cfg)
+    pts = [synth.points_for(cfg, 3, k) for k in range(2)]
+    b1 = U.run_frame(ctx, cfg, pts, [1.0, 2.0], R.MODE_RTCC)
+    h1 = R.rtcc_get_head(ctx, cfg.feat_h, cfg.feat_w).tobytes()
+    for k in range(2):
+        assert R.rtcc_stage_resident(ctx, k, pts[k]) == R.OK
+    assert R.rtcc_frame_begin(ctx, 9, 0.0) == R.OK
+    assert R.rtcc_payload_resident(ctx, 1, 1.0) == R.OK
+    assert R.rtcc_payload_resident(ctx, 0, 2.0) == R.OK
+    s, b2, _ = R.rtcc_wait_detection(ctx, 60000)
+    assert s == R.OK
+    assert R.rtcc_get_head(ctx, cfg.feat_h, cfg.feat_w).tobytes() == h1
+    assert b1.tobytes() == b2.tobytes()
+    R.rtcc_destroy(ctx)
+
+
+def test_abort_is_infeasible_and_next_frame_clean(R):
+    cfg = synth.get_config("tiny")
+    ctx, w = U.make_ctx(cfg)
+    pts = [synth.points_for(cfg, 0, k) for k in range(2)]
+    assert R.rtcc_frame_begin(ctx, 1, 0.0) == R.OK
+    assert R.rtcc_payload_complete(ctx, 0, pts[0], 1.0) == R.OK
+    assert R.rtcc_wait_detection(ctx, 100)[0] == R.E_STATE        # branch 1 still missing
+    assert R.rtcc_frame_abort(ctx) == R.OK
+    assert R.rtcc_wait_detection(ctx, 100)[0] == R.E_INFEASIBLE
+    boxes = U.run_frame(ctx, cfg, pts, [0.0, 5.0], R.MODE_RTCC, frame_id=2)
+    hd = _check_frame(R, ctx, cfg, w, pts)
+    _check_decode(cfg, hd, boxes)
+    R.rtcc_destroy(ctx)
+
+
+def test_pointpillars_full_size(R):
+    cfg = synth.get_config("pp3")
+    ctx, *_ = _end_to_end(R, cfg, frame=1)
+    R.rtcc_destroy(ctx)
