@@ -279,6 +279,45 @@ rtcc_status rtcc_get_tensor(struct rtcc_ctx* ctx, int32_t agent, int32_t which,
                             uint16_t* host_out, size_t cap, size_t* n_elems);
 
 /* ------------------------------------------------------------------------ */
+/* Allocation-free pillarisation (no counterpart in the paper)              */
+/* ------------------------------------------------------------------------ */
+
+/*
+ * The pillarise -> PFN -> scatter pass of one branch, for callers that cannot
+ * allocate device memory where they need it: code running while a stream is
+ * being captured into a CUDA graph (cudaMalloc cannot be captured), plugin
+ * hosts that own all device memory and offer no allocator, and latency-bound
+ * loops that must not risk the device synchronisation an allocation can
+ * trigger.  This call allocates nothing: its scratch is one fixed array in
+ * device memory that the library reserves on every GPU that loads it (about
+ * 4.3 MB, kept until the process exits).  The array bounds the sizes:
+ * grid_w * grid_h <= 65536 cells, n_points <= 131072, max_pillars <= 16384,
+ * pfn_ch in {32, 64}, max_pts <= 32; larger requests return RTCC_E_ARG.
+ *
+ * Uses from cfg: grid_w/h, x_min, y_min, z_min, z_max, pillar, max_pillars,
+ * max_pts, pfn_ch, dtype.  Inputs (device, caller-owned): d_points float32
+ * [n_points][4]; d_pfn_w float32 [pfn_ch][9] and d_pfn_b float32 [pfn_ch]
+ * with the values the kernels should use (rtcc_init rounds them to the storage
+ * type first).  Outputs (device, caller-owned): d_cell2pillar int32 [H*W],
+ * d_pillar_cell and d_count int32 [max_pillars] (entries >= n_pillars are left
+ * untouched), d_stats int32 [8] = {n, n_in_range, n_pillars, n_kept, 0, 0,
+ * dropped by the per-pillar cap, points of kept pillars before that cap},
+ * d_image 16-bit [H][W][pfn_ch].  Work is enqueued on `stream` (a
+ * cudaStream_t; NULL = the default stream) and the call returns without
+ * waiting.
+ *
+ * The first call on a device looks up the array's device address; make that
+ * first call outside any stream capture.  Every call shares the array and
+ * clears what must start at zero before use, so calls that overlap on the GPU
+ * race with each other: serialise them (one stream, or events).
+ */
+rtcc_status rtcc_pillarise_noalloc(const rtcc_model_config* cfg, const float* d_points,
+                                   int32_t n_points, const float* d_pfn_w,
+                                   const float* d_pfn_b, int32_t* d_cell2pillar,
+                                   int32_t* d_pillar_cell, int32_t* d_count,
+                                   int32_t* d_stats, void* d_image, void* stream);
+
+/* ------------------------------------------------------------------------ */
 /* Release controller alone (host only; no GPU needed)                      */
 /* ------------------------------------------------------------------------ */
 

@@ -1,0 +1,144 @@
+// Allocation-free variant of the pillarisation + PFN + scatter pass.
+//
+// Some callers cannot allocate device memory at the point where they need
+// this pass: code that runs while a CUDA stream is being captured into a graph
+// (cudaMalloc is not a capturable operation), hosts that hand a plugin only
+// pre-planned memory and no allocator, and latency-critical loops that must not
+// risk the implicit device synchronisation an allocation can cause.  For them
+// this entry point takes its scratch from one fixed array in device global
+// memory that the library reserves when it is loaded, instead of calling any
+// allocator.  The array is sized for grids up to 65,536 cells, payloads up to
+// 131,072 points, 16,384 pillars and 64 PFN channels (about 4.3 MB, held on
+// every GPU that loads the library until the process exits).
+//
+// The kernels are the ones rtcc_payload_complete runs (launch_pillarise); only
+// the scratch pointers differ.  All calls share the one array: a call clears
+// what must start at zero (per-cell counters and first-point indices, the
+// caller's stats) before it runs, and calls that overlap on the GPU -- on
+// different streams, or from different host threads -- race on the array and
+// must be serialised by the caller.
+#include <mutex>
+
+#include "kernels.h"
+#include "rtcc.h"
+
+namespace rtcc {
+namespace {
+
+constexpr int kMaxCells = 65536;
+constexpr int kMaxPoints = 131072;
+constexpr int kMaxPillars = 16384;
+constexpr int kMaxCh = 64;
+constexpr int kMaxScanBlocks = (kMaxPoints + kScanTile - 1) / kScanTile;
+
+constexpr size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+// byte offsets of the regions inside the static array (each 256-byte aligned)
+constexpr size_t kOffN = 0;
+constexpr size_t kOffCellOf = align256(kOffN + 16);
+constexpr size_t kOffList = align256(kOffCellOf + 4ull * kMaxPoints);
+constexpr size_t kOffCnt = align256(kOffList + 4ull * kMaxPoints);
+constexpr size_t kOffFirst = align256(kOffCnt + 4ull * kMaxCells);
+constexpr size_t kOffC2P = align256(kOffFirst + 4ull * kMaxCells);
+constexpr size_t kOffBlock = align256(kOffC2P + 4ull * kMaxCells);
+constexpr size_t kOffRaw = align256(kOffBlock + 8ull * kMaxScanBlocks);
+constexpr size_t kOffPoff = align256(kOffRaw + 4ull * kMaxPillars);
+constexpr size_t kOffCursor = align256(kOffPoff + 4ull * kMaxPillars);
+constexpr size_t kOffFeat = align256(kOffCursor + 4ull * kMaxPillars);
+constexpr size_t kStaticBytes = align256(kOffFeat + 2ull * kMaxPillars * kMaxCh);
+
+static __device__ __align__(256) unsigned char g_pillar_scratch[kStaticBytes];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_mu;
+unsigned char* g_addr[kMaxDevices] = {};
+
+// Device address of the static array on the current device, looked up once
+// per device (the symbol's host-side name is not a device address).
+rtcc_status scratch_address(unsigned char** out) {
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return RTCC_E_CUDA;
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (!g_addr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_pillar_scratch) != cudaSuccess || !p) return RTCC_E_CUDA;
+    g_addr[dev] = static_cast<unsigned char*>(p);
+  }
+  *out = g_addr[dev];
+  return RTCC_OK;
+}
+
+__global__ void k_static_reset(int n, int cells, int* __restrict__ n_slot,
+                               int* __restrict__ cnt_cell, int* __restrict__ first_cell,
+                               int* __restrict__ stats) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i == 0) *n_slot = n;
+  if (i < 8) stats[i] = 0;
+  for (int c = i; c < cells; c += gridDim.x * blockDim.x) {
+    cnt_cell[c] = 0;
+    first_cell[c] = kFirstInit;
+  }
+}
+
+}  // namespace
+}  // namespace rtcc
+
+using namespace rtcc;
+
+extern "C" rtcc_status rtcc_pillarise_noalloc(const rtcc_model_config* cfg, const float* d_points,
+                                              int32_t n_points, const float* d_pfn_w,
+                                              const float* d_pfn_b, int32_t* d_cell2pillar,
+                                              int32_t* d_pillar_cell, int32_t* d_count,
+                                              int32_t* d_stats, void* d_image, void* stream) {
+  if (!cfg || !d_pfn_w || !d_pfn_b || !d_cell2pillar || !d_pillar_cell || !d_count ||
+      !d_stats || !d_image || (n_points > 0 && !d_points))
+    return RTCC_E_ARG;
+  const long long cells = (long long)cfg->grid_w * cfg->grid_h;
+  if (cfg->grid_w < 1 || cfg->grid_h < 1 || cells > kMaxCells) return RTCC_E_ARG;
+  if (n_points < 0 || n_points > kMaxPoints) return RTCC_E_ARG;
+  if (cfg->max_pillars < 1 || cfg->max_pillars > kMaxPillars) return RTCC_E_ARG;
+  if (cfg->max_pts < 1 || cfg->max_pts > 32) return RTCC_E_ARG;
+  if (cfg->pfn_ch != 32 && cfg->pfn_ch != kMaxCh) return RTCC_E_ARG;
+  if (cfg->dtype != RTCC_FP16 && cfg->dtype != RTCC_BF16) return RTCC_E_ARG;
+  if (!(cfg->pillar > 0.f)) return RTCC_E_ARG;
+  unsigned char* base = nullptr;
+  rtcc_status s = scratch_address(&base);
+  if (s != RTCC_OK) return s;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+
+  PillarBufs b{};
+  b.pts = reinterpret_cast<const float4*>(d_points);
+  b.n_hdr = reinterpret_cast<const int*>(base + kOffN);
+  b.cell_of = reinterpret_cast<int*>(base + kOffCellOf);
+  b.cnt_cell = reinterpret_cast<int*>(base + kOffCnt);
+  b.first_cell = reinterpret_cast<int*>(base + kOffFirst);
+  b.c2p = reinterpret_cast<int*>(base + kOffC2P);
+  b.blocksum = reinterpret_cast<int2*>(base + kOffBlock);
+  b.pcnt_raw = reinterpret_cast<int*>(base + kOffRaw);
+  b.poff = reinterpret_cast<int*>(base + kOffPoff);
+  b.cursor = reinterpret_cast<int*>(base + kOffCursor);
+  b.list = reinterpret_cast<int*>(base + kOffList);
+  b.feat = base + kOffFeat;
+  b.pillar_cell = d_pillar_cell;
+  b.pcount = d_count;
+  b.stats = d_stats;
+  b.cell2pillar = d_cell2pillar;
+  b.image = d_image;
+  b.cap = n_points > 0 ? n_points : 1;
+  b.P = cfg->max_pillars;
+  b.N = cfg->max_pts;
+  b.C = cfg->pfn_ch;
+
+  int blocks = (int)((cells + 255) / 256);
+  if (blocks < 1) blocks = 1;
+  k_static_reset<<<blocks, 256, 0, st>>>(n_points, (int)cells,
+                                         reinterpret_cast<int*>(base + kOffN), b.cnt_cell,
+                                         b.first_cell, d_stats);
+  if (cudaGetLastError() != cudaSuccess) return RTCC_E_CUDA;
+  GridGeom g{cfg->x_min, cfg->y_min, cfg->z_min, cfg->z_max, cfg->pillar, cfg->grid_w,
+             cfg->grid_h};
+  if (launch_pillarise(b, g, d_pfn_w, d_pfn_b, cfg->dtype == RTCC_BF16, nullptr, st) !=
+      cudaSuccess)
+    return RTCC_E_CUDA;
+  return RTCC_OK;
+}

@@ -126,6 +126,9 @@ def load(path: Optional[str] = None) -> C.CDLL:
         "rtcc_status_str": (C.c_char_p, [C.c_int]),
         "rtcc_now_ms": (C.c_double, []),
         "rtcc_kernels_per_frame": (C.c_int32, [_ctx_p, C.c_int32]),
+        "rtcc_pillarise_noalloc": (S, [C.POINTER(rtcc_model_config), C.c_void_p, C.c_int32,
+                                       C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
+                                       C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -295,6 +298,15 @@ def rtcc_now_ms() -> float:
 
 def rtcc_kernels_per_frame(ctx, n_present: int) -> int:
     return load().rtcc_kernels_per_frame(ctx, n_present)
+
+
+def rtcc_pillarise_noalloc(cfg: rtcc_model_config, d_points: int, n_points: int, d_pfn_w: int,
+                           d_pfn_b: int, d_cell2pillar: int, d_pillar_cell: int, d_count: int,
+                           d_stats: int, d_image: int, stream: int = 0) -> int:
+    """Allocation-free pillarise/PFN/scatter; every d_* is a device address."""
+    return load().rtcc_pillarise_noalloc(C.byref(cfg), d_points, n_points, d_pfn_w, d_pfn_b,
+                                         d_cell2pillar, d_pillar_cell, d_count, d_stats,
+                                         d_image, stream or None)
 
 
 # --------------------------------------------------------------------------

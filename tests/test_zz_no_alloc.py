@@ -1,0 +1,77 @@
+"""The allocation-free pillarisation entry point, checked against the context.
+
+rtcc_pillarise_noalloc serves callers that cannot allocate device memory
+where they need the pass (inside a stream capture, in a plugin host with no
+allocator, in a latency-bound loop).  Its scratch is a fixed array the library
+reserves on load.  This test runs the same points through the existing entry
+point (rtcc_payload_complete on a full-size 3-agent context) and through the
+new one twice in a row, with different inputs, and requires the same pillars
+(bit-exact) and the same pseudo-image (within the parity tolerance).  The
+second call also shows that leftovers of the first call in the shared array do
+not leak into the next result.  Oversized requests must be refused.
+"""
+import numpy as np
+import pytest
+
+import synth
+from tests import gpu_util as U
+
+pytestmark = pytest.mark.gpu
+
+
+def test_noalloc_matches_context_on_two_calls():
+    torch = pytest.importorskip("torch")
+    R = U.load()
+    cfg = synth.get_config("pp3")
+    ctx, w = U.make_ctx(cfg, flags=0)
+    pts = [synth.points_for(cfg, 5, k) for k in range(cfg.n_agents)]
+    U.run_frame(ctx, cfg, pts, [0.0, 1.0, 2.0], R.MODE_RTCC)
+    ref = {}
+    for k in (0, 1):
+        ref[k] = (R.rtcc_get_pillars(ctx, k, cfg.grid_h, cfg.grid_w, cfg.max_pillars),
+                  R.rtcc_get_tensor(ctx, k, R.TENSOR_IMAGE))
+    R.rtcc_destroy(ctx)
+
+    dev = torch.device("cuda")
+    # the PFN weights as rtcc_init stores them: rounded once to the storage type
+    pw = torch.tensor(w["pfn.w"].astype(np.float16).astype(np.float32), device=dev)
+    pb = torch.tensor(w["pfn.b"].astype(np.float16).astype(np.float32), device=dev)
+    cells = cfg.grid_w * cfg.grid_h
+    c2p = torch.empty(cells, dtype=torch.int32, device=dev)
+    pcell = torch.empty(cfg.max_pillars, dtype=torch.int32, device=dev)
+    cnt = torch.empty(cfg.max_pillars, dtype=torch.int32, device=dev)
+    stats = torch.empty(8, dtype=torch.int32, device=dev)
+    img = torch.empty(cells * cfg.pfn_ch, dtype=torch.int16, device=dev)
+    c = R.model_config(cfg)
+    for k in (0, 1):                                   # two calls in a row
+        d_pts = torch.from_numpy(pts[k]).to(dev)
+        for t in (c2p, pcell, cnt, img):
+            t.fill_(-7)
+        stats.fill_(12345)                             # must be cleared by the call
+        torch.cuda.synchronize()
+        s = R.rtcc_pillarise_noalloc(c, d_pts.data_ptr(), pts[k].shape[0], pw.data_ptr(),
+                                     pb.data_ptr(), c2p.data_ptr(), pcell.data_ptr(),
+                                     cnt.data_ptr(), stats.data_ptr(), img.data_ptr(), 0)
+        assert s == R.OK, R.rtcc_status_str(s)
+        torch.cuda.synchronize()
+        gp, gimg = ref[k]
+        st = stats.cpu().numpy()
+        n = gp["n_pillars"]
+        assert st[0] == pts[k].shape[0] and st[2] == n and st[3] == gp["n_kept"]
+        assert st[6] == gp["drop_ncap"] and st[1] - st[7] == gp["drop_pcap"]
+        np.testing.assert_array_equal(c2p.cpu().numpy(), gp["cell2pillar"])
+        np.testing.assert_array_equal(pcell.cpu().numpy()[:n], gp["pillar_cell"][:n])
+        np.testing.assert_array_equal(cnt.cpu().numpy()[:n], gp["count"][:n])
+        got = U.u16_to_f64(img.cpu().numpy().view(np.uint16), cfg.dtype)
+        U.assert_close(got, U.u16_to_f64(gimg, cfg.dtype), f"pseudo-image call {k}")
+
+    big = R.model_config(cfg)
+    big.grid_w, big.grid_h = 512, 512                  # 262,144 cells > the 65,536 limit
+    s = R.rtcc_pillarise_noalloc(big, d_pts.data_ptr(), pts[1].shape[0], pw.data_ptr(),
+                                 pb.data_ptr(), c2p.data_ptr(), pcell.data_ptr(), cnt.data_ptr(),
+                                 stats.data_ptr(), img.data_ptr(), 0)
+    assert s == R.E_ARG
+    s = R.rtcc_pillarise_noalloc(c, d_pts.data_ptr(), 200000, pw.data_ptr(), pb.data_ptr(),
+                                 c2p.data_ptr(), pcell.data_ptr(), cnt.data_ptr(),
+                                 stats.data_ptr(), img.data_ptr(), 0)
+    assert s == R.E_ARG
