@@ -71,11 +71,36 @@ def conv_flops(cfg) -> float:
     return fl
 
 
+def layer_table(cfg):
+    """(name, algorithmic FLOPs) of every conv/deconv launch of one branch, in
+    the library's launch order (block convs, then the neck deconvs)."""
+    out = []
+    w, h, cin = cfg.grid_w, cfg.grid_h, cfg.pfn_ch
+    dims = []
+    for bi, (n, ch, st) in enumerate(cfg.blocks):
+        for li in range(n):
+            s = st if li == 0 else 1
+            w, h = w // s, h // s
+            out.append((f"b{bi}.c{li} 3x3 s{s} {cin}->{ch} @{w}x{h}", 2.0 * w * h * ch * 9 * cin))
+            cin = ch
+        dims.append((w, h, ch))
+    for bi, s in enumerate(cfg.up_strides):
+        bw, bh, bc = dims[bi]
+        out.append((f"up{bi} deconv k{s} {bc}->{cfg.up_ch} @{bw * s}x{bh * s}",
+                     2.0 * (bw * s) * (bh * s) * cfg.up_ch * bc))
+    return out
+
+
 def fusion_bytes(cfg, k_present: int) -> float:
     """Algorithmic bytes of the fusion+head kernel: each present slot read
     once (16-bit), the fp32 head map written once."""
     cells = cfg.feat_w * cfg.feat_h
     return float(k_present * cells * cfg.feat_ch * 2 + cells * 16 * 4)
+
+
+def _json_num(o):
+    """numpy scalars in the JSON line become plain numbers."""
+    return o.item() if hasattr(o, "item") else str(o)
 
 
 def pct(x, q):
@@ -202,7 +227,7 @@ def run_reference(args):
                          "sample": sample},
         "e2e": {"value": v, "unit": "ms", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
-    print(json.dumps(line), flush=True)
+    print(json.dumps(line, default=_json_num), flush=True)
     return 0
 
 
@@ -380,8 +405,39 @@ def run_ours(args):
                        f"in float64 NumPy; RTCC tail of each timed step's arrival trace on the "
                        f"single-stream timeline (Eqs. 20-22) with those service times")}
     R.rtcc_destroy(ctx)
+
+    # per-layer live times (a separate context whose graphs carry an event
+    # node between every conv launch; outside the timed region)
     if rank == 0:
-        print(json.dumps(line), flush=True)
+        pctx = R.rtcc_init(R.model_config(cfg, flags=R.FLAG_LAYER_TIMES), synth.weight_blob(w))
+        times = []
+        for f in range(4):
+            pts = frames[f % NF]
+            for k in range(K):
+                R.rtcc_stage_resident(pctx, k, pts[k])
+            R.rtcc_set_mode(pctx, R.MODE_RTCC)
+            R.rtcc_frame_begin(pctx, 9000 + f, 0.0)
+            for k in range(K):
+                R.rtcc_payload_resident(pctx, k, float(k))
+                torch.cuda.synchronize()       # branches one at a time, as in RTCC
+            R.rtcc_wait_detection(pctx, 10000)
+            if f > 0:
+                times += [R.rtcc_get_layer_times(pctx, k) for k in range(K)]
+        R.rtcc_destroy(pctx)
+        med = np.median(np.stack(times), axis=0)
+        rows = []
+        for (name, fl), t_ms in zip(layer_table(cfg), med):
+            t_ms = float(t_ms)
+            tf = fl / (t_ms * 1e-3) / 1e12
+            rows.append({"layer": name, "gflop": round(fl / 1e9, 4), "us": round(float(t_ms) * 1e3, 2),
+                         "tflops": round(tf, 1), "frac": round(tf / tflops_peak, 4)})
+        tot_us = float(np.sum(med)) * 1e3
+        line["layers"] = {"note": "each conv/deconv launch timed alone (event nodes between "
+                                  "launches remove the launch overlap of the served graph)",
+                          "sum_us": round(tot_us, 1),
+                          "tflops_isolated": round(flops / (tot_us * 1e-6) / 1e12, 1),
+                          "rows": rows}
+        print(json.dumps(line, default=_json_num), flush=True)
     if dist is not None:
         dist.destroy_process_group()
     return 0

@@ -90,6 +90,10 @@ typedef enum {
 #define RTCC_FLAG_KEEP_FUSED  2  /* also store the fused BEV map (parity)      */
 #define RTCC_FLAG_KEEP_LAYERS 4  /* give every conv layer its own output buffer
                                     so each can be read back (parity)         */
+#define RTCC_FLAG_LAYER_TIMES 8  /* record CUDA events between every conv/deconv
+                                    launch of a branch (per-layer timing; the
+                                    events also stop launch overlap between
+                                    layers, so use it to profile, not to serve) */
 
 /*
  * Network and workload description.  Supported: 1 <= n_agents <= 8;
@@ -245,6 +249,12 @@ rtcc_status rtcc_wait_detection(struct rtcc_ctx* ctx, int32_t timeout_ms,
 /* Timestamps and GPU spans of the last closed frame. */
 rtcc_status rtcc_get_frame_info(struct rtcc_ctx* ctx, rtcc_frame_info* info);
 
+/* Per-layer GPU times (ms) of `agent`'s conv and deconv launches in the last
+ * closed frame, in launch order (13 convs then 3 deconvs for the PointPillars
+ * backbone); needs RTCC_FLAG_LAYER_TIMES.  *n_out receives the layer count. */
+rtcc_status rtcc_get_layer_times(struct rtcc_ctx* ctx, int32_t agent, float* host_ms,
+                                 int32_t cap, int32_t* n_out);
+
 /* State z_k of a branch in the open (or last) frame, and its release time
  * r_k in the caller's timebase (NaN while WAITING). */
 rtcc_status rtcc_get_branch_state(struct rtcc_ctx* ctx, int32_t agent,
@@ -290,7 +300,7 @@ rtcc_status rtcc_get_tensor(struct rtcc_ctx* ctx, int32_t agent, int32_t which,
  * loops that must not risk the device synchronisation an allocation can
  * trigger.  This call allocates nothing: its scratch is one fixed array in
  * device memory that the library reserves on every GPU that loads it (about
- * 4.3 MB, kept until the process exits).  The array bounds the sizes:
+ * 5.2 MB, kept until the process exits).  The array bounds the sizes:
  * grid_w * grid_h <= 65536 cells, n_points <= 131072, max_pillars <= 16384,
  * pfn_ch in {32, 64}, max_pts <= 32; larger requests return RTCC_E_ARG.
  *

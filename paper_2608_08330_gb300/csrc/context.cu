@@ -46,10 +46,13 @@ struct Branch {
   int block_w[RTCC_MAX_BLOCKS] = {}, block_h[RTCC_MAX_BLOCKS] = {};
   void* feat = nullptr;            // agent-indexed feature slot [H'][W'][C_feat]
   std::vector<ConvLayer> layers;
+  float* splitk_ws = nullptr;      // split-K partials, shared by the branch's layers
+  int* splitk_cnt = nullptr;       // split-K per-tile arrival counters
   cudaStream_t st = nullptr;
   cudaGraphExec_t exec = nullptr;
   cudaEvent_t h2d_done = nullptr, done = nullptr;
   cudaEvent_t ev_start = nullptr, ev_bb0 = nullptr, ev_bb1 = nullptr, ev_end = nullptr;
+  std::vector<cudaEvent_t> layer_ev;   // RTCC_FLAG_LAYER_TIMES: before each layer + after last
   const float* pend_ptr = nullptr;
   int pend_n = 0;
   bool pend_resident = false;
@@ -81,7 +84,8 @@ struct rtcc_ctx {
   void** d_feat_ptrs = nullptr;
   float* head_out = nullptr;
   void* fused = nullptr;
-  unsigned long long* cand = nullptr;
+  uint32_t* keys = nullptr;           // decode key per anchor (padded)
+  uint32_t* hist0 = nullptr;          // decode level-0 histogram
   uint8_t* det_dev = nullptr;
   uint8_t* det_host = nullptr;        // pinned
   size_t det_bytes = 0;
@@ -310,6 +314,7 @@ rtcc_status build_branch(rtcc_ctx* c, int k) {
   RS(dalloc(c, &p.first_cell, (size_t)cells * 4));
   RS(dalloc(c, &p.c2p, (size_t)cells * 4));
   RS(dalloc(c, &p.blocksum, (size_t)scan_blocks(c->cap) * sizeof(int2)));
+  RS(dalloc(c, &p.items, (size_t)scan_blocks(c->cap) * kScanTile * sizeof(int2)));
   RS(dalloc(c, &p.pcnt_raw, (size_t)c->P * 4));
   RS(dalloc(c, &p.poff, (size_t)c->P * 4));
   RS(dalloc(c, &p.cursor, (size_t)c->P * 4));
@@ -355,7 +360,12 @@ rtcc_status build_branch(rtcc_ctx* c, int k) {
       L.gh = oh;
       L.ldc = co;
       L.choff = 0;
+      // 128-wide N tiles unless that leaves most SMs idle (the small, deep
+      // layers of blocks 2 and 3): then 64-wide tiles double the CTA count
+      const int m_tiles = ((ow + conv_tile_w() - 1) / conv_tile_w()) *
+                          ((oh + conv_tile_h() - 1) / conv_tile_h());
       L.bn = std::min(co, 128);
+      if (L.bn == 128 && m_tiles * (co / 128) < 120) L.bn = 64;
       L.bk = (cin >= 64) ? 64 : 32;
       L.n_tiles_n = co / L.bn;
       L.in = in;
@@ -412,6 +422,35 @@ rtcc_status build_branch(rtcc_ctx* c, int k) {
       b.layers.push_back(L);
     }
   }
+  // split-K for layers whose tile grid would leave SMs idle: the largest
+  // power-of-two split <= 8 that keeps the CTAs within one wave and every slice
+  // at >= 4 K-blocks
+  int sms = 148, dev = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  size_t ws_floats = 0, max_tiles = 0;
+  for (ConvLayer& L : b.layers) {
+    const int m_tiles = ((L.gw + conv_tile_w() - 1) / conv_tile_w()) *
+                        ((L.gh + conv_tile_h() - 1) / conv_tile_h());
+    const int base = m_tiles * L.n_tiles_n;
+    const int total_kb = (L.kind == DECONV ? 1 : 9) * (L.cin / L.bk);
+    int sp = 1;
+    while (sp * 2 <= 8 && base * sp * 2 <= sms && total_kb / (sp * 2) >= 4) sp *= 2;
+    L.splits = sp;
+    if (sp > 1) {
+      ws_floats = std::max(ws_floats, (size_t)sp * base * conv_tile_m() * L.bn);
+      max_tiles = std::max(max_tiles, (size_t)base);
+    }
+  }
+  if (ws_floats) {
+    RS(dalloc(c, &b.splitk_ws, ws_floats * sizeof(float)));
+    RS(dalloc(c, &b.splitk_cnt, max_tiles * sizeof(int)));
+    CK(cudaMemset(b.splitk_cnt, 0, max_tiles * sizeof(int)));
+  }
+  for (ConvLayer& L : b.layers) {
+    L.ws = b.splitk_ws;
+    L.counters = b.splitk_cnt;
+  }
   CK(cudaStreamCreateWithFlags(&b.st, cudaStreamNonBlocking));
   CK(cudaEventCreateWithFlags(&b.h2d_done, cudaEventDisableTiming));
   CK(cudaEventCreateWithFlags(&b.done, cudaEventDisableTiming));
@@ -419,6 +458,10 @@ rtcc_status build_branch(rtcc_ctx* c, int k) {
   CK(cudaEventCreate(&b.ev_bb0));
   CK(cudaEventCreate(&b.ev_bb1));
   CK(cudaEventCreate(&b.ev_end));
+  if (g.flags & RTCC_FLAG_LAYER_TIMES) {
+    b.layer_ev.resize(b.layers.size() + 1, nullptr);
+    for (auto& ev : b.layer_ev) CK(cudaEventCreate(&ev));
+  }
   return RTCC_OK;
 }
 
@@ -439,8 +482,12 @@ rtcc_status capture_branch(rtcc_ctx* c, int k) {
   if (e == cudaSuccess) e = cudaMemsetAsync(b.pb.stats, 0, 8 * sizeof(int), b.st);
   if (e == cudaSuccess) e = launch_pillarise(b.pb, gg, c->pfn_w, c->pfn_b, c->bf16, c->d_err, b.st);
   if (e == cudaSuccess && tl) e = record_node(b.ev_bb0, b.st);
-  for (size_t i = 0; e == cudaSuccess && i < b.layers.size(); ++i)
-    e = launch_conv(b.layers[i], c->bf16, c->d_err, b.st);
+  const bool lt = !b.layer_ev.empty();
+  for (size_t i = 0; e == cudaSuccess && i < b.layers.size(); ++i) {
+    if (lt) e = record_node(b.layer_ev[i], b.st);
+    if (e == cudaSuccess) e = launch_conv(b.layers[i], c->bf16, c->d_err, b.st);
+  }
+  if (e == cudaSuccess && lt) e = record_node(b.layer_ev.back(), b.st);
   if (e == cudaSuccess && tl) e = record_node(b.ev_bb1, b.st);
   if (e == cudaSuccess && tl) e = record_node(b.ev_end, b.st);
   cudaGraph_t graph = nullptr;
@@ -467,8 +514,14 @@ rtcc_status capture_post(rtcc_ctx* c) {
   fa.head_b = c->head_b;
   fa.head_out = c->head_out;
   fa.fused = c->fused;
+  fa.keys = c->keys;
+  fa.hist0 = c->hist0;
+  fa.cls_thresh = c->cfg.cls_thresh;
+  fa.anchors = c->cfg.anchors;
   DecodeArgs da{};
   da.head = c->head_out;
+  da.keys = c->keys;
+  da.hist0 = c->hist0;
   da.feat_w = c->Wf;
   da.feat_h = c->Hf;
   da.anchors = c->cfg.anchors;
@@ -476,9 +529,7 @@ rtcc_status capture_post(rtcc_ctx* c) {
   da.y_min = c->cfg.y_min;
   da.x_max = c->cfg.x_max;
   da.y_max = c->cfg.y_max;
-  da.cls_thresh = c->cfg.cls_thresh;
   da.max_boxes = c->cfg.max_boxes;
-  da.cand = c->cand;
   da.err = c->d_err;
   da.out = c->det_dev;
   (void)cudaGetLastError();
@@ -509,6 +560,8 @@ void free_all(rtcc_ctx* c) {
     if (b.st) cudaStreamSynchronize(b.st);
     if (b.exec) cudaGraphExecDestroy(b.exec);
     for (cudaEvent_t ev : {b.h2d_done, b.done, b.ev_start, b.ev_bb0, b.ev_bb1, b.ev_end})
+      if (ev) cudaEventDestroy(ev);
+    for (cudaEvent_t ev : b.layer_ev)
       if (ev) cudaEventDestroy(ev);
     if (b.st) cudaStreamDestroy(b.st);
   }
@@ -542,8 +595,11 @@ rtcc_status init_impl(rtcc_ctx* c, const float* weights) {
   CK(cudaMemcpy(c->d_feat_ptrs, fp, sizeof(fp), cudaMemcpyHostToDevice));
   RS(dalloc(c, &c->head_out, (size_t)cells_f * 16 * sizeof(float)));
   if (g.flags & RTCC_FLAG_KEEP_FUSED) RS(dalloc(c, &c->fused, (size_t)cells_f * c->Cf * 2));
-  const int nch = decode_chunks(cells_f * g.anchors);
-  RS(dalloc(c, &c->cand, (size_t)nch * kDecodeKeep * 8 + (size_t)nch * 4));
+  const size_t nkeys = decode_key_capacity(cells_f * g.anchors);
+  RS(dalloc(c, &c->keys, nkeys * sizeof(uint32_t)));
+  CK(cudaMemset(c->keys, 0xFF, nkeys * sizeof(uint32_t)));   // padding stays invalid
+  RS(dalloc(c, &c->hist0, kDecodeHistBins * sizeof(uint32_t)));
+  CK(cudaMemset(c->hist0, 0, kDecodeHistBins * sizeof(uint32_t)));
   c->det_bytes = sizeof(DetResultHeader) + (size_t)g.max_boxes * sizeof(rtcc_box);
   RS(dalloc(c, &c->det_dev, c->det_bytes));
   CK(cudaMemset(c->det_dev, 0, c->det_bytes));
@@ -818,6 +874,26 @@ rtcc_status rtcc_get_frame_info(rtcc_ctx* c, rtcc_frame_info* info) {
   if (!c || !info) return RTCC_E_ARG;
   std::lock_guard<std::mutex> lk(c->mu);
   *info = c->info;
+  return RTCC_OK;
+}
+
+rtcc_status rtcc_get_layer_times(rtcc_ctx* c, int32_t agent, float* host_ms, int32_t cap,
+                                 int32_t* n_out) {
+  if (!c) return RTCC_E_ARG;
+  std::lock_guard<std::mutex> lk(c->mu);
+  if (agent < 0 || agent >= c->K) return RTCC_E_AGENT;
+  Branch& b = c->br[agent];
+  if (b.layer_ev.empty()) return RTCC_E_STATE;
+  const int n = (int)b.layers.size();
+  if (n_out) *n_out = n;
+  if (!host_ms) return RTCC_OK;
+  CK(cudaStreamSynchronize(b.st));
+  for (int i = 0; i < n && i < cap; ++i) {
+    float ms = -1.f;
+    if (cudaEventElapsedTime(&ms, b.layer_ev[i], b.layer_ev[i + 1]) != cudaSuccess) ms = -1.f;
+    host_ms[i] = ms;
+  }
+  (void)cudaGetLastError();
   return RTCC_OK;
 }
 

@@ -9,6 +9,26 @@
 
 namespace rtcc {
 
+// Launch `kern` on `st` with programmatic stream serialisation, so that it may
+// begin while the previous kernel in the stream finishes (the kernel itself
+// calls pdl_wait before touching shared data).  Captured into a graph, this
+// becomes a programmatic dependency edge.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t st, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
 // Pillar grid geometry (float32, as the points are).
 struct GridGeom {
   float x_min, y_min, z_min, z_max, v;
@@ -25,6 +45,7 @@ struct PillarBufs {
   int* cnt_cell;         // [H*W]   points per cell (0 between passes)
   int* first_cell;       // [H*W]   first point index per cell (kFirstInit between passes)
   int* c2p;              // [H*W]   pillar id of a cell (valid where cnt_cell > 0)
+  int2* items;           // [cap]   per point (first-point flag, its cell's count)
   int2* blocksum;        // [nblk]  per-tile (#first points, #points of their cells)
   int* pcnt_raw;         // [P]     points of the pillar's cell before the N_max cap
   int* poff;             // [P]     offset of the pillar's point list
@@ -42,7 +63,7 @@ struct PillarBufs {
 };
 
 constexpr int kFirstInit = 0x7F7F7F7F;   // memset byte 0x7F
-constexpr int kScanTile = 4096;          // points per scan block
+constexpr int kScanTile = 1024;          // points per scan block
 inline int scan_blocks(int cap) { return (cap + kScanTile - 1) / kScanTile; }
 
 // Enqueue the 6 pillar kernels (cells, block sums, scan, fill, PFN, scatter).
@@ -65,18 +86,22 @@ struct ConvLayer {
   int ldc, choff;        // output pixel stride (channels) and channel offset
   int bn, bk;            // N tile (output channels per CTA), K chunk (channels)
   int n_tiles_n;         // grid.y
+  int splits;            // split-K factor (grid.z); 1 = none
+  float* ws;             // split-K partials [splits][m_tiles * n_tiles][128][bn] fp32
+  int* counters;         // split-K arrivals per tile [m_tiles * n_tiles], zero-initialised
   const void* in;        // device [in_h][in_w][cin]
   void* out;             // device [out_h][out_w][ldc]
   const void* wpacked;   // device, K-major: conv [Cout][9][Cin]; deconv [s*s*Cout][Cin]
   const float* bias;     // device [Cout]
-  CUtensorMap mapA, mapB;
+  CUtensorMap mapA, mapB, mapC;   // input, packed weights, output (store)
 };
 
-// Encode the layer's tensor maps (input activations and packed weights).
+// Encode the layer's tensor maps (input activations, packed weights, output).
 cudaError_t conv_make_maps(ConvLayer& L, bool bf16);
 cudaError_t launch_conv(const ConvLayer& L, bool bf16, int* err, cudaStream_t st);
 int conv_tile_w();
 int conv_tile_h();
+int conv_tile_m();
 
 // ---------------------------------------------------------------------------
 // post-join: fusion + head, decode
@@ -91,6 +116,10 @@ struct FuseArgs {
   const float* head_b;       // device [16]
   float* head_out;           // device [cells][16]
   void* fused;               // device [cells][C] or null
+  uint32_t* keys;            // device [cells][anchors] decode keys (see fuse_head.cu)
+  uint32_t* hist0;           // device [4096] histogram of the keys' top 12 bits
+  float cls_thresh;
+  int anchors;
 };
 cudaError_t launch_fuse_head(const FuseArgs& a, bool bf16, cudaStream_t st);
 // Head weight permutation expected by the fusion kernel (host side).
@@ -98,17 +127,22 @@ void permute_head_weights(const float* w /*[16][C]*/, int C, float* out /*[16*C]
 
 struct DecodeArgs {
   const float* head;         // [cells][16]
+  const uint32_t* keys;      // [cells][anchors] from the fusion kernel, padded with
+                             // 0xFFFFFFFF to decode_key_capacity() entries
+  uint32_t* hist0;           // [4096] top-12-bit histogram of the valid keys; the
+                             // decode clears it after reading
   int feat_w, feat_h, anchors;
   float x_min, y_min, x_max, y_max;
-  float cls_thresh;
   int max_boxes;
-  unsigned long long* cand;  // [n_chunks][kDecodeKeep] keys, then [n_chunks] int counts
   const int* err;            // device error word, copied into the result header
   void* out;                 // device result block: DetResultHeader + rtcc_box[max_boxes]
 };
-constexpr int kDecodeChunk = 4096;
-constexpr int kDecodeKeep = 512;     // >= max_boxes
-int decode_chunks(int n_anchors);
+constexpr int kDecodeKeep = 512;     // largest supported max_boxes
+constexpr int kDecodeHistBins = 4096;
+int decode_key_chunk4(int n_anchors);
+inline size_t decode_key_capacity(int n_anchors) {
+  return (size_t)decode_key_chunk4(n_anchors) * 4 * 1024;
+}
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t st);
 
 // Result block the post-join graph copies to pinned host memory.

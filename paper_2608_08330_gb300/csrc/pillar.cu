@@ -16,8 +16,10 @@
 //               list (slot order arbitrary).
 //   4. PFN:     one warp per pillar selects the N_max smallest indices of its
 //               list (warp bitonic sort/merge), i.e. the first N_max points in
-//               point order, then computes the 9-d features, the linear layer,
-//               ReLU and the max over points; every reduction has a fixed
+//               point order, one point per lane.  The means sum in lane order;
+//               then each lane owns C/32 output channels and folds the kept
+//               points in one at a time (broadcast by shuffle): 9-d features,
+//               linear layer, ReLU, running max.  Every reduction has a fixed
 //               order, so the result is run-to-run deterministic.
 //   5. scatter: one pass over all cells writes the pillar vector or zeros
 //               (each cell has at most one pillar: no atomics) and restores the
@@ -36,6 +38,8 @@ constexpr unsigned kFull = 0xFFFFFFFFu;
 __global__ void k_pillar_cells(const float4* __restrict__ pts, const int* __restrict__ n_hdr,
                                GridGeom g, int* __restrict__ cell_of, int* __restrict__ cnt_cell,
                                int* __restrict__ first_cell, int* __restrict__ stats) {
+  pdl_trigger();
+  pdl_wait();
   const int n = *n_hdr;
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i == 0) stats[0] = n;
@@ -79,8 +83,8 @@ __device__ __forceinline__ int2 shfl_xor2(int2 v, int d) {
   return make_int2(__shfl_xor_sync(kFull, v.x, d), __shfl_xor_sync(kFull, v.y, d));
 }
 
-// Exclusive block scan of one int2 per thread (1024 threads); returns the
-// exclusive prefix and writes the block total to *total.
+// Exclusive block scan of one int2 per thread (blockDim a multiple of 32, up to
+// 1024); returns the exclusive prefix and writes the block total to *total.
 __device__ int2 block_excl_scan(int2 v, int2* total) {
   __shared__ int2 warp_sums[32];
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
@@ -108,18 +112,30 @@ __device__ int2 block_excl_scan(int2 v, int2* total) {
   return make_int2(wpre.x + inc.x - v.x, wpre.y + inc.y - v.y);
 }
 
-constexpr int kScanThreads = 1024;
+constexpr int kScanThreads = 256;
 constexpr int kItems = kScanTile / kScanThreads;   // 4 consecutive points per thread
+static_assert(kItems == 4, "the item loads below move 4 points per thread");
 
 __global__ void __launch_bounds__(kScanThreads)
 k_pillar_blocksum(const int* __restrict__ n_hdr, const int* __restrict__ cell_of,
                   const int* __restrict__ cnt_cell, const int* __restrict__ first_cell,
-                  int2* __restrict__ blocksum) {
+                  int2* __restrict__ items, int2* __restrict__ blocksum) {
+  pdl_trigger();
+  pdl_wait();
   const int n = *n_hdr;
   const int base = blockIdx.x * kScanTile + threadIdx.x * kItems;
   int2 s = make_int2(0, 0);
+  int2 it[kItems];
 #pragma unroll
-  for (int q = 0; q < kItems; ++q) s = add2(s, first_point_item(base + q, n, cell_of, cnt_cell, first_cell));
+  for (int q = 0; q < kItems; ++q) {
+    it[q] = first_point_item(base + q, n, cell_of, cnt_cell, first_cell);
+    s = add2(s, it[q]);
+  }
+  if (base < n) {
+    int4* dst = reinterpret_cast<int4*>(items + base);
+    dst[0] = make_int4(it[0].x, it[0].y, it[1].x, it[1].y);
+    dst[1] = make_int4(it[2].x, it[2].y, it[3].x, it[3].y);
+  }
 #pragma unroll
   for (int d = 16; d > 0; d >>= 1) s = add2(s, shfl_xor2(s, d));
   __shared__ int2 ws[32];
@@ -127,7 +143,7 @@ k_pillar_blocksum(const int* __restrict__ n_hdr, const int* __restrict__ cell_of
   if (lane == 0) ws[wid] = s;
   __syncthreads();
   if (wid == 0) {
-    int2 t = ws[lane];
+    int2 t = lane < (int)(blockDim.x >> 5) ? ws[lane] : make_int2(0, 0);
 #pragma unroll
     for (int d = 16; d > 0; d >>= 1) t = add2(t, shfl_xor2(t, d));
     if (lane == 0) blocksum[blockIdx.x] = t;
@@ -136,12 +152,14 @@ k_pillar_blocksum(const int* __restrict__ n_hdr, const int* __restrict__ cell_of
 
 __global__ void __launch_bounds__(kScanThreads)
 k_pillar_scan(const int* __restrict__ n_hdr, const int* __restrict__ cell_of,
-              const int* __restrict__ cnt_cell, const int* __restrict__ first_cell,
-              const int2* __restrict__ blocksum, int P, int* __restrict__ c2p,
+              const int2* __restrict__ items, const int2* __restrict__ blocksum, int P,
+              int* __restrict__ c2p,
               int* __restrict__ pillar_cell, int* __restrict__ pcnt_raw, int* __restrict__ poff,
               int* __restrict__ cursor, int* __restrict__ stats) {
   __shared__ int2 pre;
   __shared__ int2 tot;
+  pdl_trigger();
+  pdl_wait();
   const int n = *n_hdr;
   const int lane = threadIdx.x & 31;
   if (threadIdx.x < 32) {
@@ -153,13 +171,18 @@ k_pillar_scan(const int* __restrict__ n_hdr, const int* __restrict__ cell_of,
   }
   __syncthreads();
   const int base = blockIdx.x * kScanTile + threadIdx.x * kItems;
-  int2 it[kItems];
+  int2 it[kItems] = {};
+  if (base < n) {
+    const int4* src = reinterpret_cast<const int4*>(items + base);
+    const int4 a = src[0], b = src[1];
+    it[0] = make_int2(a.x, a.y);
+    it[1] = make_int2(a.z, a.w);
+    it[2] = make_int2(b.x, b.y);
+    it[3] = make_int2(b.z, b.w);
+  }
   int2 own = make_int2(0, 0);
 #pragma unroll
-  for (int q = 0; q < kItems; ++q) {
-    it[q] = first_point_item(base + q, n, cell_of, cnt_cell, first_cell);
-    own = add2(own, it[q]);
-  }
+  for (int q = 0; q < kItems; ++q) own = add2(own, it[q]);
   int2 run = block_excl_scan(own, &tot);
   run = add2(run, pre);
 #pragma unroll
@@ -187,6 +210,8 @@ k_pillar_scan(const int* __restrict__ n_hdr, const int* __restrict__ cell_of,
 __global__ void k_pillar_fill(const int* __restrict__ n_hdr, const int* __restrict__ cell_of,
                               const int* __restrict__ c2p, int P, const int* __restrict__ poff,
                               int* __restrict__ cursor, int* __restrict__ list) {
+  pdl_trigger();
+  pdl_wait();
   const int n = *n_hdr;
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n) return;
@@ -238,69 +263,81 @@ k_pfn(const float4* __restrict__ pts, const int* __restrict__ stats_in,
       T* __restrict__ feat, int* __restrict__ pcount, int* __restrict__ stats) {
   __shared__ float sw[C * 9];
   __shared__ float sb[C];
-  for (int j = threadIdx.x; j < C * 9; j += blockDim.x) sw[j] = w[j];
+  __shared__ int s_stat[3];                   // kept, capped, raw (block partial sums)
+  pdl_trigger();
+  for (int j = threadIdx.x; j < C * 9; j += blockDim.x) sw[j] = w[j];   // weights: constant
+  pdl_wait();
   for (int j = threadIdx.x; j < C; j += blockDim.x) sb[j] = b[j];
+  if (threadIdx.x < 3) s_stat[threadIdx.x] = 0;
   __syncthreads();
   const int lane = threadIdx.x & 31;
   const int p = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int np = stats_in[2];
-  if (p >= np) return;
-  const int raw = pcnt_raw[p];
-  const int base = poff[p];
-  // the min(raw, N) smallest point indices, ascending = the pillar's first points
-  int idx = lane < raw ? list[base + lane] : INT_MAX;
-  idx = warp_sort_asc(idx, lane);
-  for (int c = 32; c < raw; c += 32) {
-    int v = (c + lane < raw) ? list[base + c + lane] : INT_MAX;
-    v = warp_sort_asc(v, lane);
-    const int vr = __shfl_sync(kFull, v, 31 - lane);
-    idx = warp_merge_asc(min(idx, vr), lane);
-  }
-  const int m = raw < N ? raw : N;
-  const bool valid = lane < m;
-  const float4 q = valid ? pts[idx] : make_float4(0.f, 0.f, 0.f, 0.f);
-  const float fm = (float)m;
-  const float mx = __fdiv_rn(warp_sum(q.x), fm);
-  const float my = __fdiv_rn(warp_sum(q.y), fm);
-  const float mz = __fdiv_rn(warp_sum(q.z), fm);
-  const int cell = pillar_cell[p];
-  const int cx = cell % g.W, cy = cell / g.W;
-  const float xc = __fadd_rn(g.x_min, __fmul_rn((float)cx + 0.5f, g.v));
-  const float yc = __fadd_rn(g.y_min, __fmul_rn((float)cy + 0.5f, g.v));
-  float f[9] = {q.x, q.y, q.z, q.w, q.x - mx, q.y - my, q.z - mz, q.x - xc, q.y - yc};
-  float acc[C];
+  if (p < np) {
+    const int raw = pcnt_raw[p];
+    const int base = poff[p];
+    // the min(raw, N) smallest point indices, ascending = the pillar's first points
+    int idx = lane < raw ? list[base + lane] : INT_MAX;
+    idx = warp_sort_asc(idx, lane);
+    for (int c = 32; c < raw; c += 32) {
+      int v = (c + lane < raw) ? list[base + c + lane] : INT_MAX;
+      v = warp_sort_asc(v, lane);
+      const int vr = __shfl_sync(kFull, v, 31 - lane);
+      idx = warp_merge_asc(min(idx, vr), lane);
+    }
+    const int m = raw < N ? raw : N;
+    const bool valid = lane < m;
+    const float4 q = valid ? pts[idx] : make_float4(0.f, 0.f, 0.f, 0.f);
+    const float fm = (float)m;
+    const float mx = __fdiv_rn(warp_sum(q.x), fm);
+    const float my = __fdiv_rn(warp_sum(q.y), fm);
+    const float mz = __fdiv_rn(warp_sum(q.z), fm);
+    const int cell = pillar_cell[p];
+    const int cx = cell % g.W, cy = cell / g.W;
+    const float xc = __fadd_rn(g.x_min, __fmul_rn((float)cx + 0.5f, g.v));
+    const float yc = __fadd_rn(g.y_min, __fmul_rn((float)cy + 0.5f, g.v));
+    // channel-parallel: lane l owns channels [l*PER, (l+1)*PER); the pillar's
+    // kept points (one per lane, in point order) are broadcast one at a time
+    constexpr int PER = C / 32;
+    float wl[PER][9], bl[PER], acc[PER];
 #pragma unroll
-  for (int j = 0; j < C; ++j) {
-    float s = sb[j];
+    for (int i = 0; i < PER; ++i) {
+      bl[i] = sb[lane * PER + i];
+      acc[i] = 0.f;                       // every h >= 0 after ReLU and m >= 1
 #pragma unroll
-    for (int d = 0; d < 9; ++d) s = fmaf(sw[j * 9 + d], f[d], s);
-    acc[j] = valid ? relu_f(s) : 0.f;   // invalid lanes add 0: the max is >= 0 anyway
-  }
-  // reduce-scatter max over lanes: lane l ends with channels [l*C/32, (l+1)*C/32)
-  int n = C;
+      for (int d = 0; d < 9; ++d) wl[i][d] = sw[(lane * PER + i) * 9 + d];
+    }
+    for (int j = 0; j < m; ++j) {
+      const float x = __shfl_sync(kFull, q.x, j);
+      const float y = __shfl_sync(kFull, q.y, j);
+      const float zz = __shfl_sync(kFull, q.z, j);
+      const float it = __shfl_sync(kFull, q.w, j);
+      const float f[9] = {x, y, zz, it, x - mx, y - my, zz - mz, x - xc, y - yc};
 #pragma unroll
-  for (int off = 16; off > 0; off >>= 1) {
-    const int h = n >> 1;
-    const bool upper = (lane & off) != 0;
+      for (int i = 0; i < PER; ++i) {
+        float sacc = bl[i];
 #pragma unroll
-    for (int i = 0; i < C / 2; ++i) {
-      if (i < h) {
-        const float send = upper ? acc[i] : acc[i + h];
-        const float keep = upper ? acc[i + h] : acc[i];
-        acc[i] = fmaxf(keep, __shfl_xor_sync(kFull, send, off));
+        for (int d = 0; d < 9; ++d) sacc = fmaf(wl[i][d], f[d], sacc);
+        acc[i] = fmaxf(acc[i], relu_f(sacc));
       }
     }
-    n = h;
-  }
-  constexpr int PER = C / 32;
-  T* dst = feat + (size_t)p * C + lane * PER;
+    T* dst = feat + (size_t)p * C + lane * PER;
 #pragma unroll
-  for (int i = 0; i < PER; ++i) dst[i] = Store<T>::from_f(acc[i]);
-  if (lane == 0) {
-    pcount[p] = m;
-    atomicAdd(&stats[3], m);
-    atomicAdd(&stats[6], raw - m);
-    atomicAdd(&stats[7], raw);
+    for (int i = 0; i < PER; ++i) dst[i] = Store<T>::from_f(acc[i]);
+    if (lane == 0) {
+      pcount[p] = m;
+      atomicAdd(&s_stat[0], m);
+      atomicAdd(&s_stat[1], raw - m);
+      atomicAdd(&s_stat[2], raw);
+    }
+  }
+  // one global update per block (same-address atomics from every pillar
+  // serialise in L2)
+  __syncthreads();
+  if (threadIdx.x == 0 && s_stat[2] > 0) {
+    atomicAdd(&stats[3], s_stat[0]);
+    atomicAdd(&stats[6], s_stat[1]);
+    atomicAdd(&stats[7], s_stat[2]);
   }
 }
 
@@ -312,6 +349,8 @@ __global__ void k_scatter(const int* __restrict__ stats_in, const int* __restric
                           int* __restrict__ first_cell, int* __restrict__ cell2pillar,
                           uint4* __restrict__ image) {
   constexpr int CH = C * 2 / 16;   // 16-byte chunks per cell (divides 32)
+  pdl_trigger();
+  pdl_wait();
   const int t = blockIdx.x * blockDim.x + threadIdx.x;
   const int cell = t / CH, ch = t % CH;
   if (cell >= cells) return;     // all CH threads of a cell leave together
@@ -336,23 +375,30 @@ cudaError_t launch_all(const PillarBufs& b, const GridGeom& g, const float* pfn_
                        const float* pfn_b, cudaStream_t st) {
   const int cells = g.W * g.H;
   const int nblk = scan_blocks(b.cap);
-  k_pillar_cells<<<(b.cap + 255) / 256, 256, 0, st>>>(b.pts, b.n_hdr, g, b.cell_of, b.cnt_cell,
-                                                     b.first_cell, b.stats);
-  k_pillar_blocksum<<<nblk, kScanThreads, 0, st>>>(b.n_hdr, b.cell_of, b.cnt_cell, b.first_cell,
-                                                   b.blocksum);
-  k_pillar_scan<<<nblk, kScanThreads, 0, st>>>(b.n_hdr, b.cell_of, b.cnt_cell, b.first_cell,
-                                               b.blocksum, b.P, b.c2p, b.pillar_cell, b.pcnt_raw,
-                                               b.poff, b.cursor, b.stats);
-  k_pillar_fill<<<(b.cap + 255) / 256, 256, 0, st>>>(b.n_hdr, b.cell_of, b.c2p, b.P, b.poff,
-                                                     b.cursor, b.list);
-  k_pfn<T, C><<<(b.P + 7) / 8, 256, 0, st>>>(b.pts, b.stats, b.pcnt_raw, b.poff, b.list,
-                                             b.pillar_cell, pfn_w, pfn_b, g, b.N,
-                                             static_cast<T*>(b.feat), b.pcount, b.stats);
+  cudaError_t e;
+  e = launch_pdl(k_pillar_cells, dim3((b.cap + 255) / 256), dim3(256), 0, st, b.pts, b.n_hdr, g,
+                 b.cell_of, b.cnt_cell, b.first_cell, b.stats);
+  if (e != cudaSuccess) return e;
+  e = launch_pdl(k_pillar_blocksum, dim3(nblk), dim3(kScanThreads), 0, st, b.n_hdr, b.cell_of,
+                 b.cnt_cell, b.first_cell, b.items, b.blocksum);
+  if (e != cudaSuccess) return e;
+  e = launch_pdl(k_pillar_scan, dim3(nblk), dim3(kScanThreads), 0, st, b.n_hdr, b.cell_of,
+                 b.items, b.blocksum, b.P, b.c2p, b.pillar_cell, b.pcnt_raw, b.poff, b.cursor,
+                 b.stats);
+  if (e != cudaSuccess) return e;
+  e = launch_pdl(k_pillar_fill, dim3((b.cap + 255) / 256), dim3(256), 0, st, b.n_hdr, b.cell_of,
+                 b.c2p, b.P, b.poff, b.cursor, b.list);
+  if (e != cudaSuccess) return e;
+  e = launch_pdl(k_pfn<T, C>, dim3((b.P + 7) / 8), dim3(256), 0, st, b.pts, b.stats, b.pcnt_raw,
+                 b.poff, b.list, b.pillar_cell, pfn_w, pfn_b, g, b.N, static_cast<T*>(b.feat),
+                 b.pcount, b.stats);
+  if (e != cudaSuccess) return e;
   constexpr int CH = C * 2 / 16;
   const long long thr = (long long)cells * CH;
-  k_scatter<C><<<(unsigned)((thr + 255) / 256), 256, 0, st>>>(
-      b.stats, b.c2p, b.P, static_cast<const uint4*>(b.feat), cells, b.cnt_cell, b.first_cell,
-      b.cell2pillar, static_cast<uint4*>(b.image));
+  e = launch_pdl(k_scatter<C>, dim3((unsigned)((thr + 255) / 256)), dim3(256), 0, st, b.stats,
+                 b.c2p, b.P, static_cast<const uint4*>(b.feat), cells, b.cnt_cell, b.first_cell,
+                 b.cell2pillar, static_cast<uint4*>(b.image));
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

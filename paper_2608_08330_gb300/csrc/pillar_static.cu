@@ -8,7 +8,7 @@
 // this entry point takes its scratch from one fixed array in device global
 // memory that the library reserves when it is loaded, instead of calling any
 // allocator.  The array is sized for grids up to 65,536 cells, payloads up to
-// 131,072 points, 16,384 pillars and 64 PFN channels (about 4.3 MB, held on
+// 131,072 points, 16,384 pillars and 64 PFN channels (about 5.2 MB, held on
 // every GPU that loads the library until the process exits).
 //
 // The kernels are the ones rtcc_payload_complete runs (launch_pillarise); only
@@ -41,7 +41,8 @@ constexpr size_t kOffCnt = align256(kOffList + 4ull * kMaxPoints);
 constexpr size_t kOffFirst = align256(kOffCnt + 4ull * kMaxCells);
 constexpr size_t kOffC2P = align256(kOffFirst + 4ull * kMaxCells);
 constexpr size_t kOffBlock = align256(kOffC2P + 4ull * kMaxCells);
-constexpr size_t kOffRaw = align256(kOffBlock + 8ull * kMaxScanBlocks);
+constexpr size_t kOffItems = align256(kOffBlock + 8ull * kMaxScanBlocks);
+constexpr size_t kOffRaw = align256(kOffItems + 8ull * kMaxScanBlocks * kScanTile);
 constexpr size_t kOffPoff = align256(kOffRaw + 4ull * kMaxPillars);
 constexpr size_t kOffCursor = align256(kOffPoff + 4ull * kMaxPillars);
 constexpr size_t kOffFeat = align256(kOffCursor + 4ull * kMaxPillars);
@@ -114,6 +115,7 @@ extern "C" rtcc_status rtcc_pillarise_noalloc(const rtcc_model_config* cfg, cons
   b.first_cell = reinterpret_cast<int*>(base + kOffFirst);
   b.c2p = reinterpret_cast<int*>(base + kOffC2P);
   b.blocksum = reinterpret_cast<int2*>(base + kOffBlock);
+  b.items = reinterpret_cast<int2*>(base + kOffItems);
   b.pcnt_raw = reinterpret_cast<int*>(base + kOffRaw);
   b.poff = reinterpret_cast<int*>(base + kOffPoff);
   b.cursor = reinterpret_cast<int*>(base + kOffCursor);

@@ -27,7 +27,7 @@ MODE_RTCC, MODE_BARRIER = 0, 1
 FUSE_MAX, FUSE_ATTN = 0, 1
 FP16, BF16 = 0, 1
 WAITING, RELEASED, RUNNING, FINISHED, ABSENT = range(5)
-FLAG_TIMELINE, FLAG_KEEP_FUSED, FLAG_KEEP_LAYERS = 1, 2, 4
+FLAG_TIMELINE, FLAG_KEEP_FUSED, FLAG_KEEP_LAYERS, FLAG_LAYER_TIMES = 1, 2, 4, 8
 TENSOR_IMAGE, TENSOR_FEAT, TENSOR_FUSED, TENSOR_LAYER0 = 0, 8, 9, 16
 
 
@@ -104,6 +104,8 @@ def load(path: Optional[str] = None) -> C.CDLL:
         "rtcc_get_frame_info": (S, [_ctx_p, C.POINTER(rtcc_frame_info)]),
         "rtcc_get_branch_state": (S, [_ctx_p, C.c_int32, C.POINTER(C.c_int32),
                                       C.POINTER(C.c_double)]),
+        "rtcc_get_layer_times": (S, [_ctx_p, C.c_int32, C.c_void_p, C.c_int32,
+                                     C.POINTER(C.c_int32)]),
         "rtcc_get_head": (S, [_ctx_p, C.c_void_p, C.c_size_t]),
         "rtcc_get_pillars": (S, [_ctx_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p,
                                  C.c_void_p]),
@@ -251,6 +253,17 @@ def rtcc_get_frame_info(ctx) -> rtcc_frame_info:
     info = rtcc_frame_info()
     _chk(load().rtcc_get_frame_info(ctx, C.byref(info)), "rtcc_get_frame_info")
     return info
+
+
+def rtcc_get_layer_times(ctx, agent: int) -> np.ndarray:
+    """Per-layer ms of the agent's conv/deconv launches in the last frame."""
+    lib = load()
+    n = C.c_int32(0)
+    _chk(lib.rtcc_get_layer_times(ctx, agent, None, 0, C.byref(n)), "rtcc_get_layer_times")
+    out = np.empty(n.value, dtype=np.float32)
+    _chk(lib.rtcc_get_layer_times(ctx, agent, _ptr(out), out.size, C.byref(n)),
+         "rtcc_get_layer_times")
+    return out
 
 
 def rtcc_get_branch_state(ctx, agent: int):
