@@ -90,10 +90,8 @@ typedef enum {
 #define RTCC_FLAG_KEEP_FUSED  2  /* also store the fused BEV map (parity)      */
 #define RTCC_FLAG_KEEP_LAYERS 4  /* give every conv layer its own output buffer
                                     so each can be read back (parity)         */
-#define RTCC_FLAG_LAYER_TIMES 8  /* record CUDA events between every conv/deconv
-                                    launch of a branch (per-layer timing; the
-                                    events also stop launch overlap between
-                                    layers, so use it to profile, not to serve) */
+#define RTCC_FLAG_LAYER_TIMES 8  /* record the GPU time at which the backbone
+                                    kernel starts each conv/deconv layer       */
 
 /*
  * Network and workload description.  Supported: 1 <= n_agents <= 8;
@@ -249,9 +247,11 @@ rtcc_status rtcc_wait_detection(struct rtcc_ctx* ctx, int32_t timeout_ms,
 /* Timestamps and GPU spans of the last closed frame. */
 rtcc_status rtcc_get_frame_info(struct rtcc_ctx* ctx, rtcc_frame_info* info);
 
-/* Per-layer GPU times (ms) of `agent`'s conv and deconv launches in the last
- * closed frame, in launch order (13 convs then 3 deconvs for the PointPillars
- * backbone); needs RTCC_FLAG_LAYER_TIMES.  *n_out receives the layer count. */
+/* Per-layer GPU times (ms) of `agent`'s conv and deconv layers in the last
+ * closed frame, in order (13 convs then 3 deconvs for the PointPillars
+ * backbone): the time between the backbone kernel starting consecutive layers
+ * (the last layer: until every CTA finished it).  Needs
+ * RTCC_FLAG_LAYER_TIMES.  *n_out receives the layer count. */
 rtcc_status rtcc_get_layer_times(struct rtcc_ctx* ctx, int32_t agent, float* host_ms,
                                  int32_t cap, int32_t* n_out);
 

@@ -48,11 +48,13 @@ struct Branch {
   std::vector<ConvLayer> layers;
   float* splitk_ws = nullptr;      // split-K partials, shared by the branch's layers
   int* splitk_cnt = nullptr;       // split-K per-tile arrival counters
+  unsigned* grid_bar = nullptr;    // backbone per-layer arrival counters
+  unsigned long long* stamps = nullptr;   // RTCC_FLAG_LAYER_TIMES: layer start times
+  BackboneParams* bb = nullptr;    // backbone kernel parameters (host copy)
   cudaStream_t st = nullptr;
   cudaGraphExec_t exec = nullptr;
   cudaEvent_t h2d_done = nullptr, done = nullptr;
   cudaEvent_t ev_start = nullptr, ev_bb0 = nullptr, ev_bb1 = nullptr, ev_end = nullptr;
-  std::vector<cudaEvent_t> layer_ev;   // RTCC_FLAG_LAYER_TIMES: before each layer + after last
   const float* pend_ptr = nullptr;
   int pend_n = 0;
   bool pend_resident = false;
@@ -334,6 +336,7 @@ rtcc_status build_branch(rtcc_ctx* c, int k) {
 
   // backbone layers
   const bool neck = g.up_stride[0] != 0;
+  int block_last[RTCC_MAX_BLOCKS] = {};
   const void* in = p.image;
   int cin = c->Cp, w = c->W, h = c->H;
   int wi = 0;
@@ -383,6 +386,7 @@ rtcc_status build_branch(rtcc_ctx* c, int k) {
       b.layer_elems.push_back((size_t)ow * oh * co);
       L.wpacked = c->wbufs[wi];
       L.bias = c->bbufs[wi];
+      L.wait_layers = (int)b.layers.size();          // reads the previous conv's output
       ++wi;
       if (conv_make_maps(L, c->bf16) != cudaSuccess) return RTCC_E_CUDA;
       b.layers.push_back(L);
@@ -390,6 +394,8 @@ rtcc_status build_branch(rtcc_ctx* c, int k) {
       cin = co;
     }
     b.block_out[bi] = const_cast<void*>(in);
+    block_last[bi] = (int)b.layers.size();          // layers [0, block_last) done
+
     b.block_w[bi] = ow;
     b.block_h[bi] = oh;
     w = ow;
@@ -417,14 +423,15 @@ rtcc_status build_branch(rtcc_ctx* c, int k) {
       L.out = b.feat;
       L.wpacked = c->wbufs[wi];
       L.bias = c->bbufs[wi];
+      L.wait_layers = block_last[bi];                 // only its block's output
       ++wi;
       if (conv_make_maps(L, c->bf16) != cudaSuccess) return RTCC_E_CUDA;
       b.layers.push_back(L);
     }
   }
   // split-K for layers whose tile grid would leave SMs idle: the largest
-  // power-of-two split <= 8 that keeps the CTAs within one wave and every slice
-  // at >= 4 K-blocks
+  // power-of-two split <= kMaxSplits that keeps the CTAs within one wave and
+  // every slice at >= 4 K-blocks
   int sms = 148, dev = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
@@ -435,7 +442,10 @@ rtcc_status build_branch(rtcc_ctx* c, int k) {
     const int base = m_tiles * L.n_tiles_n;
     const int total_kb = (L.kind == DECONV ? 1 : 9) * (L.cin / L.bk);
     int sp = 1;
-    while (sp * 2 <= 8 && base * sp * 2 <= sms && total_kb / (sp * 2) >= 4) sp *= 2;
+    // deconvs do not wait on their predecessor, so they may not share its
+    // split-K workspace: no split for them
+    while (L.kind != DECONV && sp * 2 <= kMaxSplits && base * sp * 2 <= sms && total_kb / (sp * 2) >= 4)
+      sp *= 2;
     L.splits = sp;
     if (sp > 1) {
       ws_floats = std::max(ws_floats, (size_t)sp * base * conv_tile_m() * L.bn);
@@ -451,6 +461,16 @@ rtcc_status build_branch(rtcc_ctx* c, int k) {
     L.ws = b.splitk_ws;
     L.counters = b.splitk_cnt;
   }
+  RS(dalloc(c, &b.grid_bar, kMaxLayers * sizeof(unsigned)));
+  CK(cudaMemset(b.grid_bar, 0, kMaxLayers * sizeof(unsigned)));
+  if (g.flags & RTCC_FLAG_LAYER_TIMES) {
+    RS(dalloc(c, &b.stamps, (b.layers.size() + 1) * sizeof(unsigned long long)));
+    CK(cudaMemset(b.stamps, 0, (b.layers.size() + 1) * sizeof(unsigned long long)));
+  }
+  b.bb = new (std::nothrow) BackboneParams;
+  if (!b.bb) return RTCC_E_NOMEM;
+  if (backbone_fill(b.layers, b.grid_bar, c->d_err, b.stamps, b.bb) != cudaSuccess)
+    return RTCC_E_ARG;
   CK(cudaStreamCreateWithFlags(&b.st, cudaStreamNonBlocking));
   CK(cudaEventCreateWithFlags(&b.h2d_done, cudaEventDisableTiming));
   CK(cudaEventCreateWithFlags(&b.done, cudaEventDisableTiming));
@@ -458,10 +478,6 @@ rtcc_status build_branch(rtcc_ctx* c, int k) {
   CK(cudaEventCreate(&b.ev_bb0));
   CK(cudaEventCreate(&b.ev_bb1));
   CK(cudaEventCreate(&b.ev_end));
-  if (g.flags & RTCC_FLAG_LAYER_TIMES) {
-    b.layer_ev.resize(b.layers.size() + 1, nullptr);
-    for (auto& ev : b.layer_ev) CK(cudaEventCreate(&ev));
-  }
   return RTCC_OK;
 }
 
@@ -482,12 +498,8 @@ rtcc_status capture_branch(rtcc_ctx* c, int k) {
   if (e == cudaSuccess) e = cudaMemsetAsync(b.pb.stats, 0, 8 * sizeof(int), b.st);
   if (e == cudaSuccess) e = launch_pillarise(b.pb, gg, c->pfn_w, c->pfn_b, c->bf16, c->d_err, b.st);
   if (e == cudaSuccess && tl) e = record_node(b.ev_bb0, b.st);
-  const bool lt = !b.layer_ev.empty();
-  for (size_t i = 0; e == cudaSuccess && i < b.layers.size(); ++i) {
-    if (lt) e = record_node(b.layer_ev[i], b.st);
-    if (e == cudaSuccess) e = launch_conv(b.layers[i], c->bf16, c->d_err, b.st);
-  }
-  if (e == cudaSuccess && lt) e = record_node(b.layer_ev.back(), b.st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(b.grid_bar, 0, kMaxLayers * sizeof(unsigned), b.st);
+  if (e == cudaSuccess) e = launch_backbone(*b.bb, c->bf16, b.st);
   if (e == cudaSuccess && tl) e = record_node(b.ev_bb1, b.st);
   if (e == cudaSuccess && tl) e = record_node(b.ev_end, b.st);
   cudaGraph_t graph = nullptr;
@@ -561,8 +573,8 @@ void free_all(rtcc_ctx* c) {
     if (b.exec) cudaGraphExecDestroy(b.exec);
     for (cudaEvent_t ev : {b.h2d_done, b.done, b.ev_start, b.ev_bb0, b.ev_bb1, b.ev_end})
       if (ev) cudaEventDestroy(ev);
-    for (cudaEvent_t ev : b.layer_ev)
-      if (ev) cudaEventDestroy(ev);
+    delete b.bb;
+    b.bb = nullptr;
     if (b.st) cudaStreamDestroy(b.st);
   }
   if (c->post) cudaStreamSynchronize(c->post);
@@ -883,17 +895,15 @@ rtcc_status rtcc_get_layer_times(rtcc_ctx* c, int32_t agent, float* host_ms, int
   std::lock_guard<std::mutex> lk(c->mu);
   if (agent < 0 || agent >= c->K) return RTCC_E_AGENT;
   Branch& b = c->br[agent];
-  if (b.layer_ev.empty()) return RTCC_E_STATE;
+  if (!b.stamps) return RTCC_E_STATE;
   const int n = (int)b.layers.size();
   if (n_out) *n_out = n;
   if (!host_ms) return RTCC_OK;
   CK(cudaStreamSynchronize(b.st));
-  for (int i = 0; i < n && i < cap; ++i) {
-    float ms = -1.f;
-    if (cudaEventElapsedTime(&ms, b.layer_ev[i], b.layer_ev[i + 1]) != cudaSuccess) ms = -1.f;
-    host_ms[i] = ms;
-  }
-  (void)cudaGetLastError();
+  std::vector<unsigned long long> t(n + 1);
+  CK(cudaMemcpy(t.data(), b.stamps, (n + 1) * sizeof(unsigned long long), cudaMemcpyDeviceToHost));
+  for (int i = 0; i < n && i < cap; ++i)
+    host_ms[i] = (t[i + 1] >= t[i] && t[i] > 0) ? (float)((t[i + 1] - t[i]) * 1e-6) : -1.f;
   return RTCC_OK;
 }
 
@@ -1018,7 +1028,7 @@ double rtcc_now_ms(void) { return now_ms(); }
 
 int32_t rtcc_kernels_per_frame(rtcc_ctx* c, int32_t n_present) {
   if (!c) return 0;
-  return n_present * (6 + c->n_conv + c->n_deconv) + 3;
+  return n_present * (6 + 1) + 2;     // pillar chain + backbone per branch; fusion, decode
 }
 
 }  // extern "C"

@@ -1,25 +1,44 @@
-// Implicit-GEMM convolutions of the encoder backbone and neck on the
-// 5th-generation tensor cores (tcgen05, accumulator in tensor memory), fed by
-// TMA tiled loads.  Used for every 3x3 conv (stride 1 and 2, zero padding 1)
-// and every transposed conv with kernel = stride (the PointPillars neck), all
-// followed by bias + ReLU (Sec. III-B: the per-agent encoder E_k).
+// Persistent implicit-GEMM backbone of one encoder branch on the 5th-
+// generation tensor cores (tcgen05, accumulators in tensor memory), fed by TMA.
+// One launch runs every 3x3 conv (stride 1 and 2, zero padding 1) and every
+// transposed conv with kernel = stride (the PointPillars neck) of a branch,
+// each followed by bias + ReLU (Sec. III-B: the per-agent encoder E_k).
 //
-// GEMM view, one CTA per (128-pixel tile, BN output channels):
+// GEMM view of a layer, one work item per (128-pixel tile, BN output
+// channels, K slice):
 //   D[m][n] = sum_k A[m][k] * B[n][k],  m = pixel, n = output channel,
 //   k = (tap, input channel), tap-major.
-// A (activations, NHWC) is never materialised: for each tap the producer warp
+// A (activations, NHWC) is never materialised: for each tap the producer
 // issues a TMA box load of the input shifted by the tap's offset; TMA fills
 // out-of-image elements with zeros, which is exactly the zero padding.  Stride
 // 2 uses a 5-D view of the same tensor, (2C, W/2, 2, H/2, 1), in which the
 // stride-2 gather becomes a unit-stride box at a tap-dependent (channel half,
 // column, row parity, row) offset.  B (weights) is pre-packed K-major.
 //
+// The grid is one CTA per SM, co-resident (cooperative launch).  Work items of
+// a layer are dealt round-robin over the CTAs; each CTA counts itself in the
+// layer's arrival counter once its part of the layer is written, and a layer
+// whose input another CTA writes starts once the counter of the layer it
+// depends on shows every CTA (one counter per layer: a CTA with no work in
+// some layers runs ahead and must not be counted for a layer it has not
+// reached in the others' order).  Keeping the CTAs resident replaces
+// sixteen kernel boundaries (each a full drain and relaunch) by counter waits,
+// and lets the TMA/MMA pipeline and the tensor-memory allocation carry across
+// tiles and layers.
+//
 // Roles (192 threads): warp 0 = TMA producer, warp 1 = tensor-memory owner and
-// MMA issuer, warps 2..5 = epilogue (tensor memory -> registers -> bias, ReLU,
-// 16-bit, staged in shared memory and written by TMA tensor stores).  Every mbarrier wait is bounded; a wait that runs out sets a
-// bit in the error word and the CTA winds down without hanging.
+// MMA issuer, warps 2..5 = epilogue.  Tensor memory holds two 128-column
+// accumulators, so the epilogue of one tile overlaps the MMAs of the next.
+// The epilogue adds bias, applies ReLU, rounds to 16 bits, stages the tile in
+// shared memory in the store map's swizzle and writes it with TMA tensor
+// stores.  Split-K slices publish fp32 partials and the last-arriving slice of
+// a tile sums them in slice order, so results do not depend on timing.  Every
+// wait is bounded; one that runs out sets a bit in the error word and the CTA
+// winds down instead of hanging.
+#include <cstring>
 #include <mutex>
 #include <type_traits>
+#include <vector>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -28,54 +47,34 @@ namespace rtcc {
 
 namespace {
 
-constexpr int TW = 32;            // tile width in pixels
-constexpr int TH = 4;             // tile height
-constexpr int BM = TW * TH;       // 128 = MMA M
+constexpr int TW = 32;                       // tile width in pixels
+constexpr int TH = 4;                        // tile height
+constexpr int BM = TW * TH;                  // 128 = MMA M
 constexpr int kThreads = 192;
-constexpr int kSmemBudget = 160 * 1024;
-
-struct ConvArgs {
-  const float* bias;
-  void* out;
-  int gw, gh;          // extent of the M grid
-  int out_w;           // output map width (pixels)
-  int ldc, choff;
-  int cin, cout, s;
-  int tiles_x;
-  int splits;          // K split across gridDim.z CTAs (1 = none)
-  float* ws;           // [splits][tiles][BN/4][BM][4] fp32 partials (splits > 1)
-  int* counters;       // [tiles] arrivals per tile, 0 between launches
-  int* err;
-};
-
-template <int BN, int BK>
-struct Geo {
-  static constexpr int A_BYTES = BM * BK * 2;
-  static constexpr int B_BYTES = BN * BK * 2;
-  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr int STAGES = (kSmemBudget / STAGE_BYTES) > 8 ? 8 : (kSmemBudget / STAGE_BYTES);
-  static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 256;
-  static constexpr int TMEM_COLS = BN < 32 ? 32 : BN;
-  static constexpr uint32_t SWZ = (BK == 64) ? 2u : 4u;     // 128B : 64B swizzle
-  static constexpr uint32_t SBO = 8 * BK * 2;               // bytes between 8-row atoms
-};
+constexpr int kStages = 6;
+constexpr int kABytes = BM * 64 * 2;         // A slot (BK <= 64)
+constexpr int kBBytes = 128 * 64 * 2;        // B slot (BN <= 128, BK <= 64)
+constexpr int kStageBytes = kABytes + kBBytes;
+constexpr int kStagingBytes = BM * 128 * 2;  // output tile (BN <= 128)
+constexpr int kSmem = kStages * kStageBytes + kStagingBytes + 1024 + 256;
+constexpr uint32_t kTmemCols = 256;          // two 128-column accumulators
 
 // bias + ReLU of 16 fp32 columns [c0, c0+16) of tile row `row`, packed to
 // 16 bits and written to the staging tile.  Channels are staged in groups of
-// SG (64 or 32): group g is a [BM][SG] block with SG*2-byte rows in the
-// 128-byte (SG = 64) or 64-byte (SG = 32) swizzle of the store tensor map, so
+// sg (64 or 32): group g is a [BM][sg] block with sg*2-byte rows in the
+// 128-byte (sg = 64) or 64-byte (sg = 32) swizzle of the store tensor map, so
 // a warp's 16-byte writes spread over all banks.
-template <typename T, int SG>
-__device__ __forceinline__ void stage16(uint8_t* stage, int row, int c0, const float* v,
+template <typename T>
+__device__ __forceinline__ void stage16(uint8_t* stage, int sg, int row, int c0, const float* v,
                                         const float* bias) {
   uint32_t pk[8];
 #pragma unroll
   for (int j = 0; j < 8; ++j)
     pk[j] = Store<T>::pack2(relu_f(v[2 * j] + bias[2 * j]), relu_f(v[2 * j + 1] + bias[2 * j + 1]));
-  constexpr int RB = SG * 2;                           // bytes per staged row
-  uint8_t* base = stage + (c0 / SG) * (BM * RB) + row * RB;
-  const int j0 = (c0 % SG) / 8;                        // 16-byte chunk within the row
-  const int x = (SG == 64) ? (row & 7) : ((row >> 1) & 3);
+  const int rb = sg * 2;                               // bytes per staged row
+  uint8_t* base = stage + (c0 / sg) * (BM * rb) + row * rb;
+  const int j0 = (c0 % sg) / 8;                        // 16-byte chunk within the row
+  const int x = (sg == 64) ? (row & 7) : ((row >> 1) & 3);
   *reinterpret_cast<uint4*>(base + ((j0 ^ x) << 4)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
   *reinterpret_cast<uint4*>(base + (((j0 + 1) ^ x) << 4)) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
 }
@@ -83,220 +82,405 @@ __device__ __forceinline__ void stage16(uint8_t* stage, int row, int c0, const f
 // barrier among the 4 epilogue warps only (named barrier 1, 128 threads)
 __device__ __forceinline__ void epilogue_sync() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
-template <int KIND, int BN, int BK, typename T>
-__global__ void __launch_bounds__(kThreads, 1)
-k_conv_tc(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
-          const __grid_constant__ CUtensorMap mapC, const ConvArgs a) {
-  using G = Geo<BN, BK>;
-  constexpr int STAGES = G::STAGES;
-  constexpr int SG = BN < 64 ? BN : 64;          // channels per staged output group
-  static_assert(STAGES * G::A_BYTES >= BM * BN * 2, "staging tile must fit the A buffers");
+// Wait until the grid-wide arrival counter reaches `target` (bounded).
+__device__ __forceinline__ bool grid_wait(const unsigned* ctr, unsigned target) {
+  unsigned v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
+  if (v >= target) return true;
+  const long long t0 = clock64();
+  while (true) {
+    __nanosleep(64);
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
+    if (v >= target) return true;
+    if (clock64() - t0 > kWaitBudgetCycles) return false;
+  }
+}
+
+// The scalars of one layer, read once per layer into registers.  The layer
+// table lives in kernel parameter space and is indexed by the (dynamic) layer
+// number; re-reading its fields inside the k-loops (every asm statement with a
+// memory clobber forces a reload) costs a constant-cache round trip each.
+struct LayerScalars {
+  const float* bias;
+  float* ws;
+  int* counters;
+  int kind, cin, cout, s, bn, bk, splits;
+  int tiles_x, m_tiles, n_tiles, choff, wait_layers;
+  int n_items, total_kb;
+};
+__device__ __forceinline__ LayerScalars layer_scalars(const LayerDesc& D) {
+  LayerScalars S;
+  S.bias = D.bias;
+  S.ws = D.ws;
+  S.counters = D.counters;
+  S.kind = D.kind;
+  S.cin = D.cin;
+  S.cout = D.cout;
+  S.s = D.s;
+  S.bn = D.bn;
+  S.bk = D.bk;
+  S.splits = D.splits;
+  S.tiles_x = D.tiles_x;
+  S.m_tiles = D.m_tiles;
+  S.n_tiles = D.n_tiles;
+  S.choff = D.choff;
+  S.wait_layers = D.wait_layers;
+  S.n_items = S.m_tiles * S.n_tiles * S.splits;
+  S.total_kb = (S.kind == DECONV ? 1 : 9) * (S.cin / S.bk);
+  return S;
+}
+
+// Work item t of a layer -> (m tile, n tile, K slice), its tile origin and
+// its k-block range [kb0, kb1).
+struct Item {
+  int x0, y0, n0, z, kb0, kb1;
+};
+__device__ __forceinline__ Item item_of(const LayerScalars& S, int t) {
+  Item it;
+  const int mt = t % S.m_tiles;
+  const int r = t / S.m_tiles;
+  const int nt = r % S.n_tiles;
+  it.z = r / S.n_tiles;
+  it.x0 = (mt % S.tiles_x) * TW;
+  it.y0 = (mt / S.tiles_x) * TH;
+  it.n0 = nt * S.bn;
+  it.kb0 = (it.z * S.total_kb) / S.splits;
+  it.kb1 = ((it.z + 1) * S.total_kb) / S.splits;
+  return it;
+}
+
+// TMA load of the activation (A) box of k-block kb of item I.
+__device__ __forceinline__ void load_a(const LayerScalars& S, const CUtensorMap* map, uint8_t* dA,
+                                       uint64_t* bar, const Item& I, int kb) {
+  const int ncb = S.cin / S.bk;
+  const int tap = kb / ncb;
+  const int cb = kb - tap * ncb;
+  if (S.kind == CONV3_S1) {
+    const int dy = tap / 3, dx = tap - 3 * (tap / 3);
+    tma_load_4d(dA, map, bar, cb * S.bk, I.x0 + dx - 1, I.y0 + dy - 1, 0);
+  } else if (S.kind == CONV3_S2) {
+    // input x = 2*ox + dx - 1 = 2*j + p; input y = 2*oy + dy - 1 = 2*i + q
+    const int dy = tap / 3, dx = tap - 3 * (tap / 3);
+    const int j = I.x0 + (dx == 0 ? -1 : 0);
+    const int p = (dx == 1) ? 0 : 1;
+    const int i = I.y0 + (dy == 0 ? -1 : 0);
+    const int q = (dy == 1) ? 0 : 1;
+    tma_load_5d(dA, map, bar, p * S.cin + cb * S.bk, j, q, i, 0);
+  } else {
+    tma_load_4d(dA, map, bar, cb * S.bk, I.x0, I.y0, 0);
+  }
+}
+
+// TMA load of the weight (B) box of k-block kb of item I.
+__device__ __forceinline__ void load_b(const LayerScalars& S, const CUtensorMap* map, uint8_t* dB,
+                                       uint64_t* bar, const Item& I, int kb) {
+  const int ncb = S.cin / S.bk;
+  const int tap = kb / ncb;
+  const int cb = kb - tap * ncb;
+  tma_load_2d(dB, map, bar, tap * S.cin + cb * S.bk, I.n0);
+}
+
+// One k-block of MMAs (BK = 64 or 32 -> 4 or 2 MMAs of K = 16) from
+// precomputed descriptors; advancing K by 16 elements = 32 bytes = +2 in the
+// descriptors' 16-byte address field (the start stays inside the stage).
+__device__ __forceinline__ void mma_kblock(uint32_t d_tmem, uint64_t ad, uint64_t bd, uint32_t idesc,
+                                           uint32_t acc0, bool bk64) {
+  umma_f16(d_tmem, ad, bd, idesc, acc0);
+  umma_f16(d_tmem, ad + 2, bd + 2, idesc, 1u);
+  if (bk64) {
+    umma_f16(d_tmem, ad + 4, bd + 4, idesc, 1u);
+    umma_f16(d_tmem, ad + 6, bd + 6, idesc, 1u);
+  }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant__ BackboneParams P) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint8_t* sA = smem;
-  uint8_t* sB = smem + STAGES * G::A_BYTES;
-  uint64_t* full = reinterpret_cast<uint64_t*>(sB + STAGES * G::B_BYTES);
-  uint64_t* empty = full + STAGES;
-  uint64_t* accum = empty + STAGES;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accum + 1);
+  uint8_t* stage = smem + kStages * kStageBytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(stage + kStagingBytes);
+  uint64_t* empty = full + kStages;
+  uint64_t* accfull = empty + kStages;         // [2]
+  uint64_t* accempty = accfull + 2;            // [2]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accempty + 2);
+  __shared__ int s_last;
+  __shared__ float s_bias[2][128];             // bias of the tile in each accumulator
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int tile = blockIdx.x;
-  const int x0 = (tile % a.tiles_x) * TW;
-  const int y0 = (tile / a.tiles_x) * TH;
-  const int n0 = blockIdx.y * BN;
-  const int ncb = a.cin / BK;
-  const int total_kb = (KIND == DECONV ? 1 : 9) * ncb;
-  // this CTA's slice of the K loop (all of it without split-K)
-  const int z = blockIdx.z;
-  const int kb_begin = (z * total_kb) / a.splits;
-  const int num_kb = ((z + 1) * total_kb) / a.splits - kb_begin;
+  const unsigned G = gridDim.x;
 
   if (warp == 0 && lane == 0) {
-    tma_prefetch_desc(&mapA);
-    tma_prefetch_desc(&mapB);
-    tma_prefetch_desc(&mapC);
-    for (int s = 0; s < STAGES; ++s) {
+    for (int s = 0; s < kStages; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
-    mbar_init(accum, 1);
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&accfull[a], 1);
+      mbar_init(&accempty[a], 4);              // one arrival per epilogue warp
+    }
     fence_barrier_init();
   }
   if (warp == 1) {
-    tmem_alloc(tmem_slot, G::TMEM_COLS);
+    tmem_alloc(tmem_slot, kTmemCols);
     tmem_relinquish();
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  // the prologue above overlapped the previous layer; from here on this CTA
-  // reads its input and writes its output
   pdl_trigger();
-  pdl_wait();
+  pdl_wait();                                  // the pseudo-image is the previous kernel's output
 
   if (warp == 0) {
     if (lane == 0) {
       // ---------------- TMA producer ----------------
-      for (int it = 0; it < num_kb; ++it) {
-        const int s = it % STAGES;
-        const uint32_t ph = (it / STAGES) & 1;
-        if (!mbar_wait(&empty[s], ph ^ 1)) {
-          atomicOr(a.err, ERR_WAIT_PRODUCER);
-          break;
+      uint32_t it = 0;
+      bool alive = true;
+      for (int l = 0; l < P.n_layers && alive; ++l) {
+        const LayerDesc& D = P.L[l];
+        const LayerScalars S = layer_scalars(D);
+        const CUtensorMap* mapA = &D.mapA;
+        const CUtensorMap* mapB = &D.mapB;
+        tma_prefetch_desc(mapA);
+        tma_prefetch_desc(mapB);
+        const uint32_t bytes = (uint32_t)(BM + S.bn) * S.bk * 2;
+        // The weights do not depend on the previous layer: load the B boxes
+        // of the first k-blocks of this CTA's first item before waiting for
+        // the layer's input, so only the A boxes remain after the wait.
+        int npre = 0;
+        Item I0{};
+        if ((int)blockIdx.x < S.n_items) {
+          I0 = item_of(S, blockIdx.x);
+          npre = I0.kb1 - I0.kb0;
+          if (npre > kStages) npre = kStages;
+          for (int j = 0; j < npre; ++j) {
+            const uint32_t u = it + j;
+            const int s = u % kStages;
+            if (!mbar_wait(&empty[s], ((u / kStages) & 1) ^ 1)) {
+              atomicOr(P.err, ERR_WAIT_PRODUCER);
+              alive = false;
+              break;
+            }
+            mbar_arrive_expect_tx(&full[s], bytes);
+            load_b(S, mapB, smem + s * kStageBytes + kABytes, &full[s], I0, I0.kb0 + j);
+          }
+          if (!alive) break;
         }
-        const int kb = kb_begin + it;
-        const int tap = kb / ncb;
-        const int cb = kb - tap * ncb;
-        mbar_arrive_expect_tx(&full[s], G::STAGE_BYTES);
-        void* dA = sA + s * G::A_BYTES;
-        void* dB = sB + s * G::B_BYTES;
-        if (KIND == CONV3_S1) {
-          const int dy = tap / 3, dx = tap - 3 * (tap / 3);
-          tma_load_4d(dA, &mapA, &full[s], cb * BK, x0 + dx - 1, y0 + dy - 1, 0);
-        } else if (KIND == CONV3_S2) {
-          // input x = 2*ox + dx - 1 = 2*j + p; input y = 2*oy + dy - 1 = 2*i + q
-          const int dy = tap / 3, dx = tap - 3 * (tap / 3);
-          const int j = x0 + (dx == 0 ? -1 : 0);
-          const int p = (dx == 1) ? 0 : 1;
-          const int i = y0 + (dy == 0 ? -1 : 0);
-          const int q = (dy == 1) ? 0 : 1;
-          tma_load_5d(dA, &mapA, &full[s], p * a.cin + cb * BK, j, q, i, 0);
-        } else {
-          tma_load_4d(dA, &mapA, &full[s], cb * BK, x0, y0, 0);
+        if (S.wait_layers > 0) {
+          // every CTA has finished layer wait_layers - 1 (and, as each CTA
+          // runs its layers in order, every layer before it)
+          if (!grid_wait(&P.grid_bar[S.wait_layers - 1], G)) {
+            atomicOr(P.err, ERR_WAIT_PRODUCER);
+            alive = false;
+            break;
+          }
+          fence_async_global();
         }
-        tma_load_2d(dB, &mapB, &full[s], tap * a.cin + cb * BK, n0);
+        if (P.stamps && blockIdx.x == 0) P.stamps[l] = global_ns();
+        for (int t = blockIdx.x; t < S.n_items && alive; t += G) {
+          const Item I = (t == (int)blockIdx.x) ? I0 : item_of(S, t);
+          for (int kb = I.kb0; kb < I.kb1; ++kb, ++it) {
+            const int s = it % kStages;
+            uint8_t* dA = smem + s * kStageBytes;
+            if (t == (int)blockIdx.x && kb - I.kb0 < npre) {
+              load_a(S, mapA, dA, &full[s], I, kb);    // B already in flight
+              continue;
+            }
+            if (!mbar_wait(&empty[s], ((it / kStages) & 1) ^ 1)) {
+              atomicOr(P.err, ERR_WAIT_PRODUCER);
+              alive = false;
+              break;
+            }
+            mbar_arrive_expect_tx(&full[s], bytes);
+            load_a(S, mapA, dA, &full[s], I, kb);
+            load_b(S, mapB, dA + kABytes, &full[s], I, kb);
+          }
+        }
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
       // ---------------- MMA issuer ----------------
-      constexpr uint32_t IDESC = idesc_f16(BM, BN, std::is_same<T, __nv_bfloat16>::value);
-      for (int kb = 0; kb < num_kb; ++kb) {
-        const int s = kb % STAGES;
-        const uint32_t ph = (kb / STAGES) & 1;
-        if (!mbar_wait(&full[s], ph)) {
-          atomicOr(a.err, ERR_WAIT_MMA);
-          break;
+      uint32_t it = 0, tc = 0;
+      bool alive = true;
+      const uint32_t smem0 = smem_u32(smem);
+      for (int l = 0; l < P.n_layers && alive; ++l) {
+        const LayerScalars S = layer_scalars(P.L[l]);
+        const uint32_t idesc = idesc_f16(BM, S.bn, std::is_same<T, __nv_bfloat16>::value);
+        const bool bk64 = S.bk == 64;
+        const uint32_t swz = bk64 ? 2u : 4u;          // 128B : 64B swizzle
+        const uint32_t sbo = 8u * S.bk * 2u;          // bytes between 8-row atoms
+        for (int t = blockIdx.x; t < S.n_items && alive; t += G, ++tc) {
+          const Item I = item_of(S, t);
+          const int acc = tc & 1;
+          if (!mbar_wait(&accempty[acc], ((tc >> 1) & 1) ^ 1)) {
+            atomicOr(P.err, ERR_WAIT_MMA);
+            alive = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t d_tmem = tmem + acc * 128;
+          for (int kb = I.kb0; kb < I.kb1; ++kb, ++it) {
+            const int s = it % kStages;
+            if (!mbar_wait(&full[s], (it / kStages) & 1)) {
+              atomicOr(P.err, ERR_WAIT_MMA);
+              alive = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t aa = smem0 + s * kStageBytes;
+            mma_kblock(d_tmem, smem_desc(aa, sbo, swz), smem_desc(aa + kABytes, sbo, swz), idesc,
+                       kb > I.kb0 ? 1u : 0u, bk64);
+            umma_commit(&empty[s]);
+          }
+          umma_commit(&accfull[acc]);
         }
-        tc_fence_after();
-        const uint32_t aa = smem_u32(sA + s * G::A_BYTES);
-        const uint32_t bb = smem_u32(sB + s * G::B_BYTES);
-#pragma unroll
-        for (int k = 0; k < BK / 16; ++k) {
-          umma_f16(tmem, smem_desc(aa + k * 32, G::SBO, G::SWZ),
-                   smem_desc(bb + k * 32, G::SBO, G::SWZ), IDESC, (kb | k) != 0);
-        }
-        umma_commit(&empty[s]);
       }
-      umma_commit(accum);
     }
   } else {
     // ---------------- epilogue ----------------
-    // accumulator -> bias + ReLU -> 16-bit, staged in shared memory in the
-    // store map's swizzled layout, then written by TMA tensor stores (full
-    // lines; rows outside the image are clipped by the store)
-    const int qd = warp & 3;                 // tensor-memory lane quarter of this warp
-    const int row = qd * 32 + lane;          // pixel within the tile
-    const bool ok = mbar_wait(accum, 0);
-    if (!ok && lane == 0) atomicOr(a.err, ERR_WAIT_EPILOGUE);
-    tc_fence_after();
-    const float* bias = a.bias + (KIND == DECONV ? 0 : n0);
-    const uint32_t taddr = tmem + (static_cast<uint32_t>(qd * 32) << 16);
-    uint8_t* stage = sA;                     // pipeline buffers are idle once the MMAs are done
-    bool store = true;
-    if (a.splits == 1) {
-#pragma unroll
-      for (int c0 = 0; c0 < BN; c0 += 16) {
-        float v[16];
-        tmem_ld16(taddr + c0, v);
-        stage16<T, SG>(stage, row, c0, v, bias + c0);
-      }
-    } else {
-      // split-K: publish this slice's fp32 partial, then the last CTA of the
-      // tile sums the slices in slice order (deterministic) and stores
-      // workspace layout per (slice, tile): [BN/4 column quads][BM rows][4],
-      // so a warp's float4 stores cover 512 contiguous bytes
-      const int tiles = gridDim.x * gridDim.y;
-      const int tile_id = blockIdx.y * gridDim.x + blockIdx.x;
-      float4* mine = reinterpret_cast<float4*>(a.ws + (size_t)(z * tiles + tile_id) * BM * BN) + row;
-#pragma unroll
-      for (int c0 = 0; c0 < BN; c0 += 16) {
-        float v[16];
-        tmem_ld16(taddr + c0, v);
-#pragma unroll
-        for (int q = 0; q < 4; ++q)
-          mine[(c0 / 4 + q) * BM] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-      }
-      __threadfence();
-      epilogue_sync();
-      __shared__ int s_last;
-      if (row == 0) {
-        const int old = atomicAdd(&a.counters[tile_id], 1);
-        s_last = (old == a.splits - 1);
-      }
-      epilogue_sync();
-      store = s_last != 0;
-      if (store) {
-        __threadfence();
-#pragma unroll
-        for (int c0 = 0; c0 < BN; c0 += 16) {
-          float acc[16];
-#pragma unroll
-          for (int j = 0; j < 16; ++j) acc[j] = 0.f;
-          for (int zz = 0; zz < a.splits; ++zz) {
-            float v[16];
-            if (zz == z) {
-              tmem_ld16(taddr + c0, v);
-            } else {
-              const float4* src =
-                  reinterpret_cast<const float4*>(a.ws + (size_t)(zz * tiles + tile_id) * BM * BN) +
-                  row;
-#pragma unroll
-              for (int q = 0; q < 4; ++q) {
-                const float4 f = __ldcg(src + (c0 / 4 + q) * BM);
-                v[4 * q] = f.x; v[4 * q + 1] = f.y; v[4 * q + 2] = f.z; v[4 * q + 3] = f.w;
-              }
-            }
-#pragma unroll
-            for (int j = 0; j < 16; ++j) acc[j] += v[j];
-          }
-          stage16<T, SG>(stage, row, c0, acc, bias + c0);
+    const int qd = warp & 3;                   // tensor-memory lane quarter of this warp
+    const int row = qd * 32 + lane;            // pixel within the tile
+    // The four epilogue warps meet at named barriers, so they never leave the
+    // loops early: after a wait runs out they skip further waits (the values
+    // are then garbage, the error word says so) but keep the same sequence of
+    // barriers and grid arrivals.
+    uint32_t tc = 0;
+    bool alive = true;
+    for (int l = 0; l < P.n_layers; ++l) {
+      const LayerDesc& D = P.L[l];
+      const LayerScalars S = layer_scalars(D);
+      const CUtensorMap* mapC = &D.mapC;
+      const int sg = S.bn < 64 ? S.bn : 64;    // channels per staged store box
+      for (int t = blockIdx.x; t < S.n_items; t += G, ++tc) {
+        const Item I = item_of(S, t);
+        const int acc = tc & 1;
+        // bias of this tile, read while the MMAs run (the slot was last read
+        // two tiles ago, before the barriers in between)
+        if (row < S.bn) s_bias[acc][row] = S.bias[(S.kind == DECONV ? 0 : I.n0) + row];
+        if (alive && !mbar_wait(&accfull[acc], (tc >> 1) & 1)) {
+          if (lane == 0) atomicOr(P.err, ERR_WAIT_EPILOGUE);
+          alive = false;
         }
-        if (row == 0) a.counters[tile_id] = 0;       // ready for the next launch
+        tc_fence_after();
+        const float* bias = s_bias[acc];
+        const uint32_t taddr = tmem + acc * 128 + (static_cast<uint32_t>(qd * 32) << 16);
+        // the previous tile's stores must have read the staging buffer
+        if (row == 0) bulk_wait_read_all();
+        epilogue_sync();
+        bool store = true;
+        if (S.splits == 1) {
+          for (int c0 = 0; c0 < S.bn; c0 += 16) {
+            float v[16];
+            tmem_ld16(taddr + c0, v);
+            stage16<T>(stage, sg, row, c0, v, bias + c0);
+          }
+        } else {
+          // publish this slice's fp32 partial ([bn/4][BM][4] per (slice, tile),
+          // so a warp's float4 stores cover 512 contiguous bytes), then the
+          // last slice of the tile sums the slices in slice order
+          const int tiles = S.m_tiles * S.n_tiles;
+          const int tile_id = t % tiles;
+          float4* mine =
+              reinterpret_cast<float4*>(S.ws + (size_t)(I.z * tiles + tile_id) * BM * S.bn) + row;
+          for (int c0 = 0; c0 < S.bn; c0 += 16) {
+            float v[16];
+            tmem_ld16(taddr + c0, v);
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+              mine[(c0 / 4 + q) * BM] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+          }
+          __threadfence();
+          epilogue_sync();
+          if (row == 0) {
+            const int old = atomicAdd(&S.counters[tile_id], 1);
+            s_last = (old == S.splits - 1);
+          }
+          epilogue_sync();
+          store = s_last != 0;
+          if (store) {
+            __threadfence();
+            for (int c0 = 0; c0 < S.bn; c0 += 16) {
+              // all other slices' loads of this column group in flight at once
+              float4 f[kMaxSplits][4];
+#pragma unroll
+              for (int zz = 0; zz < kMaxSplits; ++zz) {
+                if (zz < S.splits && zz != I.z) {
+                  const float4* src =
+                      reinterpret_cast<const float4*>(S.ws + (size_t)(zz * tiles + tile_id) * BM * S.bn) +
+                      row;
+#pragma unroll
+                  for (int q = 0; q < 4; ++q) f[zz][q] = __ldcg(src + (c0 / 4 + q) * BM);
+                }
+              }
+              float v[16];
+              tmem_ld16(taddr + c0, v);
+              float sum[16];
+#pragma unroll
+              for (int j = 0; j < 16; ++j) sum[j] = 0.f;
+#pragma unroll
+              for (int zz = 0; zz < kMaxSplits; ++zz) {
+                if (zz < S.splits) {
+                  if (zz == I.z) {
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) sum[j] += v[j];
+                  } else {
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                      sum[4 * q] += f[zz][q].x;
+                      sum[4 * q + 1] += f[zz][q].y;
+                      sum[4 * q + 2] += f[zz][q].z;
+                      sum[4 * q + 3] += f[zz][q].w;
+                    }
+                  }
+                }
+              }
+              stage16<T>(stage, sg, row, c0, sum, bias + c0);
+            }
+            if (row == 0) S.counters[tile_id] = 0;     // ready for the next launch
+          }
+        }
+        // the accumulator has been read: hand it back to the MMA issuer
+        tc_fence_before();
+        if (lane == 0) mbar_arrive(&accempty[acc]);
+        if (store) {
+          fence_async_smem();
+          epilogue_sync();
+          if (row == 0) {
+            const int GB = BM * sg * 2;                // bytes of one staged channel group
+            if (S.kind == DECONV) {
+              const int sub = I.n0 / S.cout;
+              const int sy = sub / S.s, sx = sub - sy * S.s;
+              for (int g = 0; g < S.bn / sg; ++g)
+                tma_store_5d(mapC, stage + g * GB, S.choff + g * sg, sx, I.x0, sy, I.y0);
+            } else {
+              for (int g = 0; g < S.bn / sg; ++g)
+                tma_store_3d(mapC, stage + g * GB, I.n0 + g * sg, I.x0, I.y0);
+            }
+            bulk_commit();
+          }
+        }
+      }
+      // this CTA's part of layer l is written: count it in the grid barrier
+      if (row == 0) {
+        bulk_wait_all();
+        fence_async_global();
+        __threadfence();
+        atomicAdd(&P.grid_bar[l], 1u);
       }
     }
-    if (store) {                                     // uniform over the epilogue warps
-      fence_async_smem();
-      epilogue_sync();
-      if (row == 0 && ok) {
-        constexpr int GB = BM * SG * 2;              // bytes of one staged channel group
-        if (KIND == DECONV) {
-          const int sub = n0 / a.cout;
-          const int sy = sub / a.s, sx = sub - sy * a.s;
-#pragma unroll
-          for (int g = 0; g < BN / SG; ++g)
-            tma_store_5d(&mapC, stage + g * GB, a.choff + g * SG, sx, x0, sy, y0);
-        } else {
-#pragma unroll
-          for (int g = 0; g < BN / SG; ++g) tma_store_3d(&mapC, stage + g * GB, n0 + g * SG, x0, y0);
-        }
-        bulk_commit();
-        bulk_wait_all();
-      }
+    if (row == 0 && P.stamps && blockIdx.x == 0) {
+      if (grid_wait(&P.grid_bar[P.n_layers - 1], G)) P.stamps[P.n_layers] = global_ns();
     }
   }
 
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
-    // every MMA this CTA issued has retired before its accumulator is freed
-    mbar_wait(accum, 0);
     tc_fence_after();
-    tmem_dealloc(tmem, G::TMEM_COLS);
+    tmem_dealloc(tmem, kTmemCols);
   }
 }
 
@@ -321,52 +505,6 @@ EncodeFn encode_fn() {
       fn = reinterpret_cast<EncodeFn>(p);
   });
   return fn;
-}
-
-template <int KIND, int BN, int BK, typename T>
-cudaError_t launch_t(const ConvLayer& L, int* err, cudaStream_t st) {
-  using G = Geo<BN, BK>;
-  static std::once_flag once;
-  static cudaError_t attr_err = cudaSuccess;
-  std::call_once(once, [] {
-    attr_err = cudaFuncSetAttribute(k_conv_tc<KIND, BN, BK, T>,
-                                    cudaFuncAttributeMaxDynamicSharedMemorySize, G::SMEM);
-  });
-  if (attr_err != cudaSuccess) return attr_err;
-  ConvArgs a;
-  a.bias = L.bias;
-  a.out = L.out;
-  a.gw = L.gw;
-  a.gh = L.gh;
-  a.out_w = L.out_w;
-  a.ldc = L.ldc;
-  a.choff = L.choff;
-  a.cin = L.cin;
-  a.cout = L.cout;
-  a.s = L.s;
-  a.tiles_x = (L.gw + TW - 1) / TW;
-  a.splits = L.splits < 1 ? 1 : L.splits;
-  a.ws = L.ws;
-  a.counters = L.counters;
-  a.err = err;
-  const int tiles_y = (L.gh + TH - 1) / TH;
-  dim3 grid(a.tiles_x * tiles_y, L.n_tiles_n, a.splits);
-  return launch_pdl(k_conv_tc<KIND, BN, BK, T>, grid, dim3(kThreads), G::SMEM, st, L.mapA, L.mapB,
-                    L.mapC, a);
-}
-
-template <int KIND, typename T>
-cudaError_t launch_kind(const ConvLayer& L, int* err, cudaStream_t st) {
-  if (L.bk == 64) {
-    if (L.bn == 128) return launch_t<KIND, 128, 64, T>(L, err, st);
-    if (L.bn == 64) return launch_t<KIND, 64, 64, T>(L, err, st);
-    if (L.bn == 32) return launch_t<KIND, 32, 64, T>(L, err, st);
-  } else if (L.bk == 32) {
-    if (L.bn == 128) return launch_t<KIND, 128, 32, T>(L, err, st);
-    if (L.bn == 64) return launch_t<KIND, 64, 32, T>(L, err, st);
-    if (L.bn == 32) return launch_t<KIND, 32, 32, T>(L, err, st);
-  }
-  return cudaErrorInvalidValue;
 }
 
 }  // namespace
@@ -438,26 +576,72 @@ cudaError_t conv_make_maps(ConvLayer& L, bool bf16) {
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-cudaError_t launch_conv(const ConvLayer& L, bool bf16, int* err, cudaStream_t st) {
-  if (L.cin % L.bk || (L.kind != DECONV && L.cout % L.bn) ||
-      (L.kind == DECONV && L.bn != L.cout))
-    return cudaErrorInvalidValue;
-  const int total_kb = (L.kind == DECONV ? 1 : 9) * (L.cin / L.bk);
-  if (L.splits > 1 && (!L.ws || !L.counters || L.splits > total_kb)) return cudaErrorInvalidValue;
-  if (bf16) {
-    switch (L.kind) {
-      case CONV3_S1: return launch_kind<CONV3_S1, __nv_bfloat16>(L, err, st);
-      case CONV3_S2: return launch_kind<CONV3_S2, __nv_bfloat16>(L, err, st);
-      case DECONV: return launch_kind<DECONV, __nv_bfloat16>(L, err, st);
-    }
-  } else {
-    switch (L.kind) {
-      case CONV3_S1: return launch_kind<CONV3_S1, __half>(L, err, st);
-      case CONV3_S2: return launch_kind<CONV3_S2, __half>(L, err, st);
-      case DECONV: return launch_kind<DECONV, __half>(L, err, st);
-    }
+cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, unsigned* grid_bar, int* err,
+                          unsigned long long* stamps, BackboneParams* P) {
+  if (layers.empty() || layers.size() > (size_t)kMaxLayers) return cudaErrorInvalidValue;
+  std::memset(P, 0, sizeof(*P));
+  P->n_layers = (int)layers.size();
+  P->grid_bar = grid_bar;
+  P->err = err;
+  P->stamps = stamps;
+  for (size_t i = 0; i < layers.size(); ++i) {
+    const ConvLayer& L = layers[i];
+    if (L.cin % L.bk || (L.kind != DECONV && L.cout % L.bn) ||
+        (L.kind == DECONV && L.bn != L.cout) || L.bn > 128 || L.bk > 64 || L.bn % 32)
+      return cudaErrorInvalidValue;
+    const int total_kb = (L.kind == DECONV ? 1 : 9) * (L.cin / L.bk);
+    if (L.splits < 1 || L.splits > kMaxSplits || L.splits > total_kb || (L.splits > 1 && (!L.ws || !L.counters)))
+      return cudaErrorInvalidValue;
+    LayerDesc& D = P->L[i];
+    D.mapA = L.mapA;
+    D.mapB = L.mapB;
+    D.mapC = L.mapC;
+    D.bias = L.bias;
+    D.ws = L.ws;
+    D.counters = L.counters;
+    D.kind = L.kind;
+    D.cin = L.cin;
+    D.cout = L.cout;
+    D.s = L.s;
+    D.bn = L.bn;
+    D.bk = L.bk;
+    D.splits = L.splits;
+    D.tiles_x = (L.gw + TW - 1) / TW;
+    D.m_tiles = D.tiles_x * ((L.gh + TH - 1) / TH);
+    D.n_tiles = L.n_tiles_n;
+    D.choff = L.choff;
+    D.wait_layers = L.wait_layers;
   }
-  return cudaErrorInvalidValue;
+  return cudaSuccess;
+}
+
+cudaError_t launch_backbone(const BackboneParams& P, bool bf16, cudaStream_t st) {
+  static std::once_flag once;
+  static cudaError_t attr_err = cudaSuccess;
+  std::call_once(once, [] {
+    attr_err = cudaFuncSetAttribute(k_backbone<__half>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    kSmem);
+    if (attr_err == cudaSuccess)
+      attr_err = cudaFuncSetAttribute(k_backbone<__nv_bfloat16>,
+                                      cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
+  });
+  if (attr_err != cudaSuccess) return attr_err;
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (sms < 1) return cudaErrorInvalidValue;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(sms);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = kSmem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;   // every CTA resident: grid barriers are safe
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (bf16) return cudaLaunchKernelEx(&cfg, k_backbone<__nv_bfloat16>, P);
+  return cudaLaunchKernelEx(&cfg, k_backbone<__half>, P);
 }
 
 }  // namespace rtcc

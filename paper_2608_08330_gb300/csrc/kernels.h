@@ -5,6 +5,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <vector>
+
 #include "rtcc.h"
 
 namespace rtcc {
@@ -84,9 +86,10 @@ struct ConvLayer {
   int out_w, out_h;      // output map
   int gw, gh;            // M grid the tiles cover (conv: output; deconv: input)
   int ldc, choff;        // output pixel stride (channels) and channel offset
-  int bn, bk;            // N tile (output channels per CTA), K chunk (channels)
-  int n_tiles_n;         // grid.y
-  int splits;            // split-K factor (grid.z); 1 = none
+  int bn, bk;            // N tile (output channels per item), K chunk (channels)
+  int n_tiles_n;         // N tiles
+  int splits;            // split-K factor; 1 = none
+  int wait_layers;       // this layer reads outputs of layers [0, wait_layers)
   float* ws;             // split-K partials [splits][m_tiles * n_tiles][128][bn] fp32
   int* counters;         // split-K arrivals per tile [m_tiles * n_tiles], zero-initialised
   const void* in;        // device [in_h][in_w][cin]
@@ -98,10 +101,36 @@ struct ConvLayer {
 
 // Encode the layer's tensor maps (input activations, packed weights, output).
 cudaError_t conv_make_maps(ConvLayer& L, bool bf16);
-cudaError_t launch_conv(const ConvLayer& L, bool bf16, int* err, cudaStream_t st);
 int conv_tile_w();
 int conv_tile_h();
 int conv_tile_m();
+
+// One layer of the persistent backbone kernel (kernel-parameter layout).
+constexpr int kMaxLayers = 20;
+constexpr int kMaxSplits = 4;     // split-K slices per tile (the reducing slice keeps one load per slice in flight)
+struct alignas(128) LayerDesc {   // CUtensorMap is 128-byte aligned
+  CUtensorMap mapA, mapB, mapC;
+  const float* bias;
+  float* ws;
+  int* counters;
+  int kind, cin, cout, s, bn, bk, splits;
+  int tiles_x, m_tiles, n_tiles, choff;
+  int wait_layers;
+};
+struct BackboneParams {
+  LayerDesc L[kMaxLayers];
+  int n_layers;
+  unsigned* grid_bar;            // [kMaxLayers] per-layer arrival counters, zero before each launch
+  int* err;
+  unsigned long long* stamps;    // optional [n_layers + 1] layer-start times (ns)
+};
+
+// Fill the kernel parameters of a branch's backbone from its layer list;
+// grid_bar holds kMaxLayers counters.
+cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, unsigned* grid_bar, int* err,
+                          unsigned long long* stamps, BackboneParams* P);
+// One cooperative launch (one CTA per SM) running every layer.
+cudaError_t launch_backbone(const BackboneParams& P, bool bf16, cudaStream_t st);
 
 // ---------------------------------------------------------------------------
 // post-join: fusion + head, decode
