@@ -78,6 +78,7 @@ struct rtcc_ctx {
   std::vector<float*> bbufs;          // conv/deconv biases
   float* head_wp = nullptr;
   float* head_b = nullptr;
+  void* head_w16 = nullptr;   // head weights [16][C] in the storage type (tensor-core head)
   Branch br[RTCC_MAX_AGENTS];
   cudaStream_t xfer = nullptr, post = nullptr;
   cudaGraphExec_t post_exec = nullptr;
@@ -290,6 +291,10 @@ rtcc_status upload_weights(rtcc_ctx* c, const float* w) {
   permute_head_weights(hw.data(), c->Cf, hp.data());
   RS(dalloc(c, &c->head_wp, hp.size() * sizeof(float)));
   CK(cudaMemcpy(c->head_wp, hp.data(), hp.size() * sizeof(float), cudaMemcpyHostToDevice));
+  std::vector<uint16_t> h16(hw.size());
+  for (size_t i = 0; i < hw.size(); ++i) h16[i] = bits_store(hw[i], c->bf16);
+  RS(dalloc(c, &c->head_w16, h16.size() * sizeof(uint16_t)));
+  CK(cudaMemcpy(c->head_w16, h16.data(), h16.size() * sizeof(uint16_t), cudaMemcpyHostToDevice));
   o += (size_t)16 * c->Cf;
   RS(upload_f32(c, w + o, 16, &c->head_b));
   return RTCC_OK;
@@ -363,12 +368,22 @@ rtcc_status build_branch(rtcc_ctx* c, int k) {
       L.gh = oh;
       L.ldc = co;
       L.choff = 0;
-      // 128-wide N tiles unless that leaves most SMs idle (the small, deep
-      // layers of blocks 2 and 3): then 64-wide tiles double the CTA count
+      // N tile: the widest of 128/64/32 that gives about one tile per SM in
+      // a single wave
+      // (narrower tiles cost no more per MMA instruction than 64-wide ones,
+      // and they avoid split-K, whose cross-CTA reduction costs several
+      // dependent global round trips); 64 where even 32-wide tiles leave most
+      // SMs idle (the deepest block), which then splits K instead
+      int sms_avail = 148, dev_id = 0;
+      cudaGetDevice(&dev_id);
+      cudaDeviceGetAttribute(&sms_avail, cudaDevAttrMultiProcessorCount, dev_id);
       const int m_tiles = ((ow + conv_tile_w() - 1) / conv_tile_w()) *
                           ((oh + conv_tile_h() - 1) / conv_tile_h());
       L.bn = std::min(co, 128);
-      if (L.bn == 128 && m_tiles * (co / 128) < 120) L.bn = 64;
+      while (L.bn > 32 && m_tiles * (co / L.bn) < sms_avail * 3 / 4 &&
+             m_tiles * (co / L.bn) * 2 <= sms_avail)
+        L.bn /= 2;
+      if (m_tiles * (co / L.bn) < sms_avail / 2) L.bn = std::min(co, 64);
       L.bk = (cin >= 64) ? 64 : 32;
       L.n_tiles_n = co / L.bn;
       L.in = in;
@@ -530,6 +545,31 @@ rtcc_status capture_post(rtcc_ctx* c) {
   fa.hist0 = c->hist0;
   fa.cls_thresh = c->cfg.cls_thresh;
   fa.anchors = c->cfg.anchors;
+  // max fusion: tensor-core kernel (TMA-staged agent tiles, max in shared
+  // memory, head as an N = 16 MMA); attention fusion: CUDA-core kernel
+  const int bkc = fuse_tc_chunk(c->Cf, c->K);
+  const bool use_tc = !fa.attention && bkc > 0;
+  FuseTcParams tp{};
+  if (use_tc) {
+    const int swz = bkc * 2;                    // 128- or 64-byte rows
+    for (int k = 0; k < c->K; ++k)
+      CK(tmap_2d(&tp.feat[k], c->br[k].feat, c->bf16, (uint64_t)c->Cf, (uint64_t)fa.cells,
+                 (uint32_t)bkc, 128u, swz));
+    CK(tmap_2d(&tp.wmap, c->head_w16, c->bf16, (uint64_t)c->Cf, 16u, (uint32_t)bkc, 16u, swz));
+    tp.present = c->d_present;
+    tp.K = c->K;
+    tp.C = c->Cf;
+    tp.cells = fa.cells;
+    tp.bkc = bkc;
+    tp.head_b = c->head_b;
+    tp.head_out = c->head_out;
+    tp.fused = c->fused;
+    tp.keys = c->keys;
+    tp.hist0 = c->hist0;
+    tp.cls_thresh = c->cfg.cls_thresh;
+    tp.anchors = c->cfg.anchors;
+    tp.err = c->d_err;
+  }
   DecodeArgs da{};
   da.head = c->head_out;
   da.keys = c->keys;
@@ -549,7 +589,12 @@ rtcc_status capture_post(rtcc_ctx* c) {
   cudaError_t e = cudaSuccess;
   if (tl) e = record_node(c->ev_post0, c->post);
   if (e == cudaSuccess && tl) e = record_node(c->ev_fuse0, c->post);
-  if (e == cudaSuccess) e = launch_fuse_head(fa, c->bf16, c->post);
+  if (e == cudaSuccess) {
+    if (use_tc)
+      e = launch_fuse_max_head(tp, c->bf16, c->post);
+    else
+      e = launch_fuse_head(fa, c->bf16, c->post);
+  }
   if (e == cudaSuccess && tl) e = record_node(c->ev_fuse1, c->post);
   if (e == cudaSuccess) e = launch_decode(da, c->post);
   if (e == cudaSuccess)

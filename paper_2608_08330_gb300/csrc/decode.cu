@@ -6,16 +6,20 @@
 // logit (score = sigmoid(logit) is monotone), so the selection is an exact
 // function of the head output.  The fusion kernel leaves one 32-bit key per
 // anchor whose ascending order is descending logit order (0xFFFFFFFF below the
-// threshold).  One block selects the K = min(max_boxes, #valid) smallest
-// (key, index) pairs:
-//   1. radix select on the key in three levels (12, 10, 10 bits) finds the
-//      exact key T of the K-th pair and the count c of keys below T (the
-//      fusion kernel builds the first level's histogram with global atomics;
-//      the block builds the others in shared memory);
-//   2. one pass collects the c keys below T; an ordered pass (each thread owns
-//      a contiguous range of anchors, a block scan ranks its ties) adds the
-//      K - c keys equal to T with the smallest indices;
-//   3. the K pairs are sorted (bitonic, K <= 512) and decoded into boxes.
+// threshold), and a histogram of the keys' top 12 bits.  One block selects the
+// K = min(max_boxes, #valid) smallest (key, index) pairs:
+//   1. a scan of the histogram finds the bin b0 that holds the K-th key and
+//      the count c of keys in lower bins (c < K);
+//   2. one coalesced pass over the keys puts the c keys of lower bins into the
+//      selection and the keys of bin b0 into a shared-memory list;
+//   3. both are sorted (bitonic, in lockstep) and the K - c smallest pairs of
+//      bin b0 complete the selection, which is then already in order;
+//   4. the K pairs are decoded into boxes.
+// If bin b0 holds more keys than the list can take, a radix select refines
+// the threshold over the next 10 + 10 key bits instead (two more passes), the
+// keys below it are collected, and an ordered pass (each thread owns a
+// contiguous range of anchors, a block scan ranks its ties) adds the
+// lowest-index keys equal to it.
 #include <cmath>
 
 #include "common.cuh"
@@ -29,6 +33,7 @@ namespace {
 constexpr uint32_t kInvalid = 0xFFFFFFFFu;
 constexpr int kThreads = 1024;
 constexpr int kMaxBins = 4096;
+constexpr int kBndCap = 4096;                // keys of bin b0 held in shared memory
 
 struct AnchorGeo {
   float x_min, y_min, sx, sy;       // cell size in metres
@@ -90,24 +95,87 @@ __device__ __forceinline__ void for_chunk(const uint32_t* __restrict__ keys, int
   }
 }
 
+// Coalesced pass over the (padded) key array: thread t takes the 16-byte
+// vectors t, t + kThreads, ...; f(key, index).
+template <typename F>
+__device__ __forceinline__ void for_strided(const uint32_t* __restrict__ keys, int n4, F f) {
+  const uint4* v = reinterpret_cast<const uint4*>(keys);
+  constexpr int B = 4;                                   // loads in flight per thread
+  for (int base = threadIdx.x; base < n4; base += B * kThreads) {
+    uint4 r[B];
+#pragma unroll
+    for (int j = 0; j < B; ++j)
+      if (base + j * kThreads < n4) r[j] = v[base + j * kThreads];
+#pragma unroll
+    for (int j = 0; j < B; ++j) {
+      const int q = base + j * kThreads;
+      if (q < n4) {
+        f(r[j].x, 4 * q);
+        f(r[j].y, 4 * q + 1);
+        f(r[j].z, 4 * q + 2);
+        f(r[j].w, 4 * q + 3);
+      }
+    }
+  }
+}
+
+__device__ __forceinline__ void cmp_swap(unsigned long long* a, int i, int l, int k) {
+  const unsigned long long x = a[i], y = a[l];
+  if ((x > y) == ((i & k) == 0)) {
+    a[i] = y;
+    a[l] = x;
+  }
+}
+
+// Ascending bitonic sort of a[0..pa) and b[0..pb) (powers of two, padded with
+// ~0) in shared memory, the two in lockstep.
+__device__ void bitonic2(unsigned long long* a, int pa, unsigned long long* b, int pb) {
+  const int P = pa > pb ? pa : pb;
+  for (int k = 2; k <= P; k <<= 1) {
+    for (int j = k >> 1; j > 0; j >>= 1) {
+      for (int i = threadIdx.x; i < P; i += kThreads) {
+        const int l = i ^ j;
+        if (l > i) {
+          if (k <= pa) cmp_swap(a, i, l, k);
+          if (k <= pb) cmp_swap(b, i, l, k);
+        }
+      }
+      __syncthreads();
+    }
+  }
+}
+
+__device__ __forceinline__ int pow2_at_least(int n) {
+  int p = 1;
+  while (p < n) p <<= 1;
+  return p;
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
 k_decode_select(const uint32_t* __restrict__ keys, uint32_t* __restrict__ hist0,
                 const float* __restrict__ head, int chunk4, int max_boxes, AnchorGeo g,
                 const int* __restrict__ err, DetResultHeader* __restrict__ hdr,
                 rtcc_box* __restrict__ boxes) {
+  extern __shared__ unsigned long long bnd[];        // [kBndCap] keys of bin b0
   __shared__ int hist[kMaxBins];
   __shared__ unsigned long long sel[kDecodeKeep];
-  __shared__ int s_total, s_bin, s_below, s_nsel;
+  __shared__ int s_total, s_bin, s_below, s_nsel, s_nb;
   const int tid = threadIdx.x;
   const int lo = tid * chunk4 * 4;
+  const int n4 = chunk4 * kThreads;                   // 16-byte vectors of padded keys
   pdl_trigger();
   pdl_wait();
+  if (tid == 0) {
+    s_nsel = 0;
+    s_nb = 0;
+  }
 
-  // ---- 1. radix select: exact threshold key T and c = #keys < T ----------
-  // level 0 (top 12 bits) was histogrammed by the fusion kernel; the others
-  // (10 + 10 bits) are built here over the keys that match the prefix so far.
+  // ---- 1. threshold bin from the top-12-bit histogram (level 0); when that
+  // bin is too full for the list, a radix select over the next 10 + 10 bits
+  // (levels 1, 2) finds the exact threshold key T and c = #keys < T
   uint32_t prefix = 0, pmask = 0;
   int below = 0, need = 0;
+  bool list_path = false;
   const int shifts[3] = {20, 10, 0};
   const int widths[3] = {12, 10, 10};
   for (int lv = 0; lv < 3; ++lv) {
@@ -154,58 +222,73 @@ k_decode_select(const uint32_t* __restrict__ keys, uint32_t* __restrict__ hist0,
     pmask |= static_cast<uint32_t>(nb - 1) << shifts[lv];
     below = s_below;
     __syncthreads();
+    if (lv == 0 && hist[prefix >> 20] <= kBndCap) {
+      list_path = true;
+      break;
+    }
   }
   if (tid == 0) {
     hdr->n_boxes = need;
     hdr->err = *err;
-    s_nsel = 0;
   }
   if (need == 0) return;
-  const uint32_t T = prefix;
-  __syncthreads();
 
-  // ---- 2. collect keys < T, then the (need - below) lowest-index ties ------
-  int ties = 0;
-  for_chunk(keys, lo, chunk4, [&](uint32_t k, int i) {
-    if (k < T) {
-      const int pos = atomicAdd(&s_nsel, 1);
-      sel[pos] = (static_cast<unsigned long long>(k) << 32) | static_cast<unsigned>(i);
-    } else if (k == T) {
-      ++ties;
-    }
-  });
-  int tie_base = block_scan_excl(ties, &s_total);
-  const int take = need - below;
-  if (ties > 0 && tie_base < take) {
+  if (list_path) {
+    // ---- 2. one pass: lower bins -> selection, bin b0 -> list ----------------
+    const uint32_t b0 = prefix >> 20;
+    const int nb0 = hist[b0];
+    for_strided(keys, n4, [&](uint32_t k, int i) {
+      if (k == kInvalid) return;
+      const uint32_t bin = k >> 20;
+      const unsigned long long e = (static_cast<unsigned long long>(k) << 32) | static_cast<unsigned>(i);
+      if (bin < b0)
+        sel[atomicAdd(&s_nsel, 1)] = e;
+      else if (bin == b0)
+        bnd[atomicAdd(&s_nb, 1)] = e;
+    });
+    __syncthreads();
+    // ---- 3. sort both, complete the selection with bin b0's smallest --------
+    const int pa = pow2_at_least(below), pb = pow2_at_least(nb0);
+    for (int i = below + tid; i < pa; i += kThreads) sel[i] = ~0ull;
+    for (int i = nb0 + tid; i < pb; i += kThreads) bnd[i] = ~0ull;
+    __syncthreads();
+    bitonic2(sel, pa, bnd, pb);
+    for (int r = tid; r < need - below; r += kThreads) sel[below + r] = bnd[r];
+    __syncthreads();
+  } else {
+    const uint32_t T = prefix;
+    __syncthreads();
+
+    // ---- 2'. collect keys < T, then the (need - below) lowest-index ties ----
+    int ties = 0;
     for_chunk(keys, lo, chunk4, [&](uint32_t k, int i) {
-      if (k == T && tie_base < take) {
-        sel[below + tie_base] = (static_cast<unsigned long long>(T) << 32) | static_cast<unsigned>(i);
-        ++tie_base;
+      if (k < T) {
+        const int pos = atomicAdd(&s_nsel, 1);
+        sel[pos] = (static_cast<unsigned long long>(k) << 32) | static_cast<unsigned>(i);
+      } else if (k == T) {
+        ++ties;
       }
     });
-  }
-  __syncthreads();
-
-  // ---- 3. sort the K selected pairs and decode -----------------------------
-  int P2 = 1;
-  while (P2 < need) P2 <<= 1;
-  for (int i = need + tid; i < P2; i += kThreads) sel[i] = ~0ull;
-  __syncthreads();
-  for (int k = 2; k <= P2; k <<= 1) {
-    for (int j = k >> 1; j > 0; j >>= 1) {
-      for (int i = tid; i < P2; i += kThreads) {
-        const int l = i ^ j;
-        if (l > i) {
-          const unsigned long long x = sel[i], y = sel[l];
-          if ((x > y) == ((i & k) == 0)) {
-            sel[i] = y;
-            sel[l] = x;
-          }
+    int tie_base = block_scan_excl(ties, &s_total);
+    const int take = need - below;
+    if (ties > 0 && tie_base < take) {
+      for_chunk(keys, lo, chunk4, [&](uint32_t k, int i) {
+        if (k == T && tie_base < take) {
+          sel[below + tie_base] = (static_cast<unsigned long long>(T) << 32) | static_cast<unsigned>(i);
+          ++tie_base;
         }
-      }
-      __syncthreads();
+      });
     }
+    __syncthreads();
+
+    // sort the K selected pairs
+    const int P2 = pow2_at_least(need);
+    for (int i = need + tid; i < P2; i += kThreads) sel[i] = ~0ull;
+    __syncthreads();
+    bitonic2(sel, P2, sel, 1);
   }
+
+  // ---- 4. decode the K pairs (in order) into boxes --------------------------
   for (int r = tid; r < need; r += kThreads) {
     const int a = static_cast<int>(sel[r] & 0xFFFFFFFFull);
     const int cell = a / g.anchors, an = a - cell * g.anchors;
@@ -250,7 +333,11 @@ cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t st) {
   g.ha = 1.56f;
   g.za = -1.0f;
   g.da = (float)std::sqrt(3.9 * 3.9 + 1.6 * 1.6);
-  return launch_pdl(k_decode_select, dim3(1), dim3(kThreads), 0, st, a.keys, a.hist0, a.head,
+  const size_t dyn = kBndCap * sizeof(unsigned long long);
+  cudaError_t e = cudaFuncSetAttribute(k_decode_select, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)dyn);
+  if (e != cudaSuccess) return e;
+  return launch_pdl(k_decode_select, dim3(1), dim3(kThreads), dyn, st, a.keys, a.hist0, a.head,
                     decode_key_chunk4(n), a.max_boxes, g, a.err, hdr, boxes);
 }
 

@@ -249,16 +249,17 @@ k_fuse_head(const void* const* __restrict__ feats, const int* __restrict__ prese
       }
       const float out = acc[c][0] + __shfl_xor_sync(kFull, acc[c][0], 1) + hb;
       const int cell = cell0 + c;
-      if ((lane & 1) == 0 && cell < cells) {
-        const int o = lane >> 1;
-        head_out[(size_t)cell * kHeadOut + o] = out;
-        if (o < anchors) {
-          const bool keep = out >= cls_thresh;
-          const uint32_t key = keep ? ord_desc(out) : 0xFFFFFFFFu;
-          keys[(size_t)cell * anchors + o] = key;
-          if (keep) atomicAdd(&hist0[key >> 20], 1u);
-        }
-      }
+      const int o = lane >> 1;
+      const bool mine = (lane & 1) == 0 && cell < cells;
+      if (mine) head_out[(size_t)cell * kHeadOut + o] = out;
+      const bool keep = mine && o < anchors && out >= cls_thresh;
+      const uint32_t key = keep ? ord_desc(out) : 0xFFFFFFFFu;
+      if (mine && o < anchors) keys[(size_t)cell * anchors + o] = key;
+      // lanes sharing a histogram bin add their count with one atomic (valid
+      // logits crowd into a few dozen bins)
+      const uint32_t bin = keep ? (key >> 20) : 0xFFFFFFFFu;
+      const unsigned peers = __match_any_sync(kFull, bin);
+      if (keep && lane == __ffs(peers) - 1) atomicAdd(&hist0[bin], (uint32_t)__popc(peers));
     }
   }
 }

@@ -151,6 +151,33 @@ struct FuseArgs {
   int anchors;
 };
 cudaError_t launch_fuse_head(const FuseArgs& a, bool bf16, cudaStream_t st);
+
+// Max fusion + head on the tensor cores (fuse_tc.cu).
+constexpr int kFuseHeadOut = 16;
+struct FuseTcParams {
+  CUtensorMap feat[RTCC_MAX_AGENTS];  // agent k's slot [cells][C], box (bkc, 128), swizzled
+  CUtensorMap wmap;                   // head weights [16][C] in the storage type, box (bkc, 16)
+  const int* present;                 // device [K]
+  int K, C, cells, bkc;
+  const float* head_b;                // device [16]
+  float* head_out;                    // device [cells][16]
+  void* fused;                        // device [cells][C] or null
+  uint32_t* keys;                     // device [cells][anchors] decode keys
+  uint32_t* hist0;                    // device [4096] top-12-bit key histogram
+  float cls_thresh;
+  int anchors;
+  int* err;                           // device error word
+};
+// Channel chunk (64 or 32) the kernel stages for C channels and K agent slots,
+// 0 if it cannot run that shape.
+int fuse_tc_chunk(int C, int K);
+cudaError_t launch_fuse_max_head(const FuseTcParams& p, bool bf16, cudaStream_t st);
+
+// Row-major 2-D 16-bit tensor map [outer][inner] with a box of
+// box_inner x box_outer elements and the given swizzle span (128, 64 or 0
+// bytes); OOB elements read as zero.
+cudaError_t tmap_2d(CUtensorMap* m, const void* base, bool bf16, uint64_t inner, uint64_t outer,
+                    uint32_t box_inner, uint32_t box_outer, int swizzle_bytes);
 // Head weight permutation expected by the fusion kernel (host side).
 void permute_head_weights(const float* w /*[16][C]*/, int C, float* out /*[16*C]*/);
 

@@ -171,6 +171,27 @@ def test_empty_and_out_of_range_payloads(R):
     R.rtcc_destroy(ctx)
 
 
+@pytest.mark.parametrize("grid", [(96, 64), (256, 256)])
+def test_decode_all_equal_logits(R, grid):
+    # Zero head weights: every logit of anchor a equals its bias, so the keys
+    # of an anchor are one value repeated over all cells.  The selection is
+    # then decided by anchor index alone (ties), and at 256x256 the threshold
+    # bin holds 16384 keys, more than the decode's shared-memory list takes
+    # (its radix-select fallback); at 96x64 it holds 1536 (the list path).
+    cfg = dataclasses.replace(_small_pp(grid=grid), cls_thresh=-1.0)
+    w = dict(synth.weights_for(cfg))
+    w["head.w"] = np.zeros_like(w["head.w"])
+    ctx = R.rtcc_init(R.model_config(cfg, flags=U.DEBUG_FLAGS), synth.weight_blob(w))
+    try:
+        pts = [synth.points_for(cfg, 0, k) for k in range(cfg.n_agents)]
+        boxes = U.run_frame(ctx, cfg, pts, [0.0] * cfg.n_agents, R.MODE_RTCC)
+        hd = U.head_to_oracle_layout(R.rtcc_get_head(ctx, cfg.feat_h, cfg.feat_w))
+        assert len(boxes) == cfg.max_boxes
+        _check_decode(cfg, hd, boxes)
+    finally:
+        R.rtcc_destroy(ctx)
+
+
 @pytest.mark.parametrize("name", ["tiny", "small_pp", "small_attn"])
 def test_rtcc_and_barrier_bit_identical(R, name):
     if name == "tiny":
