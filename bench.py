@@ -4,12 +4,15 @@ workload (256x256 grid, 100k points + 20x500 clustered points per agent, max
 fusion, arrivals U[0, 30] ms), plus the encoder's tensor-core throughput and
 the fusion kernel's bandwidth.
 
-One step = four frames of the whole hot path, each replayed in real time from
+One step = five frames of the whole hot path, each replayed in real time from
 a seeded arrival trace: {RTCC, Barrier} x {inputs resident in HBM, inputs in
-pinned host memory copied on release}.  The order of RTCC and Barrier
-alternates between steps.  L2 is flushed (a 512 MiB device write) before every
-frame.  Latency = host time the detections are ready (after the D2H of the
-boxes) minus host time of the call that delivered the last payload.
+pinned host memory copied on release} on an uninstrumented context, plus one
+RTCC frame on a context whose graphs carry CUDA event nodes around the
+backbone and fusion kernels (their live durations; that frame's latency is not
+sampled).  The order of RTCC and Barrier alternates between steps.  L2 is
+flushed (a 512 MiB device write) before every frame.  Latency = host time the
+detections are ready (after the D2H of the boxes) minus host time of the call
+that delivered the last payload.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
@@ -267,27 +270,34 @@ def run_ours(args):
 
     cfg = synth.get_config(WORKLOAD)
     w = synth.weights_for(cfg)
-    ctx = R.rtcc_init(R.model_config(cfg, flags=R.FLAG_TIMELINE), synth.weight_blob(w))
+    # latency frames run on a context without instrumentation (the served
+    # configuration); one frame per step runs on a second context whose graphs
+    # carry CUDA event nodes around the backbone and fusion kernels, for their
+    # live durations (the event nodes lengthen that frame's tail, so it is
+    # not one of the latency samples)
+    ctx = R.rtcc_init(R.model_config(cfg, flags=0), synth.weight_blob(w))
+    tctx = R.rtcc_init(R.model_config(cfg, flags=R.FLAG_TIMELINE), synth.weight_blob(w))
     K = cfg.n_agents
     NF = 4
     frames = [[synth.points_for(cfg, f, k) for k in range(K)] for f in range(NF)]
-    staging = [R.rtcc_staging_buffer(ctx, k) for k in range(K)]
+    staging = {id(c): [R.rtcc_staging_buffer(c, k) for k in range(K)] for c in (ctx, tctx)}
     flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device="cuda")
     fid = [0]
 
-    def one_frame(step, mode, resident):
+    def one_frame(step, mode, resident, c=None):
+        c = ctx if c is None else c
         pts = frames[step % NF]
         a = synth.arrivals_for(cfg, step)
         flush.zero_()
         torch.cuda.synchronize()
         for k in range(K):
             if resident:
-                assert R.rtcc_stage_resident(ctx, k, pts[k]) == R.OK
+                assert R.rtcc_stage_resident(c, k, pts[k]) == R.OK
             else:
-                staging[k][:pts[k].shape[0]] = pts[k]
-        assert R.rtcc_set_mode(ctx, mode) == R.OK
+                staging[id(c)][k][:pts[k].shape[0]] = pts[k]
+        assert R.rtcc_set_mode(c, mode) == R.OK
         fid[0] += 1
-        assert R.rtcc_frame_begin(ctx, fid[0], 0.0) == R.OK
+        assert R.rtcc_frame_begin(c, fid[0], 0.0) == R.OK
         t0 = R.rtcc_now_ms() + 0.5
         for k in sorted(range(K), key=lambda k: (a[k], k)):
             due = t0 + a[k]
@@ -298,14 +308,14 @@ def run_ours(args):
                 if rem > 2.0:
                     time.sleep((rem - 1.5) / 1e3)
             if resident:
-                s = R.rtcc_payload_resident(ctx, k, float(a[k]))
+                s = R.rtcc_payload_resident(c, k, float(a[k]))
             else:
                 n = pts[k].shape[0]
-                s = R.rtcc_payload_complete(ctx, k, staging[k][:n], float(a[k]))
+                s = R.rtcc_payload_complete(c, k, staging[id(c)][k][:n], float(a[k]))
             assert s == R.OK, R.rtcc_status_str(s)
-        s, boxes, _ = R.rtcc_wait_detection(ctx, 10000)
+        s, boxes, _ = R.rtcc_wait_detection(c, 10000)
         assert s == R.OK, R.rtcc_status_str(s)
-        info = R.rtcc_get_frame_info(ctx)
+        info = R.rtcc_get_frame_info(c)
         return {"tail": info.t_ready_ms - info.t_last_event_ms,
                 "bb": [info.gpu_backbone_ms[k] for k in range(K)],
                 "fuse": info.gpu_fusion_ms, "post": info.gpu_post_ms,
@@ -317,6 +327,7 @@ def run_ours(args):
         for resident in (True, False):
             for mode in modes:
                 out.append((mode, resident, one_frame(step, mode, resident)))
+        out.append(("timeline", True, one_frame(step, R.MODE_RTCC, True, tctx)))
         return out
 
     for s in range(args.warmup):
@@ -347,8 +358,8 @@ def run_ours(args):
 
     r_res, b_res = tails(R.MODE_RTCC, True), tails(R.MODE_BARRIER, True)
     r_e2e, b_e2e = tails(R.MODE_RTCC, False), tails(R.MODE_BARRIER, False)
-    bb = [x for (m, res, r) in rec if m == R.MODE_RTCC and res for x in r["bb"] if x > 0]
-    fu = [r["fuse"] for (m, res, r) in rec if m == R.MODE_RTCC and res and r["fuse"] > 0]
+    bb = [x for (m, res, r) in rec if m == "timeline" for x in r["bb"] if x > 0]
+    fu = [r["fuse"] for (m, res, r) in rec if m == "timeline" and r["fuse"] > 0]
     value = pct(r_res, 50)
     if dist is not None:
         t = torch.tensor([value, wall_ms], device="cuda", dtype=torch.float64)
@@ -361,7 +372,7 @@ def run_ours(args):
     enc_tflops = flops / (bb_ms * 1e-3) / 1e12 if bb_ms else None
     fu_ms = float(np.mean(fu)) if fu else None
     fu_gbs = fusion_bytes(cfg, K) / (fu_ms * 1e-3) / 1e9 if fu_ms else None
-    n_launch = R.rtcc_kernels_per_frame(ctx, K) * 4 * args.steps
+    n_launch = R.rtcc_kernels_per_frame(ctx, K) * 5 * args.steps
     h2d = sum(int(p.shape[0]) * 16 + 16 for p in frames[0])
     d2h = 16 + cfg.max_boxes * 36
 
@@ -370,7 +381,7 @@ def run_ours(args):
         "warmup": args.warmup, "ms_per_step": wall_ms / max(args.steps, 1),
         "higher_is_better": False, "scaling": "weak", "vs_baseline": None, "dtype": "fp16",
         "data": DATA,
-        "config": {"workload": _workload_desc(cfg), "frames_per_step": 4,
+        "config": {"workload": _workload_desc(cfg), "frames_per_step": 5,
                    "l2": "flushed by a 512 MiB device write before every frame",
                    "inputs": "value: payloads resident in HBM before release; e2e: pinned host "
                              "staging, H2D on release inside the measured span",
@@ -385,8 +396,8 @@ def run_ours(args):
                     "gflop_per_branch": flops / 1e9},
         "fusion": {"gbs": fu_gbs, "frac_of_hbm": (fu_gbs / hbm) if fu_gbs else None,
                    "ms": fu_ms, "mb_per_launch": fusion_bytes(cfg, K) / 1e6},
-        "roofline": {"kernel": "k_conv_tc (tcgen05 implicit-GEMM conv/deconv backbone of one "
-                               "branch, 13 convs + 3 deconvs)",
+        "roofline": {"kernel": "k_backbone (persistent tcgen05 implicit-GEMM backbone of one "
+                               "branch: 13 convs + 3 deconvs in one launch)",
                      "bound": "tensor", "achieved": enc_tflops, "peak": tflops_peak,
                      "unit": "TFLOP/s", "frac": (enc_tflops / tflops_peak) if enc_tflops else None,
                      "peak_kind": f"{peak_kind} bf16 burst (fp16 has the same nominal rate)",
@@ -405,9 +416,10 @@ def run_ours(args):
                        f"in float64 NumPy; RTCC tail of each timed step's arrival trace on the "
                        f"single-stream timeline (Eqs. 20-22) with those service times")}
     R.rtcc_destroy(ctx)
+    R.rtcc_destroy(tctx)
 
-    # per-layer live times (a separate context whose graphs carry an event
-    # node between every conv launch; outside the timed region)
+    # per-layer live times (a separate context whose backbone kernel stamps
+    # the GPU global timer as it starts each layer; outside the timed region)
     if rank == 0:
         pctx = R.rtcc_init(R.model_config(cfg, flags=R.FLAG_LAYER_TIMES), synth.weight_blob(w))
         times = []
@@ -432,8 +444,9 @@ def run_ours(args):
             rows.append({"layer": name, "gflop": round(fl / 1e9, 4), "us": round(float(t_ms) * 1e3, 2),
                          "tflops": round(tf, 1), "frac": round(tf / tflops_peak, 4)})
         tot_us = float(np.sum(med)) * 1e3
-        line["layers"] = {"note": "each conv/deconv launch timed alone (event nodes between "
-                                  "launches remove the launch overlap of the served graph)",
+        line["layers"] = {"note": "span from the start of each layer to the start of the next "
+                                  "in the persistent backbone kernel (global-timer stamps); the "
+                                  "neck deconvs overlap the deepest block",
                           "sum_us": round(tot_us, 1),
                           "tflops_isolated": round(flops / (tot_us * 1e-6) / 1e12, 1),
                           "rows": rows}

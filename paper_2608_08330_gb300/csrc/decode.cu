@@ -8,18 +8,21 @@
 // anchor whose ascending order is descending logit order (0xFFFFFFFF below the
 // threshold), and a histogram of the keys' top 12 bits.  One block selects the
 // K = min(max_boxes, #valid) smallest (key, index) pairs:
-//   1. a scan of the histogram finds the bin b0 that holds the K-th key and
-//      the count c of keys in lower bins (c < K);
-//   2. one coalesced pass over the keys puts the c keys of lower bins into the
-//      selection and the keys of bin b0 into a shared-memory list;
-//   3. both are sorted (bitonic, in lockstep) and the K - c smallest pairs of
-//      bin b0 complete the selection, which is then already in order;
-//   4. the K pairs are decoded into boxes.
-// If bin b0 holds more keys than the list can take, a radix select refines
-// the threshold over the next 10 + 10 key bits instead (two more passes), the
-// keys below it are collected, and an ordered pass (each thread owns a
-// contiguous range of anchors, a block scan ranks its ties) adds the
-// lowest-index keys equal to it.
+//   1. a scan of the histogram finds the bin b0 that holds the K-th pair and
+//      the count of keys in lower bins;
+//   2. one coalesced pass over the keys selects the keys of lower bins and
+//      lists the keys of bin b0 in shared memory;
+//   3. a histogram of the listed keys' next 10 bits splits them into selected
+//      ones, the few of the bin b1 that holds the K-th pair, and the rest;
+//   4. the selected pairs are ordered (warp bitonic runs of 32, then a rank by
+//      binary search in the other runs; the pairs are distinct) and the
+//      lowest-ranked pairs of bin b1 complete the K;
+//   5. each ranked pair is decoded into the box of its rank.
+// When bin b0 or b1 is too full for the shared-memory lists (e.g. many equal
+// logits), a radix select over the global keys (next 10 + 10 bits) finds the
+// exact K-th key instead, the keys below it are collected, and an ordered pass
+// (each thread owns a contiguous range of anchors, a block scan ranks its
+// ties) adds the lowest-index keys equal to it.
 #include <cmath>
 
 #include "common.cuh"
@@ -34,6 +37,7 @@ constexpr uint32_t kInvalid = 0xFFFFFFFFu;
 constexpr int kThreads = 1024;
 constexpr int kMaxBins = 4096;
 constexpr int kBndCap = 4096;                // keys of bin b0 held in shared memory
+constexpr int kTieCap = 64;                  // keys of the level-1 bin ranked directly
 
 struct AnchorGeo {
   float x_min, y_min, sx, sy;       // cell size in metres
@@ -100,7 +104,7 @@ __device__ __forceinline__ void for_chunk(const uint32_t* __restrict__ keys, int
 template <typename F>
 __device__ __forceinline__ void for_strided(const uint32_t* __restrict__ keys, int n4, F f) {
   const uint4* v = reinterpret_cast<const uint4*>(keys);
-  constexpr int B = 4;                                   // loads in flight per thread
+  constexpr int B = 8;                                   // loads in flight per thread
   for (int base = threadIdx.x; base < n4; base += B * kThreads) {
     uint4 r[B];
 #pragma unroll
@@ -119,36 +123,105 @@ __device__ __forceinline__ void for_strided(const uint32_t* __restrict__ keys, i
   }
 }
 
-__device__ __forceinline__ void cmp_swap(unsigned long long* a, int i, int l, int k) {
-  const unsigned long long x = a[i], y = a[l];
-  if ((x > y) == ((i & k) == 0)) {
-    a[i] = y;
-    a[l] = x;
-  }
+// Append e to arr[] if pred, one shared-memory atomic per warp on the count
+// (the appends of a pass all hit one counter).  Every active lane must call it.
+__device__ __forceinline__ void warp_append(bool pred, unsigned long long e, int* count,
+                                            unsigned long long* arr) {
+  const unsigned act = __activemask();
+  const unsigned m = __ballot_sync(act, pred);
+  if (m == 0u) return;
+  const int lane = threadIdx.x & 31;
+  const int leader = __ffs(m) - 1;
+  int base = 0;
+  if (lane == leader) base = atomicAdd(count, __popc(m));
+  base = __shfl_sync(act, base, leader);
+  if (pred) arr[base + __popc(m & ((1u << lane) - 1u))] = e;
 }
 
-// Ascending bitonic sort of a[0..pa) and b[0..pb) (powers of two, padded with
-// ~0) in shared memory, the two in lockstep.
-__device__ void bitonic2(unsigned long long* a, int pa, unsigned long long* b, int pb) {
-  const int P = pa > pb ? pa : pb;
-  for (int k = 2; k <= P; k <<= 1) {
+// Ascending bitonic sort of one value per lane across a warp.
+__device__ __forceinline__ unsigned long long warp_sort32(unsigned long long v, int lane) {
+#pragma unroll
+  for (int k = 2; k <= 32; k <<= 1) {
+#pragma unroll
     for (int j = k >> 1; j > 0; j >>= 1) {
-      for (int i = threadIdx.x; i < P; i += kThreads) {
-        const int l = i ^ j;
-        if (l > i) {
-          if (k <= pa) cmp_swap(a, i, l, k);
-          if (k <= pb) cmp_swap(b, i, l, k);
-        }
-      }
-      __syncthreads();
+      const unsigned long long p = __shfl_xor_sync(0xFFFFFFFFu, v, j);
+      const bool up = (lane & k) == 0;                   // ascending sub-sequence
+      const bool lower = (lane & j) == 0;                // lower lane of the pair
+      v = (lower == up) ? (v < p ? v : p) : (v < p ? p : v);
     }
   }
+  return v;
 }
 
-__device__ __forceinline__ int pow2_at_least(int n) {
-  int p = 1;
+// Number of entries < v in a sorted run of 32.
+__device__ __forceinline__ int below_in_run(const unsigned long long* run, unsigned long long v) {
+  int pos = 0;
+#pragma unroll
+  for (int s = 16; s > 0; s >>= 1)
+    if (run[pos + s - 1] < v) pos += s;
+  return pos + (run[pos] < v ? 1 : 0);
+}
+
+// Sort of n <= 512 distinct (key, index) pairs in two block-wide phases,
+// run by the threads [t0, t0 + P) (P = n rounded up to a power of two >= 32):
+// phase 1 sorts runs of 32 in registers (warp bitonic) into run[0..P);
+// phase 2 ranks each pair by its position in its run plus binary searches in
+// the other runs and hands the pairs of rank < limit to emit(rank, pair).
+// The caller separates the phases with __syncthreads().
+__device__ __forceinline__ int sort_width(int n) {
+  int p = 32;
   while (p < n) p <<= 1;
   return p;
+}
+__device__ __forceinline__ void sort_phase1(const unsigned long long* in, int n, int t0, int P,
+                                            unsigned long long* run, const float* head, int anchors) {
+  const int t = threadIdx.x - t0;
+  if (t >= 0 && t < P) {
+    const unsigned long long v = t < n ? in[t] : ~0ull;
+    if (t < n) {
+      // the head row of this pair is read when its box is decoded: fetch it
+      // into L1 while the pairs are ranked
+      const int cell = static_cast<int>(v & 0xFFFFFFFFull) / anchors;
+      asm volatile("prefetch.global.L1 [%0];" ::"l"(head + (size_t)cell * 16));
+    }
+    run[t] = warp_sort32(v, threadIdx.x & 31);
+  }
+}
+template <typename F>
+__device__ __forceinline__ void sort_phase2(const unsigned long long* run, int t0, int P, int limit,
+                                            F emit) {
+  const int t = threadIdx.x - t0;
+  if (t < 0 || t >= P) return;
+  const unsigned long long v = run[t];
+  if (v == ~0ull) return;                                // padding
+  int r = t & 31;
+  for (int q = 0; q < P / 32; ++q)
+    if (q != (t >> 5)) r += below_in_run(run + 32 * q, v);
+  if (r < limit) emit(r, v);
+}
+
+// Box of the selected pair v (anchor = its low 32 bits), written to out.
+__device__ __forceinline__ void decode_box(unsigned long long v, const float* __restrict__ head,
+                                           const AnchorGeo& g, rtcc_box* out) {
+  const int a = static_cast<int>(v & 0xFFFFFFFFull);
+  const int cell = a / g.anchors, an = a - cell * g.anchors;
+  const int ix = cell % g.feat_w, iy = cell / g.feat_w;
+  const float* h = head + (size_t)cell * 16;
+  const float cls = h[an];
+  const float* rg = h + g.anchors + 7 * an;
+  const float xa = g.x_min + ((float)ix + 0.5f) * g.sx;
+  const float ya = g.y_min + ((float)iy + 0.5f) * g.sy;
+  rtcc_box b;
+  b.x = xa + rg[0] * g.da;
+  b.y = ya + rg[1] * g.da;
+  b.z = g.za + rg[2] * g.ha;
+  b.l = g.la * expf(fminf(rg[3], 10.0f));
+  b.w = g.wa * expf(fminf(rg[4], 10.0f));
+  b.h = g.ha * expf(fminf(rg[5], 10.0f));
+  b.yaw = (float)an * (3.14159265358979f / (float)g.anchors) + rg[6];
+  b.score = 1.0f / (1.0f + expf(-cls));
+  b.anchor = a;
+  *out = b;
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -157,114 +230,140 @@ k_decode_select(const uint32_t* __restrict__ keys, uint32_t* __restrict__ hist0,
                 const int* __restrict__ err, DetResultHeader* __restrict__ hdr,
                 rtcc_box* __restrict__ boxes) {
   extern __shared__ unsigned long long bnd[];        // [kBndCap] keys of bin b0
-  __shared__ int hist[kMaxBins];
-  __shared__ unsigned long long sel[kDecodeKeep];
-  __shared__ int s_total, s_bin, s_below, s_nsel, s_nb;
+  __shared__ int hist[kThreads];                     // level-1/2 histograms (10 bits)
+  __shared__ unsigned long long sel[kDecodeKeep];    // selected, unordered
+  __shared__ unsigned long long tie[kTieCap];
+  __shared__ int s_total, s_bin, s_below, s_nsel, s_nb, s_nl, s_nt;
   const int tid = threadIdx.x;
-  const int lo = tid * chunk4 * 4;
   const int n4 = chunk4 * kThreads;                   // 16-byte vectors of padded keys
   pdl_trigger();
   pdl_wait();
   if (tid == 0) {
     s_nsel = 0;
-    s_nb = 0;
+    s_nl = 0;
+    s_nt = 0;
   }
 
-  // ---- 1. threshold bin from the top-12-bit histogram (level 0); when that
-  // bin is too full for the list, a radix select over the next 10 + 10 bits
-  // (levels 1, 2) finds the exact threshold key T and c = #keys < T
-  uint32_t prefix = 0, pmask = 0;
-  int below = 0, need = 0;
-  bool list_path = false;
-  const int shifts[3] = {20, 10, 0};
-  const int widths[3] = {12, 10, 10};
-  for (int lv = 0; lv < 3; ++lv) {
-    const int nb = 1 << widths[lv];
-    if (lv == 0) {
-      for (int i = tid; i < nb; i += kThreads) {
-        hist[i] = (int)hist0[i];
-        hist0[i] = 0;                                  // ready for the next frame
+  // ---- 1. level 0: the bin b0 of the top-12-bit histogram that holds the
+  // K-th key, and the count below0 of keys in lower bins -------------------
+  static_assert(kMaxBins == 4 * kThreads, "one 16-byte vector of bins per thread");
+  int need;
+  {
+    // each thread: the contiguous bins 4*tid .. 4*tid+3
+    uint4* hv = reinterpret_cast<uint4*>(hist0) + tid;
+    const uint4 q = *hv;
+    *hv = make_uint4(0u, 0u, 0u, 0u);                  // ready for the next frame
+    const int h[4] = {(int)q.x, (int)q.y, (int)q.z, (int)q.w};
+    int run = block_scan_excl(h[0] + h[1] + h[2] + h[3], &s_total);
+    need = s_total < max_boxes ? s_total : max_boxes;  // K
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      if (run < need && run + h[j] >= need) {
+        s_bin = 4 * tid + j;
+        s_below = run;
+        s_nb = h[j];
       }
-    } else {
-      for (int i = tid; i < nb; i += kThreads) hist[i] = 0;
-      __syncthreads();
-      const int sh = shifts[lv];
-      for_chunk(keys, lo, chunk4, [&](uint32_t k, int) {
-        if (k != kInvalid && (k & pmask) == prefix) atomicAdd(&hist[(k >> sh) & (nb - 1)], 1);
-      });
+      run += h[j];
     }
     __syncthreads();
-    // each thread owns a contiguous range of bins
-    const int per = (nb + kThreads - 1) / kThreads;
-    int mine = 0;
-    for (int j = 0; j < per; ++j) {
-      const int b = tid * per + j;
-      if (b < nb) mine += hist[b];
-    }
-    int run = block_scan_excl(mine, &s_total);
-    const int total = s_total;
-    if (lv == 0) need = total < max_boxes ? total : max_boxes;   // K
-    if (need == 0) break;
-    // the bin where the cumulative count (offset by `below`) reaches need
-    for (int j = 0; j < per; ++j) {
-      const int b = tid * per + j;
-      if (b < nb) {
-        const int h = hist[b];
-        if (below + run < need && below + run + h >= need) {
-          s_bin = b;
-          s_below = below + run;
-        }
-        run += h;
-      }
-    }
-    __syncthreads();
-    prefix |= static_cast<uint32_t>(s_bin) << shifts[lv];
-    pmask |= static_cast<uint32_t>(nb - 1) << shifts[lv];
-    below = s_below;
-    __syncthreads();
-    if (lv == 0 && hist[prefix >> 20] <= kBndCap) {
-      list_path = true;
-      break;
-    }
   }
   if (tid == 0) {
     hdr->n_boxes = need;
     hdr->err = *err;
   }
   if (need == 0) return;
+  const uint32_t b0 = static_cast<uint32_t>(s_bin);
+  const int below0 = s_below;
+  const int nb0 = s_nb;
+  bool done = false;
 
-  if (list_path) {
-    // ---- 2. one pass: lower bins -> selection, bin b0 -> list ----------------
-    const uint32_t b0 = prefix >> 20;
-    const int nb0 = hist[b0];
+  if (nb0 <= kBndCap) {
+    // ---- 2. one coalesced pass: lower bins -> sel, bin b0 -> bnd ----------
     for_strided(keys, n4, [&](uint32_t k, int i) {
-      if (k == kInvalid) return;
-      const uint32_t bin = k >> 20;
+      const uint32_t bin = k >> 20;                    // invalid keys: bin 4095 > b0
       const unsigned long long e = (static_cast<unsigned long long>(k) << 32) | static_cast<unsigned>(i);
-      if (bin < b0)
-        sel[atomicAdd(&s_nsel, 1)] = e;
-      else if (bin == b0)
-        bnd[atomicAdd(&s_nb, 1)] = e;
+      const bool valid = k != kInvalid;
+      warp_append(valid && bin < b0, e, &s_nsel, sel);
+      warp_append(valid && bin == b0, e, &s_nl, bnd);
     });
+    __syncthreads();                                   // every thread has read nb0
+    // ---- 3. level 1 over bnd (key bits 10..19 = pair bits 42..51) ---------
+    for (int i = tid; i < 1024; i += kThreads) hist[i] = 0;
     __syncthreads();
-    // ---- 3. sort both, complete the selection with bin b0's smallest --------
-    const int pa = pow2_at_least(below), pb = pow2_at_least(nb0);
-    for (int i = below + tid; i < pa; i += kThreads) sel[i] = ~0ull;
-    for (int i = nb0 + tid; i < pb; i += kThreads) bnd[i] = ~0ull;
+    for (int i = tid; i < nb0; i += kThreads) atomicAdd(&hist[(int)((bnd[i] >> 42) & 1023)], 1);
     __syncthreads();
-    bitonic2(sel, pa, bnd, pb);
-    for (int r = tid; r < need - below; r += kThreads) sel[below + r] = bnd[r];
-    __syncthreads();
-  } else {
-    const uint32_t T = prefix;
-    __syncthreads();
+    {
+      int run = block_scan_excl(hist[tid], &s_total);  // 1024 bins, one per thread
+      const int h = hist[tid];
+      if (below0 + run < need && below0 + run + h >= need) {
+        s_bin = tid;
+        s_below = below0 + run;
+      }
+      __syncthreads();
+    }
+    const int b1 = s_bin, below1 = s_below, nb1 = hist[b1];
+    if (nb1 <= kTieCap) {
+      // bin-1 entries below b1 are selected; those in b1 compete for the rest
+      for (int i = tid; i < nb0; i += kThreads) {
+        const unsigned long long e = bnd[i];
+        const int bin1 = (int)((e >> 42) & 1023);
+        warp_append(bin1 < b1, e, &s_nsel, sel);
+        warp_append(bin1 == b1, e, &s_nt, tie);
+      }
+      __syncthreads();
+      // ---- 4. order sel (below1 pairs) and tie (nb1 pairs, all above);
+      // ---- 5. each ranked pair is decoded straight into its box slot
+      // (bnd is free again and serves as the run buffer)
+      const int P1 = sort_width(below1), P2 = sort_width(nb1);
+      sort_phase1(sel, below1, 0, P1, bnd, head, g.anchors);
+      sort_phase1(tie, nb1, kDecodeKeep, P2, bnd + kDecodeKeep, head, g.anchors);
+      __syncthreads();
+      sort_phase2(bnd, 0, P1, below1,
+                  [&](int r, unsigned long long v) { decode_box(v, head, g, boxes + r); });
+      sort_phase2(bnd + kDecodeKeep, kDecodeKeep, P2, need - below1,
+                  [&](int r, unsigned long long v) { decode_box(v, head, g, boxes + below1 + r); });
+      done = true;
+    }
+  }
 
-    // ---- 2'. collect keys < T, then the (need - below) lowest-index ties ----
+  if (!done) {
+    __syncthreads();                                   // every thread has read hist
+    // ---- 2'. radix select over the global keys: levels 1 and 2 (10 bits
+    // each) below the bin-0 prefix give the exact K-th key T and the count
+    // `below` of keys < T ---------------------------------------------------
+    uint32_t prefix = b0 << 20, pmask = 0xFFFu << 20;
+    int below = below0;
+    const int lo = tid * chunk4 * 4;
+    for (int lv = 1; lv <= 2; ++lv) {
+      const int sh = lv == 1 ? 10 : 0;
+      for (int i = tid; i < 1024; i += kThreads) hist[i] = 0;
+      __syncthreads();
+      for_chunk(keys, lo, chunk4, [&](uint32_t k, int) {
+        if (k != kInvalid && (k & pmask) == prefix) atomicAdd(&hist[(k >> sh) & 1023], 1);
+      });
+      __syncthreads();
+      int run = block_scan_excl(hist[tid], &s_total);
+      const int h = hist[tid];
+      if (below + run < need && below + run + h >= need) {
+        s_bin = tid;
+        s_below = below + run;
+      }
+      __syncthreads();
+      prefix |= static_cast<uint32_t>(s_bin) << sh;
+      pmask |= 1023u << sh;
+      below = s_below;
+      __syncthreads();
+    }
+    const uint32_t T = prefix;
+    if (tid == 0) s_nsel = 0;
+    __syncthreads();
+    // collect keys < T, then the (need - below) lowest-index keys equal to T:
+    // each thread owns a contiguous range of anchors and a block scan ranks
+    // its ties
     int ties = 0;
     for_chunk(keys, lo, chunk4, [&](uint32_t k, int i) {
       if (k < T) {
-        const int pos = atomicAdd(&s_nsel, 1);
-        sel[pos] = (static_cast<unsigned long long>(k) << 32) | static_cast<unsigned>(i);
+        sel[atomicAdd(&s_nsel, 1)] = (static_cast<unsigned long long>(k) << 32) | static_cast<unsigned>(i);
       } else if (k == T) {
         ++ties;
       }
@@ -280,37 +379,14 @@ k_decode_select(const uint32_t* __restrict__ keys, uint32_t* __restrict__ hist0,
       });
     }
     __syncthreads();
-
-    // sort the K selected pairs
-    const int P2 = pow2_at_least(need);
-    for (int i = need + tid; i < P2; i += kThreads) sel[i] = ~0ull;
+    const int P = sort_width(need);
+    sort_phase1(sel, need, 0, P, bnd, head, g.anchors);
     __syncthreads();
-    bitonic2(sel, P2, sel, 1);
-  }
-
-  // ---- 4. decode the K pairs (in order) into boxes --------------------------
-  for (int r = tid; r < need; r += kThreads) {
-    const int a = static_cast<int>(sel[r] & 0xFFFFFFFFull);
-    const int cell = a / g.anchors, an = a - cell * g.anchors;
-    const int ix = cell % g.feat_w, iy = cell / g.feat_w;
-    const float* h = head + (size_t)cell * 16;
-    const float cls = h[an];
-    const float* rg = h + g.anchors + 7 * an;
-    const float xa = g.x_min + ((float)ix + 0.5f) * g.sx;
-    const float ya = g.y_min + ((float)iy + 0.5f) * g.sy;
-    rtcc_box b;
-    b.x = xa + rg[0] * g.da;
-    b.y = ya + rg[1] * g.da;
-    b.z = g.za + rg[2] * g.ha;
-    b.l = g.la * expf(fminf(rg[3], 10.0f));
-    b.w = g.wa * expf(fminf(rg[4], 10.0f));
-    b.h = g.ha * expf(fminf(rg[5], 10.0f));
-    b.yaw = (float)an * (3.14159265358979f / (float)g.anchors) + rg[6];
-    b.score = 1.0f / (1.0f + expf(-cls));
-    b.anchor = a;
-    boxes[r] = b;
+    sort_phase2(bnd, 0, P, need,
+                [&](int r, unsigned long long v) { decode_box(v, head, g, boxes + r); });
   }
 }
+
 
 }  // namespace
 
