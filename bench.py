@@ -39,6 +39,10 @@ if ROOT not in sys.path:
 import synth  # noqa: E402
 
 METRIC = "complete-detection latency p50/p99 ms RTCC vs barrier; conv TFLOP/s, fusion GB/s"
+# dram__bytes_read.sum + dram__bytes_write.sum of one k_backbone launch (one pp3
+# branch) from an ncu --set full capture of this build; None once the kernel
+# changes and until it is captured again
+BACKBONE_TRAFFIC = 16_547_840
 WORKLOAD = "pp3"
 DATA = ("synthetic: seeded uniform + Gaussian-cluster point clouds, He-normal fp32 weights "
         "rounded to fp16, seeded arrival traces (OPV2V and the trained OpenCOOD model are not "
@@ -401,7 +405,7 @@ def run_ours(args):
                      "bound": "tensor", "achieved": enc_tflops, "peak": tflops_peak,
                      "unit": "TFLOP/s", "frac": (enc_tflops / tflops_peak) if enc_tflops else None,
                      "peak_kind": f"{peak_kind} bf16 burst (fp16 has the same nominal rate)",
-                     "traffic": None},
+                     "traffic": BACKBONE_TRAFFIC, "traffic_unit": "bytes per launch"},
         "e2e": {"value": pct(r_e2e, 50), "unit": "ms", "h2d_bytes_per_step": 2 * h2d,
                 "d2h_bytes_per_step": 2 * d2h},
         "clocks": clk,
