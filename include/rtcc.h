@@ -300,7 +300,7 @@ rtcc_status rtcc_get_tensor(struct rtcc_ctx* ctx, int32_t agent, int32_t which,
  * loops that must not risk the device synchronisation an allocation can
  * trigger.  This call allocates nothing: its scratch is one fixed array in
  * device memory that the library reserves on every GPU that loads it (about
- * 5.2 MB, kept until the process exits).  The array bounds the sizes:
+ * 3.1 MB, kept until the process exits).  The array bounds the sizes:
  * grid_w * grid_h <= 65536 cells, n_points <= 131072, max_pillars <= 16384,
  * pfn_ch in {32, 64}, max_pts <= 32; larger requests return RTCC_E_ARG.
  *

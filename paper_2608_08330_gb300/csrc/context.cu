@@ -326,7 +326,9 @@ rtcc_status build_branch(rtcc_ctx* c, int k) {
   RS(dalloc(c, &p.poff, (size_t)c->P * 4));
   RS(dalloc(c, &p.cursor, (size_t)c->P * 4));
   RS(dalloc(c, &p.list, (size_t)c->cap * 4));
-  RS(dalloc(c, &p.feat, (size_t)c->P * c->Cp * es));
+  RS(dalloc(c, &p.np_prev, 4));
+  CK(cudaMemset(p.np_prev, 0, 4));
+  p.clear_all = 0;                              // image and cell2pillar start cleared below
   RS(dalloc(c, &p.pillar_cell, (size_t)c->P * 4));
   RS(dalloc(c, &p.pcount, (size_t)c->P * 4));
   RS(dalloc(c, &p.stats, 8 * 4));
@@ -447,9 +449,9 @@ rtcc_status build_branch(rtcc_ctx* c, int k) {
   // split-K for layers whose tile grid would leave SMs idle: the largest
   // power-of-two split <= kMaxSplits that keeps the CTAs within one wave and
   // every slice at >= 4 K-blocks
-  int sms = 148, dev = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  // the CTAs of a launch in clusters (split-K slices share a cluster)
+  int sms = backbone_grid(kMaxSplits);
+  if (sms < 1) sms = backbone_grid(1);
   size_t ws_floats = 0, max_tiles = 0;
   for (ConvLayer& L : b.layers) {
     const int m_tiles = ((L.gw + conv_tile_w() - 1) / conv_tile_w()) *
@@ -1073,7 +1075,7 @@ double rtcc_now_ms(void) { return now_ms(); }
 
 int32_t rtcc_kernels_per_frame(rtcc_ctx* c, int32_t n_present) {
   if (!c) return 0;
-  return n_present * (6 + 1) + 2;     // pillar chain + backbone per branch; fusion, decode
+  return n_present * (5 + 1) + 2;     // pillar chain + backbone per branch; fusion, decode
 }
 
 }  // extern "C"

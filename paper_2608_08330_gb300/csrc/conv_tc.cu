@@ -107,6 +107,8 @@ struct LayerScalars {
   int kind, cin, cout, s, bn, bk, splits;
   int tiles_x, m_tiles, n_tiles, choff, wait_layers;
   int n_items, total_kb;
+  int ncb_log2;            // log2(cin / bk): k-block kb = (tap << ncb_log2) + channel block
+  int dsm;                 // split-K slices reduced through distributed shared memory
 };
 __device__ __forceinline__ LayerScalars layer_scalars(const LayerDesc& D) {
   LayerScalars S;
@@ -125,22 +127,26 @@ __device__ __forceinline__ LayerScalars layer_scalars(const LayerDesc& D) {
   S.n_tiles = D.n_tiles;
   S.choff = D.choff;
   S.wait_layers = D.wait_layers;
+  S.dsm = D.dsm;
   S.n_items = S.m_tiles * S.n_tiles * S.splits;
-  S.total_kb = (S.kind == DECONV ? 1 : 9) * (S.cin / S.bk);
+  S.ncb_log2 = __ffs(S.cin / S.bk) - 1;            // cin / bk is a power of two
+  S.total_kb = (S.kind == DECONV ? 1 : 9) << S.ncb_log2;
   return S;
 }
 
-// Work item t of a layer -> (m tile, n tile, K slice), its tile origin and
-// its k-block range [kb0, kb1).
+// Work item t of a layer -> (tile = (m tile, n tile), K slice z), its tile
+// origin and its k-block range [kb0, kb1).  The slice index runs fastest, so
+// the slices of a tile are consecutive items: with one item per CTA and a
+// grid of clusters of kMaxSplits CTAs they share a cluster, slice z on rank z.
 struct Item {
-  int x0, y0, n0, z, kb0, kb1;
+  int x0, y0, n0, z, tile, kb0, kb1;
 };
 __device__ __forceinline__ Item item_of(const LayerScalars& S, int t) {
   Item it;
-  const int mt = t % S.m_tiles;
-  const int r = t / S.m_tiles;
-  const int nt = r % S.n_tiles;
-  it.z = r / S.n_tiles;
+  it.z = t % S.splits;
+  it.tile = t / S.splits;
+  const int mt = it.tile % S.m_tiles;
+  const int nt = it.tile / S.m_tiles;
   it.x0 = (mt % S.tiles_x) * TW;
   it.y0 = (mt / S.tiles_x) * TH;
   it.n0 = nt * S.bn;
@@ -152,9 +158,8 @@ __device__ __forceinline__ Item item_of(const LayerScalars& S, int t) {
 // TMA load of the activation (A) box of k-block kb of item I.
 __device__ __forceinline__ void load_a(const LayerScalars& S, const CUtensorMap* map, uint8_t* dA,
                                        uint64_t* bar, const Item& I, int kb) {
-  const int ncb = S.cin / S.bk;
-  const int tap = kb / ncb;
-  const int cb = kb - tap * ncb;
+  const int tap = kb >> S.ncb_log2;
+  const int cb = kb - (tap << S.ncb_log2);
   if (S.kind == CONV3_S1) {
     const int dy = tap / 3, dx = tap - 3 * (tap / 3);
     tma_load_4d(dA, map, bar, cb * S.bk, I.x0 + dx - 1, I.y0 + dy - 1, 0);
@@ -174,10 +179,8 @@ __device__ __forceinline__ void load_a(const LayerScalars& S, const CUtensorMap*
 // TMA load of the weight (B) box of k-block kb of item I.
 __device__ __forceinline__ void load_b(const LayerScalars& S, const CUtensorMap* map, uint8_t* dB,
                                        uint64_t* bar, const Item& I, int kb) {
-  const int ncb = S.cin / S.bk;
-  const int tap = kb / ncb;
-  const int cb = kb - tap * ncb;
-  tma_load_2d(dB, map, bar, tap * S.cin + cb * S.bk, I.n0);
+  // K index of k-block kb = tap * cin + cb * bk = kb * bk
+  tma_load_2d(dB, map, bar, kb * S.bk, I.n0);
 }
 
 // One k-block of MMAs (BK = 64 or 32 -> 4 or 2 MMAs of K = 16) from
@@ -203,7 +206,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
   uint64_t* empty = full + kStages;
   uint64_t* accfull = empty + kStages;         // [2]
   uint64_t* accempty = accfull + 2;            // [2]
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accempty + 2);
+  uint64_t* recvbar = accempty + 2;            // partials received through DSMEM
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(recvbar + 1);
   __shared__ int s_last;
   __shared__ float s_bias[2][128];             // bias of the tile in each accumulator
 
@@ -220,7 +224,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
       mbar_init(&accfull[a], 1);
       mbar_init(&accempty[a], 4);              // one arrival per epilogue warp
     }
+    mbar_init(recvbar, 1);                     // the owner's arrival + the peers' bytes
     fence_barrier_init();
+    if (P.cluster > 1) fence_mbar_init_cluster();
   }
   if (warp == 1) {
     tmem_alloc(tmem_slot, kTmemCols);
@@ -228,6 +234,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
   }
   tc_fence_before();
   __syncthreads();
+  if (P.cluster > 1) cluster_sync_all();      // peers' barriers are initialised
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   pdl_trigger();
@@ -347,12 +354,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
     // loops early: after a wait runs out they skip further waits (the values
     // are then garbage, the error word says so) but keep the same sequence of
     // barriers and grid arrivals.
-    uint32_t tc = 0;
+    uint32_t tc = 0, dsm_phase = 0;
     bool alive = true;
     for (int l = 0; l < P.n_layers; ++l) {
       const LayerDesc& D = P.L[l];
       const LayerScalars S = layer_scalars(D);
       const CUtensorMap* mapC = &D.mapC;
+      const CUtensorMap* mapC16 = &D.mapC16;
       const int sg = S.bn < 64 ? S.bn : 64;    // channels per staged store box
       for (int t = blockIdx.x; t < S.n_items; t += G, ++tc) {
         const Item I = item_of(S, t);
@@ -377,12 +385,81 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
             tmem_ld16(taddr + c0, v);
             stage16<T>(stage, sg, row, c0, v, bias + c0);
           }
+        } else if (S.dsm) {
+          // The kMaxSplits K-slices of this tile sit on the CTAs of this
+          // cluster, slice z on rank z.  Reduce-scatter through distributed
+          // shared memory: rank z owns output channels [16z, 16z + 16); each
+          // rank sends every owner its partial of the owner's channels
+          // (16-byte st.async into the owner's receive slots, counted on the
+          // owner's mbarrier), and the owner sums the slices in slice order and
+          // stores its 16 channels.  bn = 64 = kMaxSplits * 16.
+          constexpr int CW = 16;
+          const int z = I.z;
+          if (row == 0 && cluster_ctarank() != (uint32_t)z) atomicOr(P.err, ERR_BOUNDS);
+          uint8_t* recv = stage;                                   // [kMaxSplits-1][BM][CW] fp32
+          uint8_t* out16 = stage + (kMaxSplits - 1) * BM * CW * 4; // [BM][CW] 16-bit
+          if (row == 0) mbar_arrive_expect_tx(recvbar, (kMaxSplits - 1) * BM * CW * 4);
+          const uint32_t my_recv = smem_u32(recv), my_bar = smem_u32(recvbar);
+          for (int q = 0; q < kMaxSplits; ++q) {
+            if (q == z) continue;                  // uniform over the CTA
+            float v[16];
+            tmem_ld16(taddr + q * CW, v);
+            const int slot = z < q ? z : z - 1;    // this rank's slot at owner q
+            const uint32_t dst = mapa_shared(my_recv + (uint32_t)((slot * BM + row) * CW * 4), q);
+            const uint32_t bar = mapa_shared(my_bar, q);
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+              st_async_v4(dst + 16 * j, make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]), bar);
+          }
+          float own[16];
+          tmem_ld16(taddr + z * CW, own);
+          if (alive && !mbar_wait(recvbar, dsm_phase)) {
+            if (lane == 0) atomicOr(P.err, ERR_WAIT_EPILOGUE);
+            alive = false;
+          }
+          dsm_phase ^= 1u;
+          float sum[16];
+#pragma unroll
+          for (int j = 0; j < 16; ++j) sum[j] = 0.f;
+          for (int zz = 0; zz < kMaxSplits; ++zz) {
+            if (zz == z) {
+#pragma unroll
+              for (int j = 0; j < 16; ++j) sum[j] += own[j];
+            } else {
+              const int slot = zz < z ? zz : zz - 1;
+              const float4* src = reinterpret_cast<const float4*>(recv + (slot * BM + row) * CW * 4);
+#pragma unroll
+              for (int q = 0; q < 4; ++q) {
+                const float4 f = src[q];
+                sum[4 * q] += f.x;
+                sum[4 * q + 1] += f.y;
+                sum[4 * q + 2] += f.z;
+                sum[4 * q + 3] += f.w;
+              }
+            }
+          }
+          // bias + ReLU, 16-bit, staged [BM][CW] (32-byte rows, no swizzle)
+          uint32_t pk[8];
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            pk[j] = Store<T>::pack2(relu_f(sum[2 * j] + bias[z * CW + 2 * j]),
+                                    relu_f(sum[2 * j + 1] + bias[z * CW + 2 * j + 1]));
+          uint4* o = reinterpret_cast<uint4*>(out16 + row * CW * 2);
+          o[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+          o[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+          fence_async_smem();
+          epilogue_sync();
+          if (row == 0) {
+            tma_store_3d(mapC16, out16, I.n0 + z * CW, I.x0, I.y0);
+            bulk_commit();
+          }
+          store = false;
         } else {
           // publish this slice's fp32 partial ([bn/4][BM][4] per (slice, tile),
           // so a warp's float4 stores cover 512 contiguous bytes), then the
           // last slice of the tile sums the slices in slice order
           const int tiles = S.m_tiles * S.n_tiles;
-          const int tile_id = t % tiles;
+          const int tile_id = I.tile;
           float4* mine =
               reinterpret_cast<float4*>(S.ws + (size_t)(I.z * tiles + tile_id) * BM * S.bn) + row;
           for (int c0 = 0; c0 < S.bn; c0 += 16) {
@@ -478,6 +555,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
 
   tc_fence_before();
   __syncthreads();
+  if (P.cluster > 1) cluster_sync_all();      // no peer still writes into this CTA
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
@@ -591,6 +669,13 @@ cudaError_t conv_make_maps(ConvLayer& L, bool bf16) {
     cuuint32_t es[3] = {1, 1, 1};
     r = enc(&L.mapC, dt, 3, L.out, dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, osw,
             CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+    // 16-channel boxes, unswizzled 32-byte rows: one owner's share of a
+    // split-K tile reduced through distributed shared memory
+    cuuint32_t box16[3] = {16, (cuuint32_t)TW, (cuuint32_t)TH};
+    r = enc(&L.mapC16, dt, 3, L.out, dims, strides, box16, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+            CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   }
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
@@ -603,10 +688,15 @@ cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, unsigned* grid_b
   P->grid_bar = grid_bar;
   P->err = err;
   P->stamps = stamps;
+  const int grid_sm = backbone_grid(1), grid_cl = backbone_grid(kMaxSplits);
+  if (grid_sm < 1) return cudaErrorInvalidValue;
+  bool any_dsm = false;
   for (size_t i = 0; i < layers.size(); ++i) {
     const ConvLayer& L = layers[i];
-    if (L.cin % L.bk || (L.kind != DECONV && L.cout % L.bn) ||
-        (L.kind == DECONV && L.bn != L.cout) || L.bn > 128 || L.bk > 64 || L.bn % 32)
+    const int ncb = L.bk > 0 ? L.cin / L.bk : 0;
+    if (L.bk < 1 || L.cin % L.bk || ncb < 1 || (ncb & (ncb - 1)) ||   // a power of two
+        (L.kind != DECONV && L.cout % L.bn) || (L.kind == DECONV && L.bn != L.cout) ||
+        L.bn > 128 || L.bk > 64 || L.bn % 32)
       return cudaErrorInvalidValue;
     const int total_kb = (L.kind == DECONV ? 1 : 9) * (L.cin / L.bk);
     if (L.splits < 1 || L.splits > kMaxSplits || L.splits > total_kb || (L.splits > 1 && (!L.ws || !L.counters)))
@@ -630,8 +720,54 @@ cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, unsigned* grid_b
     D.n_tiles = L.n_tiles_n;
     D.choff = L.choff;
     D.wait_layers = L.wait_layers;
+    D.mapC16 = L.mapC16;
+    // a split of kMaxSplits 64-wide tiles with one item per CTA reduces its
+    // slices through distributed shared memory within a cluster
+    D.dsm = (L.kind != DECONV && L.splits == kMaxSplits && L.bn == 16 * kMaxSplits && grid_cl > 0 &&
+             D.m_tiles * D.n_tiles * L.splits <= grid_cl)
+                ? 1
+                : 0;
+    any_dsm = any_dsm || D.dsm;
   }
+  P->cluster = any_dsm ? kMaxSplits : 1;
+  P->grid = any_dsm ? grid_cl : grid_sm;
   return cudaSuccess;
+}
+
+int backbone_grid(int cluster) {
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1)
+    return 0;
+  if (cluster <= 1) return sms;
+  static std::mutex mu;
+  static int cached[64][2] = {};                  // per device: cluster size, grid
+  std::lock_guard<std::mutex> lk(mu);
+  if (dev < 64 && cached[dev][0] == cluster) return cached[dev][1];
+  if (cudaFuncSetAttribute(k_backbone<__half>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           kSmem) != cudaSuccess)
+    return 0;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(sms - sms % cluster);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = kSmem;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (unsigned)cluster;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, k_backbone<__half>, &cfg) != cudaSuccess || n < 1) {
+    (void)cudaGetLastError();
+    return 0;
+  }
+  if (dev < 64) {
+    cached[dev][0] = cluster;
+    cached[dev][1] = n * cluster;
+  }
+  return n * cluster;
 }
 
 cudaError_t launch_backbone(const BackboneParams& P, bool bf16, cudaStream_t st) {
@@ -645,20 +781,21 @@ cudaError_t launch_backbone(const BackboneParams& P, bool bf16, cudaStream_t st)
                                       cudaFuncAttributeMaxDynamicSharedMemorySize, kSmem);
   });
   if (attr_err != cudaSuccess) return attr_err;
-  int dev = 0, sms = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  if (sms < 1) return cudaErrorInvalidValue;
+  if (P.grid < 1 || (P.cluster > 1 && P.grid % P.cluster)) return cudaErrorInvalidValue;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(sms);
+  cfg.gridDim = dim3(P.grid);
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = kSmem;
   cfg.stream = st;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeCooperative;   // every CTA resident: grid barriers are safe
   attr[0].val.cooperative = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = (unsigned)P.cluster;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = P.cluster > 1 ? 2 : 1;
   if (bf16) return cudaLaunchKernelEx(&cfg, k_backbone<__nv_bfloat16>, P);
   return cudaLaunchKernelEx(&cfg, k_backbone<__half>, P);
 }

@@ -53,22 +53,27 @@ struct PillarBufs {
   int* poff;             // [P]     offset of the pillar's point list
   int* cursor;           // [P]     fill cursor
   int* list;             // [cap]   point indices grouped by pillar
-  void* feat;            // [P][C]  pillar features (storage type)
+  int* np_prev;          // [1]     pillars the previous pass wrote into image and
+                         //         cell2pillar (0 at allocation)
   // outputs
   int* pillar_cell;      // [P]
   int* pcount;           // [P]     kept points
   int* stats;            // [8]     n, in_range, n_pillars, kept, 0, 0, ncap drops,
                          //         points of kept pillars before the N_max cap
-  int* cell2pillar;      // [H*W]
-  void* image;           // [H][W][C] storage type
+  int* cell2pillar;      // [H*W]     -1 where no kept pillar
+  void* image;           // [H][W][C] storage type, zeros where no kept pillar
   int cap, P, N, C;
+  int clear_all;         // 1: the pass clears all of image and cell2pillar (their
+                         // content is unknown); 0: they hold the previous pass's
+                         // output, and only its np_prev pillar cells are cleared
 };
 
 constexpr int kFirstInit = 0x7F7F7F7F;   // memset byte 0x7F
 constexpr int kScanTile = 1024;          // points per scan block
 inline int scan_blocks(int cap) { return (cap + kScanTile - 1) / kScanTile; }
 
-// Enqueue the 6 pillar kernels (cells, block sums, scan, fill, PFN, scatter).
+// Enqueue the 5 pillar kernels (cells, block sums, scan, fill, PFN; the PFN
+// writes each pillar's vector into the BEV pseudo-image).
 cudaError_t launch_pillarise(const PillarBufs& b, const GridGeom& g, const float* pfn_w,
                              const float* pfn_b, bool bf16, int* err, cudaStream_t st);
 
@@ -97,6 +102,7 @@ struct ConvLayer {
   const void* wpacked;   // device, K-major: conv [Cout][9][Cin]; deconv [s*s*Cout][Cin]
   const float* bias;     // device [Cout]
   CUtensorMap mapA, mapB, mapC;   // input, packed weights, output (store)
+  CUtensorMap mapC16;             // output with 16-channel boxes (convs)
 };
 
 // Encode the layer's tensor maps (input activations, packed weights, output).
@@ -110,12 +116,14 @@ constexpr int kMaxLayers = 20;
 constexpr int kMaxSplits = 4;     // split-K slices per tile (the reducing slice keeps one load per slice in flight)
 struct alignas(128) LayerDesc {   // CUtensorMap is 128-byte aligned
   CUtensorMap mapA, mapB, mapC;
+  CUtensorMap mapC16;            // output map with 16-channel boxes (split-K through DSMEM)
   const float* bias;
   float* ws;
   int* counters;
   int kind, cin, cout, s, bn, bk, splits;
   int tiles_x, m_tiles, n_tiles, choff;
   int wait_layers;
+  int dsm;                       // split-K slices reduced through distributed shared memory
 };
 struct BackboneParams {
   LayerDesc L[kMaxLayers];
@@ -123,6 +131,8 @@ struct BackboneParams {
   unsigned* grid_bar;            // [kMaxLayers] per-layer arrival counters, zero before each launch
   int* err;
   unsigned long long* stamps;    // optional [n_layers + 1] layer-start times (ns)
+  int cluster;                   // 1, or kMaxSplits when some layer reduces through DSMEM
+  int grid;                      // CTAs of the launch
 };
 
 // Fill the kernel parameters of a branch's backbone from its layer list;
@@ -131,6 +141,9 @@ cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, unsigned* grid_b
                           unsigned long long* stamps, BackboneParams* P);
 // One cooperative launch (one CTA per SM) running every layer.
 cudaError_t launch_backbone(const BackboneParams& P, bool bf16, cudaStream_t st);
+// CTAs of a backbone launch: every SM (cluster = 1), or as many CTAs as can be
+// co-resident in clusters of `cluster` CTAs; 0 on error.
+int backbone_grid(int cluster);
 
 // ---------------------------------------------------------------------------
 // post-join: fusion + head, decode

@@ -21,9 +21,12 @@
 //               points in one at a time (broadcast by shuffle): 9-d features,
 //               linear layer, ReLU, running max.  Every reduction has a fixed
 //               order, so the result is run-to-run deterministic.
-//   5. scatter: one pass over all cells writes the pillar vector or zeros
-//               (each cell has at most one pillar: no atomics) and restores the
-//               per-cell scratch for the next pass.
+//   5. image:   the PFN writes each kept pillar's vector into its cell of the
+//               pseudo-image and its id into cell2pillar (each cell has at most
+//               one pillar: no atomics).  Elsewhere the image holds zeros and
+//               cell2pillar -1: the first kernel of a pass clears the cells the
+//               previous pass wrote (np_prev of them), and the fill kernel, the
+//               last reader of the per-cell counters, restores them.
 #include <climits>
 
 #include "common.cuh"
@@ -35,13 +38,35 @@ namespace {
 
 constexpr unsigned kFull = 0xFFFFFFFFu;
 
+template <int CH>
 __global__ void k_pillar_cells(const float4* __restrict__ pts, const int* __restrict__ n_hdr,
                                GridGeom g, int* __restrict__ cell_of, int* __restrict__ cnt_cell,
-                               int* __restrict__ first_cell, int* __restrict__ stats) {
+                               int* __restrict__ first_cell, int* __restrict__ stats,
+                               const int* __restrict__ prev_cell, const int* __restrict__ np_prev,
+                               int clear_all, uint4* __restrict__ image,
+                               int* __restrict__ cell2pillar) {
   pdl_trigger();
   pdl_wait();
   const int n = *n_hdr;
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  // clear what the previous pass wrote (CH 16-byte chunks per cell)
+  {
+    const long long stride = (long long)gridDim.x * blockDim.x;
+    if (clear_all) {
+      const long long tot = (long long)g.W * g.H * CH;
+      for (long long q = i; q < tot; q += stride) {
+        image[q] = make_uint4(0u, 0u, 0u, 0u);
+        if (q % CH == 0) cell2pillar[q / CH] = -1;
+      }
+    } else {
+      const long long tot = (long long)(*np_prev) * CH;
+      for (long long q = i; q < tot; q += stride) {
+        const int cell = prev_cell[q / CH];
+        image[(size_t)cell * CH + q % CH] = make_uint4(0u, 0u, 0u, 0u);
+        if (q % CH == 0) cell2pillar[cell] = -1;
+      }
+    }
+  }
   if (i == 0) stats[0] = n;
   bool ok = false;
   if (i < n) {
@@ -209,7 +234,8 @@ k_pillar_scan(const int* __restrict__ n_hdr, const int* __restrict__ cell_of,
 
 __global__ void k_pillar_fill(const int* __restrict__ n_hdr, const int* __restrict__ cell_of,
                               const int* __restrict__ c2p, int P, const int* __restrict__ poff,
-                              int* __restrict__ cursor, int* __restrict__ list) {
+                              int* __restrict__ cursor, int* __restrict__ list,
+                              int* __restrict__ cnt_cell, int* __restrict__ first_cell) {
   pdl_trigger();
   pdl_wait();
   const int n = *n_hdr;
@@ -217,6 +243,10 @@ __global__ void k_pillar_fill(const int* __restrict__ n_hdr, const int* __restri
   if (i >= n) return;
   const int cell = cell_of[i];
   if (cell < 0) return;
+  // the scan was the last reader of the per-cell counters: restore them for
+  // the next pass (every point of the cell writes the same values)
+  cnt_cell[cell] = 0;
+  first_cell[cell] = kFirstInit;
   const int p = c2p[cell];
   if (p >= P) return;
   const int pos = poff[p] + atomicAdd(&cursor[p], 1);
@@ -260,7 +290,8 @@ k_pfn(const float4* __restrict__ pts, const int* __restrict__ stats_in,
       const int* __restrict__ pcnt_raw, const int* __restrict__ poff,
       const int* __restrict__ list, const int* __restrict__ pillar_cell,
       const float* __restrict__ w, const float* __restrict__ b, GridGeom g, int N,
-      T* __restrict__ feat, int* __restrict__ pcount, int* __restrict__ stats) {
+      T* __restrict__ image, int* __restrict__ cell2pillar, int* __restrict__ np_prev,
+      int* __restrict__ pcount, int* __restrict__ stats) {
   __shared__ float sw[C * 9];
   __shared__ float sb[C];
   __shared__ int s_stat[3];                   // kept, capped, raw (block partial sums)
@@ -273,6 +304,7 @@ k_pfn(const float4* __restrict__ pts, const int* __restrict__ stats_in,
   const int lane = threadIdx.x & 31;
   const int p = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int np = stats_in[2];
+  if (blockIdx.x == 0 && threadIdx.x == 0) *np_prev = np;   // cleared by the next pass
   if (p < np) {
     const int raw = pcnt_raw[p];
     const int base = poff[p];
@@ -321,10 +353,16 @@ k_pfn(const float4* __restrict__ pts, const int* __restrict__ stats_in,
         acc[i] = fmaxf(acc[i], relu_f(sacc));
       }
     }
-    T* dst = feat + (size_t)p * C + lane * PER;
+    // the pillar's vector goes straight into its cell of the pseudo-image
+    T* dst = image + (size_t)cell * C + lane * PER;
+    if (PER == 2) {
+      *reinterpret_cast<uint32_t*>(dst) = Store<T>::pack2(acc[0], acc[PER - 1]);
+    } else {
 #pragma unroll
-    for (int i = 0; i < PER; ++i) dst[i] = Store<T>::from_f(acc[i]);
+      for (int i = 0; i < PER; ++i) dst[i] = Store<T>::from_f(acc[i]);
+    }
     if (lane == 0) {
+      cell2pillar[cell] = p;
       pcount[p] = m;
       atomicAdd(&s_stat[0], m);
       atomicAdd(&s_stat[1], raw - m);
@@ -341,43 +379,16 @@ k_pfn(const float4* __restrict__ pts, const int* __restrict__ stats_in,
   }
 }
 
-// One thread per (cell, 16-byte chunk): write the pillar's vector or zeros,
-// publish cell2pillar, and restore the per-cell scratch.
-template <int C>
-__global__ void k_scatter(const int* __restrict__ stats_in, const int* __restrict__ c2p, int P,
-                          const uint4* __restrict__ feat, int cells, int* __restrict__ cnt_cell,
-                          int* __restrict__ first_cell, int* __restrict__ cell2pillar,
-                          uint4* __restrict__ image) {
-  constexpr int CH = C * 2 / 16;   // 16-byte chunks per cell (divides 32)
-  pdl_trigger();
-  pdl_wait();
-  const int t = blockIdx.x * blockDim.x + threadIdx.x;
-  const int cell = t / CH, ch = t % CH;
-  if (cell >= cells) return;     // all CH threads of a cell leave together
-  const int cnt = cnt_cell[cell];
-  int p = cnt > 0 ? c2p[cell] : -1;
-  if (p >= P) p = -1;
-  uint4 v = make_uint4(0, 0, 0, 0);
-  if (p >= 0) v = feat[(size_t)p * CH + ch];
-  image[(size_t)cell * CH + ch] = v;
-  const int lane = threadIdx.x & 31;
-  const unsigned grp = ((CH == 32) ? kFull : ((1u << CH) - 1u)) << (lane & ~(CH - 1));
-  __syncwarp(grp);
-  if (ch == 0) {
-    cell2pillar[cell] = p;
-    cnt_cell[cell] = 0;
-    first_cell[cell] = kFirstInit;
-  }
-}
-
 template <typename T, int C>
 cudaError_t launch_all(const PillarBufs& b, const GridGeom& g, const float* pfn_w,
                        const float* pfn_b, cudaStream_t st) {
-  const int cells = g.W * g.H;
   const int nblk = scan_blocks(b.cap);
   cudaError_t e;
-  e = launch_pdl(k_pillar_cells, dim3((b.cap + 255) / 256), dim3(256), 0, st, b.pts, b.n_hdr, g,
-                 b.cell_of, b.cnt_cell, b.first_cell, b.stats);
+  constexpr int CH = C * 2 / 16;                  // 16-byte chunks per cell
+  e = launch_pdl(k_pillar_cells<CH>, dim3((b.cap + 255) / 256), dim3(256), 0, st, b.pts, b.n_hdr,
+                 g, b.cell_of, b.cnt_cell, b.first_cell, b.stats,
+                 static_cast<const int*>(b.pillar_cell), static_cast<const int*>(b.np_prev),
+                 b.clear_all, static_cast<uint4*>(b.image), b.cell2pillar);
   if (e != cudaSuccess) return e;
   e = launch_pdl(k_pillar_blocksum, dim3(nblk), dim3(kScanThreads), 0, st, b.n_hdr, b.cell_of,
                  b.cnt_cell, b.first_cell, b.items, b.blocksum);
@@ -387,17 +398,11 @@ cudaError_t launch_all(const PillarBufs& b, const GridGeom& g, const float* pfn_
                  b.stats);
   if (e != cudaSuccess) return e;
   e = launch_pdl(k_pillar_fill, dim3((b.cap + 255) / 256), dim3(256), 0, st, b.n_hdr, b.cell_of,
-                 b.c2p, b.P, b.poff, b.cursor, b.list);
+                 b.c2p, b.P, b.poff, b.cursor, b.list, b.cnt_cell, b.first_cell);
   if (e != cudaSuccess) return e;
   e = launch_pdl(k_pfn<T, C>, dim3((b.P + 7) / 8), dim3(256), 0, st, b.pts, b.stats, b.pcnt_raw,
-                 b.poff, b.list, b.pillar_cell, pfn_w, pfn_b, g, b.N, static_cast<T*>(b.feat),
-                 b.pcount, b.stats);
-  if (e != cudaSuccess) return e;
-  constexpr int CH = C * 2 / 16;
-  const long long thr = (long long)cells * CH;
-  e = launch_pdl(k_scatter<C>, dim3((unsigned)((thr + 255) / 256)), dim3(256), 0, st, b.stats,
-                 b.c2p, b.P, static_cast<const uint4*>(b.feat), cells, b.cnt_cell, b.first_cell,
-                 b.cell2pillar, static_cast<uint4*>(b.image));
+                 b.poff, b.list, b.pillar_cell, pfn_w, pfn_b, g, b.N, static_cast<T*>(b.image),
+                 b.cell2pillar, b.np_prev, b.pcount, b.stats);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }

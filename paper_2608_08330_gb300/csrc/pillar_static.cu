@@ -8,7 +8,7 @@
 // this entry point takes its scratch from one fixed array in device global
 // memory that the library reserves when it is loaded, instead of calling any
 // allocator.  The array is sized for grids up to 65,536 cells, payloads up to
-// 131,072 points, 16,384 pillars and 64 PFN channels (about 5.2 MB, held on
+// 131,072 points, 16,384 pillars and 64 PFN channels (about 3.1 MB, held on
 // every GPU that loads the library until the process exits).
 //
 // The kernels are the ones rtcc_payload_complete runs (launch_pillarise); only
@@ -45,8 +45,8 @@ constexpr size_t kOffItems = align256(kOffBlock + 8ull * kMaxScanBlocks);
 constexpr size_t kOffRaw = align256(kOffItems + 8ull * kMaxScanBlocks * kScanTile);
 constexpr size_t kOffPoff = align256(kOffRaw + 4ull * kMaxPillars);
 constexpr size_t kOffCursor = align256(kOffPoff + 4ull * kMaxPillars);
-constexpr size_t kOffFeat = align256(kOffCursor + 4ull * kMaxPillars);
-constexpr size_t kStaticBytes = align256(kOffFeat + 2ull * kMaxPillars * kMaxCh);
+constexpr size_t kOffNp = align256(kOffCursor + 4ull * kMaxPillars);
+constexpr size_t kStaticBytes = align256(kOffNp + 16);
 
 static __device__ __align__(256) unsigned char g_pillar_scratch[kStaticBytes];
 
@@ -120,7 +120,7 @@ extern "C" rtcc_status rtcc_pillarise_noalloc(const rtcc_model_config* cfg, cons
   b.poff = reinterpret_cast<int*>(base + kOffPoff);
   b.cursor = reinterpret_cast<int*>(base + kOffCursor);
   b.list = reinterpret_cast<int*>(base + kOffList);
-  b.feat = base + kOffFeat;
+  b.np_prev = reinterpret_cast<int*>(base + kOffNp);
   b.pillar_cell = d_pillar_cell;
   b.pcount = d_count;
   b.stats = d_stats;
@@ -130,6 +130,7 @@ extern "C" rtcc_status rtcc_pillarise_noalloc(const rtcc_model_config* cfg, cons
   b.P = cfg->max_pillars;
   b.N = cfg->max_pts;
   b.C = cfg->pfn_ch;
+  b.clear_all = 1;                              // the caller's image and cell2pillar: unknown content
 
   int blocks = (int)((cells + 255) / 256);
   if (blocks < 1) blocks = 1;
