@@ -300,9 +300,42 @@ rtcc_status upload_weights(rtcc_ctx* c, const float* w) {
   return RTCC_OK;
 }
 
+// N tile and split-K factor of a conv layer, from a cost model of the
+// persistent backbone kernel: one tcgen05 MMA instruction costs about the same
+// for every N <= 128, so a k-block costs the same for every N tile; a CTA
+// holds one item at a time, so items beyond the grid take another round; a
+// split into kMaxSplits slices of a 64-wide tile (one item per CTA) is reduced
+// through distributed shared memory at about the cost of 6 k-blocks (the
+// measured cost of 128-wide splits, with twice the exchange, was far higher).
+// Ties go to the narrower tile (more CTAs).
+void pick_tile(int m_tiles, int co, int total_kb, int grid, int* bn_out, int* sp_out) {
+  double best = 1e30;
+  int bb = std::min(co, 64), bs = 1;
+  for (int bn : {32, 64, 128}) {
+    if (bn > co || co % bn) continue;
+    for (int sp : {1, kMaxSplits}) {
+      const int items = m_tiles * (co / bn) * sp;
+      if (sp > 1 && (bn != 64 || total_kb / sp < 4 || items > grid)) continue;
+      const int rounds = (items + grid - 1) / grid;
+      const double cost = rounds * (double)((total_kb + sp - 1) / sp) + (sp > 1 ? 6.0 : 0.0);
+      if (cost < best - 1e-9) {
+        best = cost;
+        bb = bn;
+        bs = sp;
+      }
+    }
+  }
+  *bn_out = bb;
+  *sp_out = bs;
+}
+
 rtcc_status build_branch(rtcc_ctx* c, int k) {
   Branch& b = c->br[k];
   const rtcc_model_config& g = c->cfg;
+  // CTAs of a backbone launch in clusters (split-K slices share a cluster)
+  int grid = backbone_grid(kMaxSplits);
+  if (grid < 1) grid = backbone_grid(1);
+  if (grid < 1) return RTCC_E_CUDA;
   const size_t es = 2;   // 16-bit storage
   const int cells = c->W * c->H;
   RS(halloc(c, &b.staging, kHdrBytes + (size_t)c->cap * 16));
@@ -370,23 +403,10 @@ rtcc_status build_branch(rtcc_ctx* c, int k) {
       L.gh = oh;
       L.ldc = co;
       L.choff = 0;
-      // N tile: the widest of 128/64/32 that gives about one tile per SM in
-      // a single wave
-      // (narrower tiles cost no more per MMA instruction than 64-wide ones,
-      // and they avoid split-K, whose cross-CTA reduction costs several
-      // dependent global round trips); 64 where even 32-wide tiles leave most
-      // SMs idle (the deepest block), which then splits K instead
-      int sms_avail = 148, dev_id = 0;
-      cudaGetDevice(&dev_id);
-      cudaDeviceGetAttribute(&sms_avail, cudaDevAttrMultiProcessorCount, dev_id);
       const int m_tiles = ((ow + conv_tile_w() - 1) / conv_tile_w()) *
                           ((oh + conv_tile_h() - 1) / conv_tile_h());
-      L.bn = std::min(co, 128);
-      while (L.bn > 32 && m_tiles * (co / L.bn) < sms_avail * 3 / 4 &&
-             m_tiles * (co / L.bn) * 2 <= sms_avail)
-        L.bn /= 2;
-      if (m_tiles * (co / L.bn) < sms_avail / 2) L.bn = std::min(co, 64);
       L.bk = (cin >= 64) ? 64 : 32;
+      pick_tile(m_tiles, co, 9 * (cin / L.bk), grid, &L.bn, &L.splits);
       L.n_tiles_n = co / L.bn;
       L.in = in;
       const bool last = (bi == g.n_blocks - 1) && (li == g.block_layers[bi] - 1);
@@ -446,24 +466,16 @@ rtcc_status build_branch(rtcc_ctx* c, int k) {
       b.layers.push_back(L);
     }
   }
-  // split-K for layers whose tile grid would leave SMs idle: the largest
-  // power-of-two split <= kMaxSplits that keeps the CTAs within one wave and
-  // every slice at >= 4 K-blocks
-  // the CTAs of a launch in clusters (split-K slices share a cluster)
-  int sms = backbone_grid(kMaxSplits);
-  if (sms < 1) sms = backbone_grid(1);
+  // fp32 workspace of the global-memory split-K reduction (used when a split
+  // layer cannot reduce through DSMEM); deconvs do not wait on their
+  // predecessor, so they may not share it: they never split
   size_t ws_floats = 0, max_tiles = 0;
   for (ConvLayer& L : b.layers) {
     const int m_tiles = ((L.gw + conv_tile_w() - 1) / conv_tile_w()) *
                         ((L.gh + conv_tile_h() - 1) / conv_tile_h());
     const int base = m_tiles * L.n_tiles_n;
-    const int total_kb = (L.kind == DECONV ? 1 : 9) * (L.cin / L.bk);
-    int sp = 1;
-    // deconvs do not wait on their predecessor, so they may not share its
-    // split-K workspace: no split for them
-    while (L.kind != DECONV && sp * 2 <= kMaxSplits && base * sp * 2 <= sms && total_kb / (sp * 2) >= 4)
-      sp *= 2;
-    L.splits = sp;
+    if (L.kind == DECONV || L.splits < 1) L.splits = 1;
+    const int sp = L.splits;
     if (sp > 1) {
       ws_floats = std::max(ws_floats, (size_t)sp * base * conv_tile_m() * L.bn);
       max_tiles = std::max(max_tiles, (size_t)base);

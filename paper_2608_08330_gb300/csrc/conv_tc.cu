@@ -55,7 +55,8 @@ constexpr int kStages = 6;
 constexpr int kABytes = BM * 64 * 2;         // A slot (BK <= 64)
 constexpr int kBBytes = 128 * 64 * 2;        // B slot (BN <= 128, BK <= 64)
 constexpr int kStageBytes = kABytes + kBBytes;
-constexpr int kStagingBytes = BM * 128 * 2;  // output tile (BN <= 128)
+constexpr int kStagingBytes = 32 * 1024;     // output tile (BN <= 128) or the DSMEM receive
+                                             // slots (3 x 128 x 16 fp32) + their output
 constexpr int kSmem = kStages * kStageBytes + kStagingBytes + 1024 + 256;
 constexpr uint32_t kTmemCols = 256;          // two 128-column accumulators
 
@@ -388,69 +389,76 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
         } else if (S.dsm) {
           // The kMaxSplits K-slices of this tile sit on the CTAs of this
           // cluster, slice z on rank z.  Reduce-scatter through distributed
-          // shared memory: rank z owns output channels [16z, 16z + 16); each
-          // rank sends every owner its partial of the owner's channels
-          // (16-byte st.async into the owner's receive slots, counted on the
-          // owner's mbarrier), and the owner sums the slices in slice order and
-          // stores its 16 channels.  bn = 64 = kMaxSplits * 16.
-          constexpr int CW = 16;
+          // shared memory: rank z owns CW = bn / kMaxSplits output channels
+          // [CW z, CW (z + 1)); each rank sends every owner its partial of the
+          // owner's channels (16-byte st.async into the owner's receive slots,
+          // counted on the owner's mbarrier), and the owner sums the slices in
+          // slice order and stores its channels in 16-channel TMA boxes.
+          const int CW = S.bn / kMaxSplits;                        // 16
           const int z = I.z;
           if (row == 0 && cluster_ctarank() != (uint32_t)z) atomicOr(P.err, ERR_BOUNDS);
           uint8_t* recv = stage;                                   // [kMaxSplits-1][BM][CW] fp32
-          uint8_t* out16 = stage + (kMaxSplits - 1) * BM * CW * 4; // [BM][CW] 16-bit
-          if (row == 0) mbar_arrive_expect_tx(recvbar, (kMaxSplits - 1) * BM * CW * 4);
+          uint8_t* out16 = stage + (kMaxSplits - 1) * BM * CW * 4; // [BM][16] 16-bit
+          if (row == 0) mbar_arrive_expect_tx(recvbar, (uint32_t)((kMaxSplits - 1) * BM * CW * 4));
           const uint32_t my_recv = smem_u32(recv), my_bar = smem_u32(recvbar);
           for (int q = 0; q < kMaxSplits; ++q) {
             if (q == z) continue;                  // uniform over the CTA
-            float v[16];
-            tmem_ld16(taddr + q * CW, v);
             const int slot = z < q ? z : z - 1;    // this rank's slot at owner q
             const uint32_t dst = mapa_shared(my_recv + (uint32_t)((slot * BM + row) * CW * 4), q);
             const uint32_t bar = mapa_shared(my_bar, q);
+            for (int c0 = 0; c0 < CW; c0 += 16) {
+              float v[16];
+              tmem_ld16(taddr + q * CW + c0, v);
 #pragma unroll
-            for (int j = 0; j < 4; ++j)
-              st_async_v4(dst + 16 * j, make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]), bar);
+              for (int j = 0; j < 4; ++j)
+                st_async_v4(dst + (uint32_t)(c0 + 4 * j) * 4,
+                            make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]), bar);
+            }
           }
-          float own[16];
-          tmem_ld16(taddr + z * CW, own);
           if (alive && !mbar_wait(recvbar, dsm_phase)) {
             if (lane == 0) atomicOr(P.err, ERR_WAIT_EPILOGUE);
             alive = false;
           }
           dsm_phase ^= 1u;
-          float sum[16];
+          for (int c0 = 0; c0 < CW; c0 += 16) {
+            float own[16];
+            tmem_ld16(taddr + z * CW + c0, own);
+            float sum[16];
 #pragma unroll
-          for (int j = 0; j < 16; ++j) sum[j] = 0.f;
-          for (int zz = 0; zz < kMaxSplits; ++zz) {
-            if (zz == z) {
+            for (int j = 0; j < 16; ++j) sum[j] = 0.f;
+            for (int zz = 0; zz < kMaxSplits; ++zz) {
+              if (zz == z) {
 #pragma unroll
-              for (int j = 0; j < 16; ++j) sum[j] += own[j];
-            } else {
-              const int slot = zz < z ? zz : zz - 1;
-              const float4* src = reinterpret_cast<const float4*>(recv + (slot * BM + row) * CW * 4);
+                for (int j = 0; j < 16; ++j) sum[j] += own[j];
+              } else {
+                const int slot = zz < z ? zz : zz - 1;
+                const float4* src =
+                    reinterpret_cast<const float4*>(recv + ((slot * BM + row) * CW + c0) * 4);
 #pragma unroll
-              for (int q = 0; q < 4; ++q) {
-                const float4 f = src[q];
-                sum[4 * q] += f.x;
-                sum[4 * q + 1] += f.y;
-                sum[4 * q + 2] += f.z;
-                sum[4 * q + 3] += f.w;
+                for (int q = 0; q < 4; ++q) {
+                  const float4 f = src[q];
+                  sum[4 * q] += f.x;
+                  sum[4 * q + 1] += f.y;
+                  sum[4 * q + 2] += f.z;
+                  sum[4 * q + 3] += f.w;
+                }
               }
             }
-          }
-          // bias + ReLU, 16-bit, staged [BM][CW] (32-byte rows, no swizzle)
-          uint32_t pk[8];
+            // bias + ReLU, 16-bit, staged [BM][16] per group (32-byte rows)
+            const float* bz = bias + z * CW + c0;
+            uint32_t pk[8];
 #pragma unroll
-          for (int j = 0; j < 8; ++j)
-            pk[j] = Store<T>::pack2(relu_f(sum[2 * j] + bias[z * CW + 2 * j]),
-                                    relu_f(sum[2 * j + 1] + bias[z * CW + 2 * j + 1]));
-          uint4* o = reinterpret_cast<uint4*>(out16 + row * CW * 2);
-          o[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-          o[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+            for (int j = 0; j < 8; ++j)
+              pk[j] = Store<T>::pack2(relu_f(sum[2 * j] + bz[2 * j]), relu_f(sum[2 * j + 1] + bz[2 * j + 1]));
+            uint4* o = reinterpret_cast<uint4*>(out16 + (c0 / 16) * BM * 32 + row * 32);
+            o[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            o[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+          }
           fence_async_smem();
           epilogue_sync();
           if (row == 0) {
-            tma_store_3d(mapC16, out16, I.n0 + z * CW, I.x0, I.y0);
+            for (int c0 = 0; c0 < CW; c0 += 16)
+              tma_store_3d(mapC16, out16 + (c0 / 16) * BM * 32, I.n0 + z * CW + c0, I.x0, I.y0);
             bulk_commit();
           }
           store = false;
