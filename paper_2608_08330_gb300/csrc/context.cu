@@ -10,6 +10,7 @@
 // dispatches all present branches in index order (Sec. V).  Both modes launch
 // the same graphs on the same inputs, so outputs are bit-identical.
 #include <algorithm>
+#include <atomic>
 #include <chrono>
 #include <cmath>
 #include <cstring>
@@ -82,16 +83,16 @@ struct rtcc_ctx {
   Branch br[RTCC_MAX_AGENTS];
   cudaStream_t xfer = nullptr, post = nullptr;
   cudaGraphExec_t post_exec = nullptr;
-  int* d_present = nullptr;
-  int* h_present = nullptr;           // pinned
+  int* d_present = nullptr;           // [K] set by a branch's first kernel, cleared by the decode
   void** d_feat_ptrs = nullptr;
   float* head_out = nullptr;
   void* fused = nullptr;
   uint32_t* keys = nullptr;           // decode key per anchor (padded)
   uint32_t* hist0 = nullptr;          // decode level-0 histogram
-  uint8_t* det_dev = nullptr;
-  uint8_t* det_host = nullptr;        // pinned
+  uint8_t* det_host = nullptr;        // pinned; the decode kernel writes it directly
   size_t det_bytes = 0;
+  volatile int* h_done = nullptr;     // pinned; the decode kernel sets it to 1 when det_host is complete
+  bool present_dirty = false;         // a branch set its presence flag and no post-join cleared it
   int* d_err = nullptr;
   cudaEvent_t det_ready = nullptr;
   cudaEvent_t ev_post0 = nullptr, ev_fuse0 = nullptr, ev_fuse1 = nullptr, ev_post1 = nullptr;
@@ -362,6 +363,7 @@ rtcc_status build_branch(rtcc_ctx* c, int k) {
   RS(dalloc(c, &p.np_prev, 4));
   CK(cudaMemset(p.np_prev, 0, 4));
   p.clear_all = 0;                              // image and cell2pillar start cleared below
+  p.present_flag = c->d_present + k;
   RS(dalloc(c, &p.pillar_cell, (size_t)c->P * 4));
   RS(dalloc(c, &p.pcount, (size_t)c->P * 4));
   RS(dalloc(c, &p.stats, 8 * 4));
@@ -597,7 +599,10 @@ rtcc_status capture_post(rtcc_ctx* c) {
   da.y_max = c->cfg.y_max;
   da.max_boxes = c->cfg.max_boxes;
   da.err = c->d_err;
-  da.out = c->det_dev;
+  da.out = c->det_host;                           // pinned host memory, addressable on the device
+  da.present = c->d_present;
+  da.K = c->K;
+  da.done = c->h_done;
   (void)cudaGetLastError();
   CK(cudaStreamBeginCapture(c->post, cudaStreamCaptureModeRelaxed));
   cudaError_t e = cudaSuccess;
@@ -611,8 +616,6 @@ rtcc_status capture_post(rtcc_ctx* c) {
   }
   if (e == cudaSuccess && tl) e = record_node(c->ev_fuse1, c->post);
   if (e == cudaSuccess) e = launch_decode(da, c->post);
-  if (e == cudaSuccess)
-    e = cudaMemcpyAsync(c->det_host, c->det_dev, c->det_bytes, cudaMemcpyDeviceToHost, c->post);
   if (e == cudaSuccess && tl) e = record_node(c->ev_post1, c->post);
   cudaGraph_t graph = nullptr;
   cudaError_t e2 = cudaStreamEndCapture(c->post, &graph);
@@ -654,12 +657,10 @@ rtcc_status init_impl(rtcc_ctx* c, const float* weights) {
   RS(upload_weights(c, weights));
   RS(dalloc(c, &c->d_err, 16));
   CK(cudaMemset(c->d_err, 0, 16));
+  RS(dalloc(c, &c->d_present, RTCC_MAX_AGENTS * 4));
+  CK(cudaMemset(c->d_present, 0, RTCC_MAX_AGENTS * 4));
   for (int k = 0; k < c->K; ++k) RS(build_branch(c, k));
   const int cells_f = c->Wf * c->Hf;
-  RS(dalloc(c, &c->d_present, RTCC_MAX_AGENTS * 4));
-  RS(halloc(c, &c->h_present, RTCC_MAX_AGENTS * 4));
-  for (int k = 0; k < RTCC_MAX_AGENTS; ++k) c->h_present[k] = k < c->K ? 1 : 0;
-  CK(cudaMemcpy(c->d_present, c->h_present, RTCC_MAX_AGENTS * 4, cudaMemcpyHostToDevice));
   RS(dalloc(c, &c->d_feat_ptrs, RTCC_MAX_AGENTS * sizeof(void*)));
   void* fp[RTCC_MAX_AGENTS] = {};
   for (int k = 0; k < c->K; ++k) fp[k] = c->br[k].feat;
@@ -672,9 +673,14 @@ rtcc_status init_impl(rtcc_ctx* c, const float* weights) {
   RS(dalloc(c, &c->hist0, kDecodeHistBins * sizeof(uint32_t)));
   CK(cudaMemset(c->hist0, 0, kDecodeHistBins * sizeof(uint32_t)));
   c->det_bytes = sizeof(DetResultHeader) + (size_t)g.max_boxes * sizeof(rtcc_box);
-  RS(dalloc(c, &c->det_dev, c->det_bytes));
-  CK(cudaMemset(c->det_dev, 0, c->det_bytes));
   RS(halloc(c, &c->det_host, c->det_bytes));
+  std::memset(c->det_host, 0, c->det_bytes);
+  {
+    int* d = nullptr;
+    RS(halloc(c, &d, sizeof(int)));
+    *d = 0;
+    c->h_done = d;
+  }
   CK(cudaStreamCreateWithFlags(&c->xfer, cudaStreamNonBlocking));
   CK(cudaStreamCreateWithFlags(&c->post, cudaStreamNonBlocking));
   CK(cudaEventCreateWithFlags(&c->det_ready, cudaEventDisableTiming));
@@ -713,19 +719,19 @@ rtcc_status launch_branch(rtcc_ctx* c, int k) {
   CK(cudaEventRecord(b.done, b.st));
   b.launched = true;
   c->ctrl.mark(k, RTCC_RUNNING);
+  c->present_dirty = true;
   c->info.t_release_ms[k] = now_ms();
   if (c->info.n_dispatched < RTCC_MAX_AGENTS) c->info.dispatch_order[c->info.n_dispatched++] = k;
   return RTCC_OK;
 }
 
 rtcc_status launch_post(rtcc_ctx* c) {
-  for (int k = 0; k < c->K; ++k) {
-    const bool pres = c->ctrl.present(k);
-    c->h_present[k] = pres ? 1 : 0;
-    if (pres) CK(cudaStreamWaitEvent(c->post, c->br[k].done, 0));
-  }
-  CK(cudaMemcpyAsync(c->d_present, c->h_present, RTCC_MAX_AGENTS * 4, cudaMemcpyHostToDevice,
-                     c->post));
+  // the presence flags are set on the device by the branches that ran (their
+  // first kernel) and cleared by the decode kernel
+  for (int k = 0; k < c->K; ++k)
+    if (c->ctrl.present(k)) CK(cudaStreamWaitEvent(c->post, c->br[k].done, 0));
+  *c->h_done = 0;                                 // the decode kernel sets it when the boxes are written
+  std::atomic_thread_fence(std::memory_order_seq_cst);
   CK(cudaGraphLaunch(c->post_exec, c->post));
   CK(cudaEventRecord(c->det_ready, c->post));
   c->post_launched = true;
@@ -834,6 +840,13 @@ rtcc_status rtcc_frame_begin(rtcc_ctx* c, uint64_t frame_id, double t0_ms) {
   if (!c) return RTCC_E_ARG;
   std::lock_guard<std::mutex> lk(c->mu);
   RS(c->ctrl.begin(frame_id, t0_ms));
+  if (c->present_dirty) {
+    // a previous frame launched branches but ran no post-join to clear their
+    // presence flags
+    for (int k = 0; k < c->K; ++k) CK(cudaStreamSynchronize(c->br[k].st));
+    CK(cudaMemset(c->d_present, 0, RTCC_MAX_AGENTS * 4));
+    c->present_dirty = false;
+  }
   c->post_launched = false;
   c->t_last_event = 0.0;
   std::memset(&c->info, 0, sizeof(c->info));
@@ -901,20 +914,36 @@ rtcc_status rtcc_wait_detection(rtcc_ctx* c, int32_t timeout_ms, rtcc_box* out, 
     if (c->ctrl.aborted()) {
       for (int k = 0; k < c->K; ++k)
         if (c->br[k].launched) cudaStreamSynchronize(c->br[k].st);
+      // no decode ran to clear the presence flags of the branches that did
+      if (cudaMemset(c->d_present, 0, RTCC_MAX_AGENTS * 4) != cudaSuccess) return RTCC_E_CUDA;
+      c->present_dirty = false;
       c->ctrl.end();
       return RTCC_E_INFEASIBLE;
     }
     if (!c->post_launched) return RTCC_E_STATE;
     ev = c->det_ready;
   }
+  // The decode kernel writes the result block into pinned host memory and then
+  // sets h_done; spinning on that word sees the result without a driver call.
+  // Every 4096 polls the post stream's event is queried for errors (and to
+  // notice a post-join that completed without setting the word).
   const double t0 = now_ms();
-  while (true) {
-    const cudaError_t q = cudaEventQuery(ev);
-    if (q == cudaSuccess) break;
-    if (q != cudaErrorNotReady) return RTCC_E_CUDA;
-    if (timeout_ms >= 0 && now_ms() - t0 > (double)timeout_ms) return RTCC_E_TIMEOUT;
+  for (uint32_t it = 1;; ++it) {
+    if (*c->h_done) break;
+    if ((it & 4095u) == 0) {
+      const cudaError_t q = cudaEventQuery(ev);
+      if (q != cudaSuccess && q != cudaErrorNotReady) return RTCC_E_CUDA;
+      if (q == cudaSuccess && !*c->h_done) return RTCC_E_CUDA;
+      if (timeout_ms >= 0 && now_ms() - t0 > (double)timeout_ms) return RTCC_E_TIMEOUT;
+    }
   }
   const double t_ready = now_ms();
+  std::atomic_thread_fence(std::memory_order_acquire);   // the block was written before the flag
+  c->present_dirty = false;                              // the decode cleared the presence flags
+  if (c->cfg.flags & RTCC_FLAG_TIMELINE) {
+    // the event nodes' times are read below: wait for the graph's end
+    if (cudaEventSynchronize(ev) != cudaSuccess) return RTCC_E_CUDA;
+  }
   std::lock_guard<std::mutex> lk(c->mu);
   const DetResultHeader* hdr = reinterpret_cast<const DetResultHeader*>(c->det_host);
   const rtcc_box* boxes = reinterpret_cast<const rtcc_box*>(hdr + 1);

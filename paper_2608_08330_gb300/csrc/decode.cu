@@ -228,7 +228,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 k_decode_select(const uint32_t* __restrict__ keys, uint32_t* __restrict__ hist0,
                 const float* __restrict__ head, int chunk4, int max_boxes, AnchorGeo g,
                 const int* __restrict__ err, DetResultHeader* __restrict__ hdr,
-                rtcc_box* __restrict__ boxes) {
+                rtcc_box* __restrict__ boxes, int* __restrict__ present, int K,
+                volatile int* __restrict__ done) {
   extern __shared__ unsigned long long bnd[];        // [kBndCap] keys of bin b0
   __shared__ int hist[kThreads];                     // level-1/2 histograms (10 bits)
   __shared__ unsigned long long sel[kDecodeKeep];    // selected, unordered
@@ -271,120 +272,128 @@ k_decode_select(const uint32_t* __restrict__ keys, uint32_t* __restrict__ hist0,
     hdr->n_boxes = need;
     hdr->err = *err;
   }
-  if (need == 0) return;
-  const uint32_t b0 = static_cast<uint32_t>(s_bin);
-  const int below0 = s_below;
-  const int nb0 = s_nb;
-  bool done = false;
+  if (need > 0) {
+    const uint32_t b0 = static_cast<uint32_t>(s_bin);
+    const int below0 = s_below;
+    const int nb0 = s_nb;
+    bool ranked = false;
 
-  if (nb0 <= kBndCap) {
-    // ---- 2. one coalesced pass: lower bins -> sel, bin b0 -> bnd ----------
-    for_strided(keys, n4, [&](uint32_t k, int i) {
-      const uint32_t bin = k >> 20;                    // invalid keys: bin 4095 > b0
-      const unsigned long long e = (static_cast<unsigned long long>(k) << 32) | static_cast<unsigned>(i);
-      const bool valid = k != kInvalid;
-      warp_append(valid && bin < b0, e, &s_nsel, sel);
-      warp_append(valid && bin == b0, e, &s_nl, bnd);
-    });
-    __syncthreads();                                   // every thread has read nb0
-    // ---- 3. level 1 over bnd (key bits 10..19 = pair bits 42..51) ---------
-    for (int i = tid; i < 1024; i += kThreads) hist[i] = 0;
-    __syncthreads();
-    for (int i = tid; i < nb0; i += kThreads) atomicAdd(&hist[(int)((bnd[i] >> 42) & 1023)], 1);
-    __syncthreads();
-    {
-      int run = block_scan_excl(hist[tid], &s_total);  // 1024 bins, one per thread
-      const int h = hist[tid];
-      if (below0 + run < need && below0 + run + h >= need) {
-        s_bin = tid;
-        s_below = below0 + run;
-      }
-      __syncthreads();
-    }
-    const int b1 = s_bin, below1 = s_below, nb1 = hist[b1];
-    if (nb1 <= kTieCap) {
-      // bin-1 entries below b1 are selected; those in b1 compete for the rest
-      for (int i = tid; i < nb0; i += kThreads) {
-        const unsigned long long e = bnd[i];
-        const int bin1 = (int)((e >> 42) & 1023);
-        warp_append(bin1 < b1, e, &s_nsel, sel);
-        warp_append(bin1 == b1, e, &s_nt, tie);
-      }
-      __syncthreads();
-      // ---- 4. order sel (below1 pairs) and tie (nb1 pairs, all above);
-      // ---- 5. each ranked pair is decoded straight into its box slot
-      // (bnd is free again and serves as the run buffer)
-      const int P1 = sort_width(below1), P2 = sort_width(nb1);
-      sort_phase1(sel, below1, 0, P1, bnd, head, g.anchors);
-      sort_phase1(tie, nb1, kDecodeKeep, P2, bnd + kDecodeKeep, head, g.anchors);
-      __syncthreads();
-      sort_phase2(bnd, 0, P1, below1,
-                  [&](int r, unsigned long long v) { decode_box(v, head, g, boxes + r); });
-      sort_phase2(bnd + kDecodeKeep, kDecodeKeep, P2, need - below1,
-                  [&](int r, unsigned long long v) { decode_box(v, head, g, boxes + below1 + r); });
-      done = true;
-    }
-  }
-
-  if (!done) {
-    __syncthreads();                                   // every thread has read hist
-    // ---- 2'. radix select over the global keys: levels 1 and 2 (10 bits
-    // each) below the bin-0 prefix give the exact K-th key T and the count
-    // `below` of keys < T ---------------------------------------------------
-    uint32_t prefix = b0 << 20, pmask = 0xFFFu << 20;
-    int below = below0;
-    const int lo = tid * chunk4 * 4;
-    for (int lv = 1; lv <= 2; ++lv) {
-      const int sh = lv == 1 ? 10 : 0;
+    if (nb0 <= kBndCap) {
+      // ---- 2. one coalesced pass: lower bins -> sel, bin b0 -> bnd ----------
+      for_strided(keys, n4, [&](uint32_t k, int i) {
+        const uint32_t bin = k >> 20;                    // invalid keys: bin 4095 > b0
+        const unsigned long long e = (static_cast<unsigned long long>(k) << 32) | static_cast<unsigned>(i);
+        const bool valid = k != kInvalid;
+        warp_append(valid && bin < b0, e, &s_nsel, sel);
+        warp_append(valid && bin == b0, e, &s_nl, bnd);
+      });
+      __syncthreads();                                   // every thread has read nb0
+      // ---- 3. level 1 over bnd (key bits 10..19 = pair bits 42..51) ---------
       for (int i = tid; i < 1024; i += kThreads) hist[i] = 0;
       __syncthreads();
-      for_chunk(keys, lo, chunk4, [&](uint32_t k, int) {
-        if (k != kInvalid && (k & pmask) == prefix) atomicAdd(&hist[(k >> sh) & 1023], 1);
-      });
+      for (int i = tid; i < nb0; i += kThreads) atomicAdd(&hist[(int)((bnd[i] >> 42) & 1023)], 1);
       __syncthreads();
-      int run = block_scan_excl(hist[tid], &s_total);
-      const int h = hist[tid];
-      if (below + run < need && below + run + h >= need) {
-        s_bin = tid;
-        s_below = below + run;
+      {
+        int run = block_scan_excl(hist[tid], &s_total);  // 1024 bins, one per thread
+        const int h = hist[tid];
+        if (below0 + run < need && below0 + run + h >= need) {
+          s_bin = tid;
+          s_below = below0 + run;
+        }
+        __syncthreads();
       }
-      __syncthreads();
-      prefix |= static_cast<uint32_t>(s_bin) << sh;
-      pmask |= 1023u << sh;
-      below = s_below;
-      __syncthreads();
+      const int b1 = s_bin, below1 = s_below, nb1 = hist[b1];
+      if (nb1 <= kTieCap) {
+        // bin-1 entries below b1 are selected; those in b1 compete for the rest
+        for (int i = tid; i < nb0; i += kThreads) {
+          const unsigned long long e = bnd[i];
+          const int bin1 = (int)((e >> 42) & 1023);
+          warp_append(bin1 < b1, e, &s_nsel, sel);
+          warp_append(bin1 == b1, e, &s_nt, tie);
+        }
+        __syncthreads();
+        // ---- 4. order sel (below1 pairs) and tie (nb1 pairs, all above);
+        // ---- 5. each ranked pair is decoded straight into its box slot
+        // (bnd is free again and serves as the run buffer)
+        const int P1 = sort_width(below1), P2 = sort_width(nb1);
+        sort_phase1(sel, below1, 0, P1, bnd, head, g.anchors);
+        sort_phase1(tie, nb1, kDecodeKeep, P2, bnd + kDecodeKeep, head, g.anchors);
+        __syncthreads();
+        sort_phase2(bnd, 0, P1, below1,
+                    [&](int r, unsigned long long v) { decode_box(v, head, g, boxes + r); });
+        sort_phase2(bnd + kDecodeKeep, kDecodeKeep, P2, need - below1,
+                    [&](int r, unsigned long long v) { decode_box(v, head, g, boxes + below1 + r); });
+        ranked = true;
+      }
     }
-    const uint32_t T = prefix;
-    if (tid == 0) s_nsel = 0;
-    __syncthreads();
-    // collect keys < T, then the (need - below) lowest-index keys equal to T:
-    // each thread owns a contiguous range of anchors and a block scan ranks
-    // its ties
-    int ties = 0;
-    for_chunk(keys, lo, chunk4, [&](uint32_t k, int i) {
-      if (k < T) {
-        sel[atomicAdd(&s_nsel, 1)] = (static_cast<unsigned long long>(k) << 32) | static_cast<unsigned>(i);
-      } else if (k == T) {
-        ++ties;
+
+    if (!ranked) {
+      __syncthreads();                                   // every thread has read hist
+      // ---- 2'. radix select over the global keys: levels 1 and 2 (10 bits
+      // each) below the bin-0 prefix give the exact K-th key T and the count
+      // `below` of keys < T ---------------------------------------------------
+      uint32_t prefix = b0 << 20, pmask = 0xFFFu << 20;
+      int below = below0;
+      const int lo = tid * chunk4 * 4;
+      for (int lv = 1; lv <= 2; ++lv) {
+        const int sh = lv == 1 ? 10 : 0;
+        for (int i = tid; i < 1024; i += kThreads) hist[i] = 0;
+        __syncthreads();
+        for_chunk(keys, lo, chunk4, [&](uint32_t k, int) {
+          if (k != kInvalid && (k & pmask) == prefix) atomicAdd(&hist[(k >> sh) & 1023], 1);
+        });
+        __syncthreads();
+        int run = block_scan_excl(hist[tid], &s_total);
+        const int h = hist[tid];
+        if (below + run < need && below + run + h >= need) {
+          s_bin = tid;
+          s_below = below + run;
+        }
+        __syncthreads();
+        prefix |= static_cast<uint32_t>(s_bin) << sh;
+        pmask |= 1023u << sh;
+        below = s_below;
+        __syncthreads();
       }
-    });
-    int tie_base = block_scan_excl(ties, &s_total);
-    const int take = need - below;
-    if (ties > 0 && tie_base < take) {
+      const uint32_t T = prefix;
+      if (tid == 0) s_nsel = 0;
+      __syncthreads();
+      // collect keys < T, then the (need - below) lowest-index keys equal to T:
+      // each thread owns a contiguous range of anchors and a block scan ranks
+      // its ties
+      int ties = 0;
       for_chunk(keys, lo, chunk4, [&](uint32_t k, int i) {
-        if (k == T && tie_base < take) {
-          sel[below + tie_base] = (static_cast<unsigned long long>(T) << 32) | static_cast<unsigned>(i);
-          ++tie_base;
+        if (k < T) {
+          sel[atomicAdd(&s_nsel, 1)] = (static_cast<unsigned long long>(k) << 32) | static_cast<unsigned>(i);
+        } else if (k == T) {
+          ++ties;
         }
       });
+      int tie_base = block_scan_excl(ties, &s_total);
+      const int take = need - below;
+      if (ties > 0 && tie_base < take) {
+        for_chunk(keys, lo, chunk4, [&](uint32_t k, int i) {
+          if (k == T && tie_base < take) {
+            sel[below + tie_base] = (static_cast<unsigned long long>(T) << 32) | static_cast<unsigned>(i);
+            ++tie_base;
+          }
+        });
+      }
+      __syncthreads();
+      const int P = sort_width(need);
+      sort_phase1(sel, need, 0, P, bnd, head, g.anchors);
+      __syncthreads();
+      sort_phase2(bnd, 0, P, need,
+                  [&](int r, unsigned long long v) { decode_box(v, head, g, boxes + r); });
     }
-    __syncthreads();
-    const int P = sort_width(need);
-    sort_phase1(sel, need, 0, P, bnd, head, g.anchors);
-    __syncthreads();
-    sort_phase2(bnd, 0, P, need,
-                [&](int r, unsigned long long v) { decode_box(v, head, g, boxes + r); });
-  }
+  }  // need > 0
+
+  // the fusion kernel has read the presence flags: clear them for the next
+  // frame, then publish the result block to the host
+  if (tid < K) present[tid] = 0;
+  __threadfence_system();                          // this thread's box writes, system-wide
+  __syncthreads();
+  if (tid == 0) *done = 1;
 }
 
 
@@ -413,8 +422,10 @@ cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t st) {
   cudaError_t e = cudaFuncSetAttribute(k_decode_select, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)dyn);
   if (e != cudaSuccess) return e;
+  if (!a.present || !a.done || a.K < 1 || a.K > RTCC_MAX_AGENTS) return cudaErrorInvalidValue;
   return launch_pdl(k_decode_select, dim3(1), dim3(kThreads), dyn, st, a.keys, a.hist0, a.head,
-                    decode_key_chunk4(n), a.max_boxes, g, a.err, hdr, boxes);
+                    decode_key_chunk4(n), a.max_boxes, g, a.err, hdr, boxes, a.present, a.K,
+                    a.done);
 }
 
 }  // namespace rtcc

@@ -62,6 +62,7 @@ struct PillarBufs {
                          //         points of kept pillars before the N_max cap
   int* cell2pillar;      // [H*W]     -1 where no kept pillar
   void* image;           // [H][W][C] storage type, zeros where no kept pillar
+  int* present_flag;     // optional: set to 1 by the pass (the agent's slot is filled)
   int cap, P, N, C;
   int clear_all;         // 1: the pass clears all of image and cell2pillar (their
                          // content is unknown); 0: they hold the previous pass's
@@ -204,7 +205,11 @@ struct DecodeArgs {
   float x_min, y_min, x_max, y_max;
   int max_boxes;
   const int* err;            // device error word, copied into the result header
-  void* out;                 // device result block: DetResultHeader + rtcc_box[max_boxes]
+  void* out;                 // result block DetResultHeader + rtcc_box[max_boxes], in
+                             // pinned host memory (written directly by the kernel)
+  int* present;              // device [K] per-agent presence flags: cleared for the next frame
+  int K;
+  volatile int* done;        // pinned host word: set to 1 once `out` is complete
 };
 constexpr int kDecodeKeep = 512;     // largest supported max_boxes
 constexpr int kDecodeHistBins = 4096;
@@ -214,7 +219,7 @@ inline size_t decode_key_capacity(int n_anchors) {
 }
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t st);
 
-// Result block the post-join graph copies to pinned host memory.
+// Result block the decode kernel writes into pinned host memory.
 struct DetResultHeader {
   int n_boxes;
   int err;

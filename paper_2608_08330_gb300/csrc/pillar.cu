@@ -44,11 +44,12 @@ __global__ void k_pillar_cells(const float4* __restrict__ pts, const int* __rest
                                int* __restrict__ first_cell, int* __restrict__ stats,
                                const int* __restrict__ prev_cell, const int* __restrict__ np_prev,
                                int clear_all, uint4* __restrict__ image,
-                               int* __restrict__ cell2pillar) {
+                               int* __restrict__ cell2pillar, int* __restrict__ present_flag) {
   pdl_trigger();
   pdl_wait();
   const int n = *n_hdr;
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i == 0 && present_flag) *present_flag = 1;     // this agent's slot is filled this frame
   // clear what the previous pass wrote (CH 16-byte chunks per cell)
   {
     const long long stride = (long long)gridDim.x * blockDim.x;
@@ -388,7 +389,7 @@ cudaError_t launch_all(const PillarBufs& b, const GridGeom& g, const float* pfn_
   e = launch_pdl(k_pillar_cells<CH>, dim3((b.cap + 255) / 256), dim3(256), 0, st, b.pts, b.n_hdr,
                  g, b.cell_of, b.cnt_cell, b.first_cell, b.stats,
                  static_cast<const int*>(b.pillar_cell), static_cast<const int*>(b.np_prev),
-                 b.clear_all, static_cast<uint4*>(b.image), b.cell2pillar);
+                 b.clear_all, static_cast<uint4*>(b.image), b.cell2pillar, b.present_flag);
   if (e != cudaSuccess) return e;
   e = launch_pdl(k_pillar_blocksum, dim3(nblk), dim3(kScanThreads), 0, st, b.n_hdr, b.cell_of,
                  b.cnt_cell, b.first_cell, b.items, b.blocksum);
