@@ -577,6 +577,7 @@ rtcc_status capture_post(rtcc_ctx* c) {
     tp.C = c->Cf;
     tp.cells = fa.cells;
     tp.bkc = bkc;
+    tp.stages = fuse_tc_stages(c->Cf, c->K);
     tp.head_b = c->head_b;
     tp.head_out = c->head_out;
     tp.fused = c->fused;

@@ -17,8 +17,11 @@
 // unsigned integer whose ascending order is descending logit order, or
 // 0xFFFFFFFF below the threshold) with a histogram of its top 12 bits.
 //
-// Roles (192 threads): warp 0 = TMA producer, warp 1 = tensor-memory owner and
-// MMA issuer, warps 2..5 = max workers and epilogue.  The slots hold ReLU
+// Roles (320 threads): warp 0 = TMA producer, warp 1 = tensor-memory owner and
+// MMA issuer, warps 2..9 = max workers, of which warps 2..5 (one tensor-memory
+// lane quarter each) also run the epilogue.  The workers write the
+// max into one of two fused-chunk buffers and release the agent stage at
+// once, so the producer refills it while the MMA still reads the fused chunk.  The slots hold ReLU
 // outputs, so the 16-bit max is exact and matches the agent-index-order max;
 // the MMA's summation order is fixed by the hardware, so the output is
 // bit-reproducible.  Every wait is bounded (an error bit, no hang).
@@ -29,13 +32,16 @@ namespace rtcc {
 
 namespace {
 
-constexpr int kThreads = 192;
+constexpr int kThreads = 320;
+constexpr int kWorkers = kThreads - 64;        // warps 2..9 take the max; warps 2..5 the epilogue
 constexpr int kTile = 128;                     // cells per work item (MMA M)
-constexpr int kStages = 3;
-constexpr int kStageBytes = 64 * 1024;         // present agents x 128 cells x chunk x 2 B
+constexpr int kMaxStages = 8;
+constexpr int kStageArea = 176 * 1024;         // agent-chunk stages
 constexpr int kMaxC = 512;
+constexpr int kFBytes = kTile * 64 * 2;        // one fused chunk (bkc <= 64)
 constexpr int kWBytes = kFuseHeadOut * kMaxC * 2;
-constexpr int kSmem = kStages * kStageBytes + kWBytes + 1024 + 256;
+constexpr int kSmem = kStageArea + 2 * kFBytes + kWBytes + 1024 + 256;
+static_assert(kSmem <= 227 * 1024, "shared memory budget");
 
 template <typename T>
 __device__ __forceinline__ uint32_t max2(uint32_t a, uint32_t b);
@@ -73,16 +79,51 @@ __device__ __forceinline__ void hist_add(uint32_t* hist0, bool keep, uint32_t ke
   if (keep && lane == __ffs(peers) - 1) atomicAdd(&hist0[bin], (uint32_t)__popc(peers));
 }
 
+// Element-wise max of the KP present agents' copies of one staged chunk (nvec
+// 16-byte vectors each, agent i at st + i * nvec) into fb, by the worker
+// threads; 0 agents give zeros.  KP fixed at compile time lets the loads of
+// two vectors be in flight together.
+template <typename T, int KP>
+__device__ __forceinline__ void max_chunk(const uint4* __restrict__ st, uint4* __restrict__ fb,
+                                          int nvec, int wt) {
+#pragma unroll 2
+  for (int v = wt; v < nvec; v += kWorkers) {
+    uint4 m = make_uint4(0u, 0u, 0u, 0u);
+    if (KP > 0) m = st[v];
+#pragma unroll
+    for (int i = 1; i < KP; ++i) m = max8<T>(m, st[i * nvec + v]);
+    fb[v] = m;
+  }
+}
+template <typename T>
+__device__ __forceinline__ void max_chunk_any(const uint4* st, uint4* fb, int nvec, int wt, int kp) {
+  switch (kp) {
+    case 0: max_chunk<T, 0>(st, fb, nvec, wt); break;
+    case 1: max_chunk<T, 1>(st, fb, nvec, wt); break;
+    case 2: max_chunk<T, 2>(st, fb, nvec, wt); break;
+    case 3: max_chunk<T, 3>(st, fb, nvec, wt); break;
+    case 4: max_chunk<T, 4>(st, fb, nvec, wt); break;
+    default:
+      for (int v = wt; v < nvec; v += kWorkers) {
+        uint4 m = st[v];
+        for (int i = 1; i < kp; ++i) m = max8<T>(m, st[i * nvec + v]);
+        fb[v] = m;
+      }
+  }
+}
+
 template <typename T>
 __global__ void __launch_bounds__(kThreads, 1) k_fuse_max_head(const __grid_constant__ FuseTcParams P) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint8_t* wsm = smem + kStages * kStageBytes;
-  uint64_t* full = reinterpret_cast<uint64_t*>(wsm + kWBytes);
-  uint64_t* ready = full + kStages;            // fused chunk written (128 arrivals)
-  uint64_t* empty = ready + kStages;           // MMA has read the stage
-  uint64_t* accfull = empty + kStages;         // [2]
+  uint8_t* fbuf = smem + kStageArea;           // [2] fused chunks (the MMA's A operand)
+  uint8_t* wsm = fbuf + 2 * kFBytes;           // head weights [C / bkc][16][bkc]
+  uint64_t* full = reinterpret_cast<uint64_t*>(wsm + kWBytes);   // [kMaxStages] agent chunks landed
+  uint64_t* empty = full + kMaxStages;         // [kMaxStages] workers have read the stage
+  uint64_t* fready = empty + kMaxStages;       // [2] fused chunk written
+  uint64_t* fempty = fready + 2;               // [2] MMA has read the fused chunk
+  uint64_t* accfull = fempty + 2;              // [2]
   uint64_t* accempty = accfull + 2;            // [2] (4 arrivals)
   uint64_t* wbar = accempty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(wbar + 1);
@@ -94,17 +135,20 @@ __global__ void __launch_bounds__(kThreads, 1) k_fuse_max_head(const __grid_cons
   const int C = P.C, bkc = P.bkc;
   const int nch = C / bkc;
   const int slot_bytes = kTile * bkc * 2;
+  const int stage_bytes = P.K * slot_bytes;    // room for every configured agent
+  const int nst = P.stages;
   const int tiles = (P.cells + kTile - 1) / kTile;
 
   if (warp == 0 && lane == 0) {
-    for (int s = 0; s < kStages; ++s) {
+    for (int s = 0; s < nst; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&ready[s], 128);
-      mbar_init(&empty[s], 1);
+      mbar_init(&empty[s], kWorkers);
     }
-    for (int a = 0; a < 2; ++a) {
-      mbar_init(&accfull[a], 1);
-      mbar_init(&accempty[a], 4);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&fready[b], kWorkers);
+      mbar_init(&fempty[b], 1);
+      mbar_init(&accfull[b], 1);
+      mbar_init(&accempty[b], 4);
     }
     mbar_init(wbar, 1);
     fence_barrier_init();
@@ -137,34 +181,34 @@ __global__ void __launch_bounds__(kThreads, 1) k_fuse_max_head(const __grid_cons
 
   if (warp == 0) {
     if (lane == 0) {
-      // ---------------- TMA producer ----------------
+      // ---------------- TMA producer: agent chunks -> stages ----------------
       for (int k = 0; k < Kp; ++k) tma_prefetch_desc(&P.feat[s_list[k]]);
       uint32_t it = 0;
       bool alive = true;
       for (int t = blockIdx.x; t < tiles && alive; t += gridDim.x) {
         for (int j = 0; j < nch; ++j, ++it) {
-          const int s = it % kStages;
-          if (!mbar_wait(&empty[s], ((it / kStages) & 1) ^ 1)) {
+          const int s = it % nst;
+          if (!mbar_wait(&empty[s], ((it / nst) & 1) ^ 1)) {
             atomicOr(P.err, ERR_WAIT_FUSE);
             alive = false;
             break;
           }
           mbar_arrive_expect_tx(&full[s], (uint32_t)(Kp * slot_bytes));
           for (int i = 0; i < Kp; ++i)
-            tma_load_2d(smem + s * kStageBytes + i * slot_bytes, &P.feat[s_list[i]], &full[s],
+            tma_load_2d(smem + s * stage_bytes + i * slot_bytes, &P.feat[s_list[i]], &full[s],
                         j * bkc, t * kTile);
         }
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
-      // ---------------- MMA issuer ----------------
+      // ---------------- MMA issuer: fused chunk x head weights ----------------
       bool alive = mbar_wait(wbar, 0);
       if (!alive) atomicOr(P.err, ERR_WAIT_FUSE);
       const uint32_t idesc = idesc_f16(kTile, kFuseHeadOut, std::is_same<T, __nv_bfloat16>::value);
       const uint32_t swz = bkc == 64 ? 2u : 4u;   // 128B : 64B swizzle
       const uint32_t sbo = 8u * bkc * 2u;          // bytes between 8-row atoms
-      const uint32_t a0 = smem_u32(smem), w0 = smem_u32(wsm);
+      const uint32_t f0 = smem_u32(fbuf), w0 = smem_u32(wsm);
       uint32_t it = 0, tc = 0;
       for (int t = blockIdx.x; t < tiles && alive; t += gridDim.x, ++tc) {
         const int acc = tc & 1;
@@ -175,25 +219,26 @@ __global__ void __launch_bounds__(kThreads, 1) k_fuse_max_head(const __grid_cons
         tc_fence_after();
         const uint32_t d_tmem = tmem + acc * kFuseHeadOut;
         for (int j = 0; j < nch; ++j, ++it) {
-          const int s = it % kStages;
-          if (!mbar_wait(&ready[s], (it / kStages) & 1)) {
+          const int b = it & 1;
+          if (!mbar_wait(&fready[b], (it >> 1) & 1)) {
             atomicOr(P.err, ERR_WAIT_FUSE);
             alive = false;
             break;
           }
           tc_fence_after();
-          const uint64_t ad = smem_desc(a0 + s * kStageBytes, sbo, swz);
+          const uint64_t ad = smem_desc(f0 + b * kFBytes, sbo, swz);
           const uint64_t bd = smem_desc(w0 + j * kFuseHeadOut * bkc * 2, sbo, swz);
           for (int kk = 0; kk < bkc / 16; ++kk)      // K advance: 32 bytes = +2
             umma_f16(d_tmem, ad + 2 * kk, bd + 2 * kk, idesc, (j > 0 || kk > 0) ? 1u : 0u);
-          umma_commit(&empty[s]);
+          umma_commit(&fempty[b]);
         }
         umma_commit(&accfull[acc]);
       }
     }
   } else {
     // ---------------- max workers + epilogue ----------------
-    const int wt = threadIdx.x - 64;           // 0..127
+    const int wt = threadIdx.x - 64;           // 0..kWorkers-1
+    const bool epi = warp < 6;                 // warps 2..5: one TMEM lane quarter each
     const int qd = warp & 3;                   // tensor-memory lane quarter of this warp
     const int row = qd * 32 + lane;            // cell within the tile
     float hb[kFuseHeadOut];
@@ -206,30 +251,37 @@ __global__ void __launch_bounds__(kThreads, 1) k_fuse_max_head(const __grid_cons
     bool alive = true;
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++tc) {
       for (int j = 0; j < nch; ++j, ++it) {
-        const int s = it % kStages;
-        if (alive && !mbar_wait(&full[s], (it / kStages) & 1)) {
+        const int s = it % nst, b = it & 1;
+        if (alive && !mbar_wait(&full[s], (it / nst) & 1)) {
           atomicOr(P.err, ERR_WAIT_FUSE);
           alive = false;
         }
-        uint4* s0 = reinterpret_cast<uint4*>(smem + s * kStageBytes);
-        for (int v = wt; v < nvec; v += 128) {
-          uint4 m = make_uint4(0u, 0u, 0u, 0u);  // no agent present: F = 0
-          if (Kp > 0) m = s0[v];
-          for (int i = 1; i < Kp; ++i) m = max8<T>(m, s0[i * nvec + v]);
-          if (Kp != 1) s0[v] = m;
-          if (fused) {
+        // the fused buffer must have been read by the MMA of two chunks ago
+        if (alive && !mbar_wait(&fempty[b], ((it >> 1) & 1) ^ 1)) {
+          atomicOr(P.err, ERR_WAIT_FUSE);
+          alive = false;
+        }
+        const uint4* st = reinterpret_cast<const uint4*>(smem + s * stage_bytes);
+        uint4* fb = reinterpret_cast<uint4*>(fbuf + b * kFBytes);
+        max_chunk_any<T>(st, fb, nvec, wt, Kp);
+        if (fused) {
+          // debug copy of the fused features, unswizzled to [cell][C]
+          for (int v = wt; v < nvec; v += kWorkers) {
             const int r = v / vpr, ch = v - r * vpr;
             const int x = (bkc == 64) ? (r & 7) : ((r >> 1) & 3);
             const int cell = t * kTile + r;
             if (cell < P.cells)
-              *reinterpret_cast<uint4*>(fused + (size_t)cell * C + j * bkc + ((ch ^ x) << 3)) = m;
+              *reinterpret_cast<uint4*>(fused + (size_t)cell * C + j * bkc + ((ch ^ x) << 3)) = fb[v];
           }
         }
-        // generic-proxy writes of the fused chunk -> visible to the MMA
+        // the stage is read: hand it back to the producer at once; the fused
+        // chunk (generic-proxy writes) goes to the MMA
+        mbar_arrive(&empty[s]);
         fence_async_smem();
-        mbar_arrive(&ready[s]);
+        mbar_arrive(&fready[b]);
       }
-      // epilogue of tile t
+      // epilogue of tile t (warps 2..5)
+      if (!epi) continue;
       const int acc = tc & 1;
       if (alive && !mbar_wait(&accfull[acc], (tc >> 1) & 1)) {
         if (lane == 0) atomicOr(P.err, ERR_WAIT_FUSE);
@@ -273,13 +325,21 @@ __global__ void __launch_bounds__(kThreads, 1) k_fuse_max_head(const __grid_cons
 
 int fuse_tc_chunk(int C, int K) {
   if (C % 32 != 0 || C > kMaxC || K < 1 || K > RTCC_MAX_AGENTS) return 0;
-  const int bkc = (C % 64 == 0 && K * kTile * 64 * 2 <= kStageBytes) ? 64 : 32;
-  return K * kTile * bkc * 2 <= kStageBytes ? bkc : 0;
+  // 64-channel chunks while at least 3 stages of K agent chunks fit, else 32
+  if (C % 64 == 0 && 3 * K * kTile * 64 * 2 <= kStageArea) return 64;
+  return 2 * K * kTile * 32 * 2 <= kStageArea ? 32 : 0;
+}
+
+int fuse_tc_stages(int C, int K) {
+  const int bkc = fuse_tc_chunk(C, K);
+  if (bkc == 0) return 0;
+  const int n = kStageArea / (K * kTile * bkc * 2);
+  return n < kMaxStages ? n : kMaxStages;
 }
 
 cudaError_t launch_fuse_max_head(const FuseTcParams& p, bool bf16, cudaStream_t st) {
-  if (p.bkc != fuse_tc_chunk(p.C, p.K) || p.anchors < 1 || p.anchors > kFuseHeadOut ||
-      p.cells < 1)
+  if (p.bkc != fuse_tc_chunk(p.C, p.K) || p.stages != fuse_tc_stages(p.C, p.K) || p.stages < 2 ||
+      p.anchors < 1 || p.anchors > kFuseHeadOut || p.cells < 1)
     return cudaErrorInvalidValue;
   int dev = 0, sms = 148;
   cudaGetDevice(&dev);

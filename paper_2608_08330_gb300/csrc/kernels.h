@@ -172,7 +172,7 @@ struct FuseTcParams {
   CUtensorMap feat[RTCC_MAX_AGENTS];  // agent k's slot [cells][C], box (bkc, 128), swizzled
   CUtensorMap wmap;                   // head weights [16][C] in the storage type, box (bkc, 16)
   const int* present;                 // device [K]
-  int K, C, cells, bkc;
+  int K, C, cells, bkc, stages;
   const float* head_b;                // device [16]
   float* head_out;                    // device [cells][16]
   void* fused;                        // device [cells][C] or null
@@ -185,6 +185,7 @@ struct FuseTcParams {
 // Channel chunk (64 or 32) the kernel stages for C channels and K agent slots,
 // 0 if it cannot run that shape.
 int fuse_tc_chunk(int C, int K);
+int fuse_tc_stages(int C, int K);   // pipeline stages for that chunk
 cudaError_t launch_fuse_max_head(const FuseTcParams& p, bool bf16, cudaStream_t st);
 
 // Row-major 2-D 16-bit tensor map [outer][inner] with a box of
