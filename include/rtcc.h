@@ -92,6 +92,10 @@ typedef enum {
                                     so each can be read back (parity)         */
 #define RTCC_FLAG_LAYER_TIMES 8  /* record the GPU time at which the backbone
                                     kernel starts each conv/deconv layer       */
+#define RTCC_FLAG_NO_CLUSTERS 16 /* launch the backbone without thread-block
+                                    clusters: split-K slices then reduce
+                                    through global memory instead of
+                                    distributed shared memory (same results)  */
 
 /*
  * Network and workload description.  Supported: 1 <= n_agents <= 8;

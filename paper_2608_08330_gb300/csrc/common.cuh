@@ -241,6 +241,13 @@ __device__ __forceinline__ uint32_t cluster_ctarank() {
   return r;
 }
 
+// CTAs in this CTA's cluster as launched (1 without a cluster launch).
+__device__ __forceinline__ uint32_t cluster_nctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
+  return r;
+}
+
 // Address of the same shared-memory location in CTA `rank` of the cluster.
 __device__ __forceinline__ uint32_t mapa_shared(uint32_t saddr, uint32_t rank) {
   uint32_t r;

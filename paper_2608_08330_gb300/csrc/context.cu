@@ -500,7 +500,8 @@ rtcc_status build_branch(rtcc_ctx* c, int k) {
   }
   b.bb = new (std::nothrow) BackboneParams;
   if (!b.bb) return RTCC_E_NOMEM;
-  if (backbone_fill(b.layers, b.grid_bar, c->d_err, b.stamps, b.bb) != cudaSuccess)
+  if (backbone_fill(b.layers, b.grid_bar, c->d_err, b.stamps,
+                    (g.flags & RTCC_FLAG_NO_CLUSTERS) == 0, b.bb) != cudaSuccess)
     return RTCC_E_ARG;
   CK(cudaStreamCreateWithFlags(&b.st, cudaStreamNonBlocking));
   CK(cudaEventCreateWithFlags(&b.h2d_done, cudaEventDisableTiming));

@@ -215,6 +215,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const unsigned G = gridDim.x;
+  // The DSMEM reduction needs the launch to be in clusters of kMaxSplits CTAs;
+  // the cluster size is read from the hardware, not trusted from the
+  // parameters, and without such clusters split layers reduce through global
+  // memory (the workspace exists for every split layer).
+  const uint32_t ncl = cluster_nctarank();
+  const bool clustered = ncl == (uint32_t)kMaxSplits;
 
   if (warp == 0 && lane == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -227,7 +233,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
     }
     mbar_init(recvbar, 1);                     // the owner's arrival + the peers' bytes
     fence_barrier_init();
-    if (P.cluster > 1) fence_mbar_init_cluster();
+    if (ncl > 1) fence_mbar_init_cluster();
   }
   if (warp == 1) {
     tmem_alloc(tmem_slot, kTmemCols);
@@ -235,7 +241,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
   }
   tc_fence_before();
   __syncthreads();
-  if (P.cluster > 1) cluster_sync_all();      // peers' barriers are initialised
+  if (ncl > 1) cluster_sync_all();            // peers' barriers are initialised
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   pdl_trigger();
@@ -386,7 +392,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
             tmem_ld16(taddr + c0, v);
             stage16<T>(stage, sg, row, c0, v, bias + c0);
           }
-        } else if (S.dsm) {
+        } else if (S.dsm && clustered) {
           // The kMaxSplits K-slices of this tile sit on the CTAs of this
           // cluster, slice z on rank z.  Reduce-scatter through distributed
           // shared memory: rank z owns CW = bn / kMaxSplits output channels
@@ -563,7 +569,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
 
   tc_fence_before();
   __syncthreads();
-  if (P.cluster > 1) cluster_sync_all();      // no peer still writes into this CTA
+  if (ncl > 1) cluster_sync_all();            // no peer still writes into this CTA
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
@@ -689,14 +695,14 @@ cudaError_t conv_make_maps(ConvLayer& L, bool bf16) {
 }
 
 cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, unsigned* grid_bar, int* err,
-                          unsigned long long* stamps, BackboneParams* P) {
+                          unsigned long long* stamps, bool allow_clusters, BackboneParams* P) {
   if (layers.empty() || layers.size() > (size_t)kMaxLayers) return cudaErrorInvalidValue;
   std::memset(P, 0, sizeof(*P));
   P->n_layers = (int)layers.size();
   P->grid_bar = grid_bar;
   P->err = err;
   P->stamps = stamps;
-  const int grid_sm = backbone_grid(1), grid_cl = backbone_grid(kMaxSplits);
+  const int grid_sm = backbone_grid(1), grid_cl = allow_clusters ? backbone_grid(kMaxSplits) : 0;
   if (grid_sm < 1) return cudaErrorInvalidValue;
   bool any_dsm = false;
   for (size_t i = 0; i < layers.size(); ++i) {

@@ -139,7 +139,7 @@ struct BackboneParams {
 // Fill the kernel parameters of a branch's backbone from its layer list;
 // grid_bar holds kMaxLayers counters.
 cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, unsigned* grid_bar, int* err,
-                          unsigned long long* stamps, BackboneParams* P);
+                          unsigned long long* stamps, bool allow_clusters, BackboneParams* P);
 // One cooperative launch (one CTA per SM) running every layer.
 cudaError_t launch_backbone(const BackboneParams& P, bool bf16, cudaStream_t st);
 // CTAs of a backbone launch: every SM (cluster = 1), or as many CTAs as can be

@@ -28,6 +28,7 @@ FUSE_MAX, FUSE_ATTN = 0, 1
 FP16, BF16 = 0, 1
 WAITING, RELEASED, RUNNING, FINISHED, ABSENT = range(5)
 FLAG_TIMELINE, FLAG_KEEP_FUSED, FLAG_KEEP_LAYERS, FLAG_LAYER_TIMES = 1, 2, 4, 8
+FLAG_NO_CLUSTERS = 16
 TENSOR_IMAGE, TENSOR_FEAT, TENSOR_FUSED, TENSOR_LAYER0 = 0, 8, 9, 16
 
 

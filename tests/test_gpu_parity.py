@@ -192,6 +192,28 @@ def test_decode_all_equal_logits(R, grid):
         R.rtcc_destroy(ctx)
 
 
+def test_split_k_without_clusters_bit_identical(R):
+    # The deepest block's 4-way split-K reduces through distributed shared
+    # memory when the backbone runs in clusters of four CTAs, and through
+    # global memory without clusters; both sum the slices in slice order, so
+    # the outputs must match bit for bit (and the oracle within tolerance).
+    cfg = _small_pp()
+    pts = [synth.points_for(cfg, 0, k) for k in range(cfg.n_agents)]
+    heads = []
+    for flags in (U.DEBUG_FLAGS, U.DEBUG_FLAGS | R.FLAG_NO_CLUSTERS):
+        ctx, w = U.make_ctx(cfg, flags=flags)
+        try:
+            U.run_frame(ctx, cfg, pts, [0.0, 1.0, 2.0], R.MODE_RTCC)
+            heads.append(R.rtcc_get_head(ctx, cfg.feat_h, cfg.feat_w).copy())
+            if flags & R.FLAG_NO_CLUSTERS:
+                hd = _check_frame(R, ctx, cfg, w, pts)
+                full = of.forward(pts, w, cfg, store=cfg.dtype)
+                U.assert_close(hd, full["head"], "head (no clusters)")
+        finally:
+            R.rtcc_destroy(ctx)
+    assert heads[0].tobytes() == heads[1].tobytes()
+
+
 @pytest.mark.parametrize("name", ["tiny", "small_pp", "small_attn"])
 def test_rtcc_and_barrier_bit_identical(R, name):
     if name == "tiny":
