@@ -40,9 +40,11 @@ import synth  # noqa: E402
 
 METRIC = "complete-detection latency p50/p99 ms RTCC vs barrier; conv TFLOP/s, fusion GB/s"
 # dram__bytes_read.sum + dram__bytes_write.sum of one k_backbone launch (one pp3
-# branch) from an ncu capture of this build; None once the kernel changes and
-# until it is captured again
-BACKBONE_TRAFFIC = None
+# branch) from an ncu capture of this build (the profiler replays the launch
+# without its cluster dimension, so block 3 reduced its split-K partials
+# through global memory; they stay in L2 either way); None once the kernel
+# changes and until it is captured again
+BACKBONE_TRAFFIC = 16_538_624
 WORKLOAD = "pp3"
 DATA = ("synthetic: seeded uniform + Gaussian-cluster point clouds, He-normal fp32 weights "
         "rounded to fp16, seeded arrival traces (OPV2V and the trained OpenCOOD model are not "
