@@ -49,7 +49,8 @@ struct Branch {
   std::vector<ConvLayer> layers;
   float* splitk_ws = nullptr;      // split-K partials, shared by the branch's layers
   int* splitk_cnt = nullptr;       // split-K per-tile arrival counters
-  unsigned* grid_bar = nullptr;    // backbone per-layer arrival counters
+  unsigned* grid_bar = nullptr;      // inside frame_zero
+  void* frame_zero = nullptr;         // [kFrameZeroBytes] cleared at the start of every branch graph    // backbone per-layer arrival counters
   unsigned long long* stamps = nullptr;   // RTCC_FLAG_LAYER_TIMES: layer start times
   BackboneParams* bb = nullptr;    // backbone kernel parameters (host copy)
   cudaStream_t st = nullptr;
@@ -330,6 +331,8 @@ void pick_tile(int m_tiles, int co, int total_kb, int grid, int* bn_out, int* sp
   *sp_out = bs;
 }
 
+constexpr size_t kFrameZeroBytes = 8 * sizeof(int) + kMaxLayers * sizeof(unsigned);
+
 rtcc_status build_branch(rtcc_ctx* c, int k) {
   Branch& b = c->br[k];
   const rtcc_model_config& g = c->cfg;
@@ -366,7 +369,11 @@ rtcc_status build_branch(rtcc_ctx* c, int k) {
   p.present_flag = c->d_present + k;
   RS(dalloc(c, &p.pillar_cell, (size_t)c->P * 4));
   RS(dalloc(c, &p.pcount, (size_t)c->P * 4));
-  RS(dalloc(c, &p.stats, 8 * 4));
+  // words cleared at the start of every branch graph (one memset): the pillar
+  // stats [8] and the backbone's per-layer arrival counters [kMaxLayers]
+  RS(dalloc(c, &b.frame_zero, kFrameZeroBytes));
+  CK(cudaMemset(b.frame_zero, 0, kFrameZeroBytes));
+  p.stats = reinterpret_cast<int*>(b.frame_zero);
   RS(dalloc(c, &p.cell2pillar, (size_t)cells * 4));
   RS(dalloc(c, &p.image, (size_t)cells * c->Cp * es));
   CK(cudaMemset(p.cnt_cell, 0, (size_t)cells * 4));
@@ -492,8 +499,7 @@ rtcc_status build_branch(rtcc_ctx* c, int k) {
     L.ws = b.splitk_ws;
     L.counters = b.splitk_cnt;
   }
-  RS(dalloc(c, &b.grid_bar, kMaxLayers * sizeof(unsigned)));
-  CK(cudaMemset(b.grid_bar, 0, kMaxLayers * sizeof(unsigned)));
+  b.grid_bar = reinterpret_cast<unsigned*>(static_cast<uint8_t*>(b.frame_zero) + 8 * sizeof(int));
   if (g.flags & RTCC_FLAG_LAYER_TIMES) {
     RS(dalloc(c, &b.stamps, (b.layers.size() + 1) * sizeof(unsigned long long)));
     CK(cudaMemset(b.stamps, 0, (b.layers.size() + 1) * sizeof(unsigned long long)));
@@ -527,10 +533,11 @@ rtcc_status capture_branch(rtcc_ctx* c, int k) {
   CK(cudaStreamBeginCapture(b.st, cudaStreamCaptureModeRelaxed));
   cudaError_t e = cudaSuccess;
   if (tl) e = record_node(b.ev_start, b.st);
-  if (e == cudaSuccess) e = cudaMemsetAsync(b.pb.stats, 0, 8 * sizeof(int), b.st);
+  // one memset of the per-frame words, then kernels only, so that the pillar
+  // chain and the backbone are programmatic dependent launches of each other
+  if (e == cudaSuccess) e = cudaMemsetAsync(b.frame_zero, 0, kFrameZeroBytes, b.st);
   if (e == cudaSuccess) e = launch_pillarise(b.pb, gg, c->pfn_w, c->pfn_b, c->bf16, c->d_err, b.st);
   if (e == cudaSuccess && tl) e = record_node(b.ev_bb0, b.st);
-  if (e == cudaSuccess) e = cudaMemsetAsync(b.grid_bar, 0, kMaxLayers * sizeof(unsigned), b.st);
   if (e == cudaSuccess) e = launch_backbone(*b.bb, c->bf16, b.st);
   if (e == cudaSuccess && tl) e = record_node(b.ev_bb1, b.st);
   if (e == cudaSuccess && tl) e = record_node(b.ev_end, b.st);

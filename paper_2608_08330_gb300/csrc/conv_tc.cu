@@ -245,7 +245,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   pdl_trigger();
-  pdl_wait();                                  // the pseudo-image is the previous kernel's output
+  // the pseudo-image is the previous kernel's output; the producer waits for it
+  // only after it has issued layer 0's weight boxes
+  if (warp != 0) pdl_wait();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -282,6 +284,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
           }
           if (!alive) break;
         }
+        if (l == 0) pdl_wait();
         if (S.wait_layers > 0) {
           // every CTA has finished layer wait_layers - 1 (and, as each CTA
           // runs its layers in order, every layer before it)
@@ -801,15 +804,23 @@ cudaError_t launch_backbone(const BackboneParams& P, bool bf16, cudaStream_t st)
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = kSmem;
   cfg.stream = st;
-  cudaLaunchAttribute attr[2];
-  attr[0].id = cudaLaunchAttributeCooperative;   // every CTA resident: grid barriers are safe
-  attr[0].val.cooperative = 1;
-  attr[1].id = cudaLaunchAttributeClusterDimension;
-  attr[1].val.clusterDim.x = (unsigned)P.cluster;
-  attr[1].val.clusterDim.y = 1;
-  attr[1].val.clusterDim.z = 1;
+  cudaLaunchAttribute attr[3];
+  int na = 0;
+  attr[na].id = cudaLaunchAttributeCooperative;  // every CTA resident: grid barriers are safe
+  attr[na++].val.cooperative = 1;
+  // programmatic dependent launch: CTAs are scheduled while the pillar chain
+  // drains and run their prologue (barriers, TMEM, cluster sync, first weight
+  // boxes) before griddepcontrol.wait
+  attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[na++].val.programmaticStreamSerializationAllowed = 1;
+  if (P.cluster > 1) {
+    attr[na].id = cudaLaunchAttributeClusterDimension;
+    attr[na].val.clusterDim.x = (unsigned)P.cluster;
+    attr[na].val.clusterDim.y = 1;
+    attr[na++].val.clusterDim.z = 1;
+  }
   cfg.attrs = attr;
-  cfg.numAttrs = P.cluster > 1 ? 2 : 1;
+  cfg.numAttrs = na;
   if (bf16) return cudaLaunchKernelEx(&cfg, k_backbone<__nv_bfloat16>, P);
   return cudaLaunchKernelEx(&cfg, k_backbone<__half>, P);
 }
