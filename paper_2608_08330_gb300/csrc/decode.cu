@@ -17,7 +17,8 @@
 //   4. the selected pairs are ordered (warp bitonic runs of 32, then a rank by
 //      binary search in the other runs; the pairs are distinct) and the
 //      lowest-ranked pairs of bin b1 complete the K;
-//   5. each ranked pair is decoded into the box of its rank.
+//   5. each ranked pair is decoded into the box of its rank (staged in shared
+//      memory, then stored into the pinned host result block).
 // When bin b0 or b1 is too full for the shared-memory lists (e.g. many equal
 // logits), a radix select over the global keys (next 10 + 10 bits) finds the
 // exact K-th key instead, the keys below it are collected, and an ordered pass
@@ -38,6 +39,7 @@ constexpr int kThreads = 1024;
 constexpr int kMaxBins = 4096;
 constexpr int kBndCap = 4096;                // keys of bin b0 held in shared memory
 constexpr int kTieCap = 64;                  // keys of the level-1 bin ranked directly
+static_assert(sizeof(DetResultHeader) % 16 == 0, "the boxes follow the header 16-byte aligned");
 
 struct AnchorGeo {
   float x_min, y_min, sx, sy;       // cell size in metres
@@ -234,6 +236,7 @@ k_decode_select(const uint32_t* __restrict__ keys, uint32_t* __restrict__ hist0,
   __shared__ int hist[kThreads];                     // level-1/2 histograms (10 bits)
   __shared__ unsigned long long sel[kDecodeKeep];    // selected, unordered
   __shared__ unsigned long long tie[kTieCap];
+  __shared__ __align__(16) rtcc_box sbox[kDecodeKeep];  // boxes in rank order
   __shared__ int s_total, s_bin, s_below, s_nsel, s_nb, s_nl, s_nt;
   const int tid = threadIdx.x;
   const int n4 = chunk4 * kThreads;                   // 16-byte vectors of padded keys
@@ -282,10 +285,14 @@ k_decode_select(const uint32_t* __restrict__ keys, uint32_t* __restrict__ hist0,
       // ---- 2. one coalesced pass: lower bins -> sel, bin b0 -> bnd ----------
       for_strided(keys, n4, [&](uint32_t k, int i) {
         const uint32_t bin = k >> 20;                    // invalid keys: bin 4095 > b0
-        const unsigned long long e = (static_cast<unsigned long long>(k) << 32) | static_cast<unsigned>(i);
-        const bool valid = k != kInvalid;
-        warp_append(valid && bin < b0, e, &s_nsel, sel);
-        warp_append(valid && bin == b0, e, &s_nl, bnd);
+        const bool cand = k != kInvalid && bin <= b0;
+        // few keys are candidates (about K of tens of thousands): a warp
+        // skips the appends after one vote
+        if (__any_sync(__activemask(), cand)) {
+          const unsigned long long e = (static_cast<unsigned long long>(k) << 32) | static_cast<unsigned>(i);
+          warp_append(cand && bin < b0, e, &s_nsel, sel);
+          warp_append(cand && bin == b0, e, &s_nl, bnd);
+        }
       });
       __syncthreads();                                   // every thread has read nb0
       // ---- 3. level 1 over bnd (key bits 10..19 = pair bits 42..51) ---------
@@ -320,9 +327,9 @@ k_decode_select(const uint32_t* __restrict__ keys, uint32_t* __restrict__ hist0,
         sort_phase1(tie, nb1, kDecodeKeep, P2, bnd + kDecodeKeep, head, g.anchors);
         __syncthreads();
         sort_phase2(bnd, 0, P1, below1,
-                    [&](int r, unsigned long long v) { decode_box(v, head, g, boxes + r); });
+                    [&](int r, unsigned long long v) { decode_box(v, head, g, sbox + r); });
         sort_phase2(bnd + kDecodeKeep, kDecodeKeep, P2, need - below1,
-                    [&](int r, unsigned long long v) { decode_box(v, head, g, boxes + below1 + r); });
+                    [&](int r, unsigned long long v) { decode_box(v, head, g, sbox + below1 + r); });
         ranked = true;
       }
     }
@@ -384,8 +391,17 @@ k_decode_select(const uint32_t* __restrict__ keys, uint32_t* __restrict__ hist0,
       sort_phase1(sel, need, 0, P, bnd, head, g.anchors);
       __syncthreads();
       sort_phase2(bnd, 0, P, need,
-                  [&](int r, unsigned long long v) { decode_box(v, head, g, boxes + r); });
+                  [&](int r, unsigned long long v) { decode_box(v, head, g, sbox + r); });
     }
+    // the boxes leave shared memory in 16-byte pieces (coalesced stores into
+    // the pinned host block)
+    __syncthreads();
+    const int nbytes = need * (int)sizeof(rtcc_box);
+    const uint4* src = reinterpret_cast<const uint4*>(sbox);
+    uint4* dst = reinterpret_cast<uint4*>(boxes);
+    for (int i = tid; i < nbytes / 16; i += kThreads) dst[i] = src[i];
+    for (int i = (nbytes / 16) * 4 + tid; i < nbytes / 4; i += kThreads)
+      reinterpret_cast<uint32_t*>(boxes)[i] = reinterpret_cast<const uint32_t*>(sbox)[i];
   }  // need > 0
 
   // the fusion kernel has read the presence flags: clear them for the next
