@@ -14,9 +14,9 @@
 //      lists the keys of bin b0 in shared memory;
 //   3. a histogram of the listed keys' next 10 bits splits them into selected
 //      ones, the few of the bin b1 that holds the K-th pair, and the rest;
-//   4. the selected pairs are ordered (warp bitonic runs of 32, then a rank by
-//      binary search in the other runs; the pairs are distinct) and the
-//      lowest-ranked pairs of bin b1 complete the K;
+//   4. the selected pairs are ordered (warp bitonic runs of 32, then merge
+//      levels that place each pair by one binary search in its partner run;
+//      the pairs are distinct) and the lowest pairs of bin b1 complete the K;
 //   5. each ranked pair is decoded into the box of its rank (staged in shared
 //      memory, then stored into the pinned host result block).
 // When bin b0 or b1 is too full for the shared-memory lists (e.g. many equal
@@ -155,15 +155,6 @@ __device__ __forceinline__ unsigned long long warp_sort32(unsigned long long v, 
   return v;
 }
 
-// Number of entries < v in a sorted run of 32.
-__device__ __forceinline__ int below_in_run(const unsigned long long* run, unsigned long long v) {
-  int pos = 0;
-#pragma unroll
-  for (int s = 16; s > 0; s >>= 1)
-    if (run[pos + s - 1] < v) pos += s;
-  return pos + (run[pos] < v ? 1 : 0);
-}
-
 // Sort of n <= 512 distinct (key, index) pairs in two block-wide phases,
 // run by the threads [t0, t0 + P) (P = n rounded up to a power of two >= 32):
 // phase 1 sorts runs of 32 in registers (warp bitonic) into run[0..P);
@@ -189,17 +180,28 @@ __device__ __forceinline__ void sort_phase1(const unsigned long long* in, int n,
     run[t] = warp_sort32(v, threadIdx.x & 31);
   }
 }
-template <typename F>
-__device__ __forceinline__ void sort_phase2(const unsigned long long* run, int t0, int P, int limit,
-                                            F emit) {
+// One level of the merge sort over warp-sorted runs, by the threads
+// [t0, t0 + P): the runs of R pairs in src[0..P) merge pairwise into runs of
+// 2R in dst.  A pair's place in the merged run is its index in its own run
+// plus the count of the partner run's pairs below it (left run: strictly
+// below; right run: below or equal), so every place is taken exactly once,
+// padding (~0) included.
+__device__ __forceinline__ void merge_level(const unsigned long long* src, unsigned long long* dst,
+                                            int t0, int P, int R) {
   const int t = threadIdx.x - t0;
-  if (t < 0 || t >= P) return;
-  const unsigned long long v = run[t];
-  if (v == ~0ull) return;                                // padding
-  int r = t & 31;
-  for (int q = 0; q < P / 32; ++q)
-    if (q != (t >> 5)) r += below_in_run(run + 32 * q, v);
-  if (r < limit) emit(r, v);
+  if (t < 0 || t >= P || R >= P) return;
+  const unsigned long long v = src[t];
+  const int base = t & ~(2 * R - 1);
+  const bool right = (t & R) != 0;
+  const unsigned long long* other = src + base + (right ? 0 : R);
+  int lo = 0, hi = R;
+  while (lo < hi) {
+    const int mid = (lo + hi) >> 1;
+    const unsigned long long o = other[mid];
+    if (right ? (o <= v) : (o < v)) lo = mid + 1;
+    else hi = mid;
+  }
+  dst[base + (t & (R - 1)) + lo] = v;
 }
 
 // Box of the selected pair v (anchor = its low 32 bits), written to out.
@@ -298,7 +300,14 @@ k_decode_select(const uint32_t* __restrict__ keys, uint32_t* __restrict__ hist0,
       // ---- 3. level 1 over bnd (key bits 10..19 = pair bits 42..51) ---------
       for (int i = tid; i < 1024; i += kThreads) hist[i] = 0;
       __syncthreads();
-      for (int i = tid; i < nb0; i += kThreads) atomicAdd(&hist[(int)((bnd[i] >> 42) & 1023)], 1);
+      // many listed keys share their next 10 bits: lanes with the same bin add
+      // their count with one atomic (uniform trip count: warps stay converged)
+      for (int i0 = 0; i0 < nb0; i0 += kThreads) {
+        const int i = i0 + tid;
+        const int bin1 = i < nb0 ? (int)((bnd[i] >> 42) & 1023) : -1;
+        const unsigned peers = __match_any_sync(0xFFFFFFFFu, bin1);
+        if (bin1 >= 0 && (tid & 31) == __ffs(peers) - 1) atomicAdd(&hist[bin1], __popc(peers));
+      }
       __syncthreads();
       {
         int run = block_scan_excl(hist[tid], &s_total);  // 1024 bins, one per thread
@@ -323,13 +332,21 @@ k_decode_select(const uint32_t* __restrict__ keys, uint32_t* __restrict__ hist0,
         // ---- 5. each ranked pair is decoded straight into its box slot
         // (bnd is free again and serves as the run buffer)
         const int P1 = sort_width(below1), P2 = sort_width(nb1);
-        sort_phase1(sel, below1, 0, P1, bnd, head, g.anchors);
-        sort_phase1(tie, nb1, kDecodeKeep, P2, bnd + kDecodeKeep, head, g.anchors);
+        unsigned long long *a = bnd, *a2 = bnd + 2 * kDecodeKeep;              // sel runs
+        unsigned long long *b = bnd + kDecodeKeep, *b2 = bnd + kDecodeKeep + kTieCap;  // tie runs
+        sort_phase1(sel, below1, 0, P1, a, head, g.anchors);
+        sort_phase1(tie, nb1, kDecodeKeep, P2, b, head, g.anchors);
         __syncthreads();
-        sort_phase2(bnd, 0, P1, below1,
-                    [&](int r, unsigned long long v) { decode_box(v, head, g, sbox + r); });
-        sort_phase2(bnd + kDecodeKeep, kDecodeKeep, P2, need - below1,
-                    [&](int r, unsigned long long v) { decode_box(v, head, g, sbox + below1 + r); });
+        for (int R = 32; R < (P1 > P2 ? P1 : P2); R *= 2) {
+          merge_level(a, a2, 0, P1, R);
+          merge_level(b, b2, kDecodeKeep, P2, R);
+          __syncthreads();
+          if (R < P1) { unsigned long long* x = a; a = a2; a2 = x; }
+          if (R < P2) { unsigned long long* x = b; b = b2; b2 = x; }
+        }
+        if (tid < below1) decode_box(a[tid], head, g, sbox + tid);
+        const int tt = tid - kDecodeKeep;
+        if (tt >= 0 && tt < need - below1) decode_box(b[tt], head, g, sbox + below1 + tt);
         ranked = true;
       }
     }
@@ -388,10 +405,17 @@ k_decode_select(const uint32_t* __restrict__ keys, uint32_t* __restrict__ hist0,
       }
       __syncthreads();
       const int P = sort_width(need);
-      sort_phase1(sel, need, 0, P, bnd, head, g.anchors);
+      unsigned long long *a = bnd, *a2 = bnd + 2 * kDecodeKeep;
+      sort_phase1(sel, need, 0, P, a, head, g.anchors);
       __syncthreads();
-      sort_phase2(bnd, 0, P, need,
-                  [&](int r, unsigned long long v) { decode_box(v, head, g, sbox + r); });
+      for (int R = 32; R < P; R *= 2) {
+        merge_level(a, a2, 0, P, R);
+        __syncthreads();
+        unsigned long long* x = a;
+        a = a2;
+        a2 = x;
+      }
+      if (tid < need) decode_box(a[tid], head, g, sbox + tid);
     }
     // the boxes leave shared memory in 16-byte pieces (coalesced stores into
     // the pinned host block)
