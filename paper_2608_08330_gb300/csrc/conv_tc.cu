@@ -51,12 +51,13 @@ constexpr int TW = 32;                       // tile width in pixels
 constexpr int TH = 4;                        // tile height
 constexpr int BM = TW * TH;                  // 128 = MMA M
 constexpr int kThreads = 192;
-constexpr int kStages = 6;
+constexpr int kStages = 5;
 constexpr int kABytes = BM * 64 * 2;         // A slot (BK <= 64)
 constexpr int kBBytes = 128 * 64 * 2;        // B slot (BN <= 128, BK <= 64)
 constexpr int kStageBytes = kABytes + kBBytes;
-constexpr int kStagingBytes = 32 * 1024;     // output tile (BN <= 128) or the DSMEM receive
-                                             // slots (3 x 128 x 16 fp32) + their output
+constexpr int kStagingBytes = 64 * 1024;     // output tile (BN <= 128: 32 KB), or for a DSMEM
+                                             // split the outgoing and receive slots (2 x 3 x
+                                             // 128 x 16 fp32) + the 16-channel output tile
 constexpr int kSmem = kStages * kStageBytes + kStagingBytes + 1024 + 256;
 constexpr uint32_t kTmemCols = 256;          // two 128-column accumulators
 
@@ -390,84 +391,113 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
         epilogue_sync();
         bool store = true;
         if (S.splits == 1) {
-          for (int c0 = 0; c0 < S.bn; c0 += 16) {
-            float v[16];
-            tmem_ld16(taddr + c0, v);
-            stage16<T>(stage, sg, row, c0, v, bias + c0);
+          // up to 64 columns per round: issue all TMEM loads, wait once
+          for (int c0 = 0; c0 < S.bn; c0 += 64) {
+            const int ng = (S.bn - c0) / 16 < 4 ? (S.bn - c0) / 16 : 4;   // uniform
+            uint32_t r[4][16];
+#pragma unroll
+            for (int g = 0; g < 4; ++g)
+              if (g < ng) tmem_ld16_issue(taddr + c0 + 16 * g, r[g]);
+            tmem_ld_wait();
+#pragma unroll
+            for (int g = 0; g < 4; ++g) {
+              if (g < ng) {
+                tmem_reg_fence(r[g]);
+                float v[16];
+#pragma unroll
+                for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[g][i]);
+                stage16<T>(stage, sg, row, c0 + 16 * g, v, bias + c0 + 16 * g);
+              }
+            }
           }
         } else if (S.dsm && clustered) {
           // The kMaxSplits K-slices of this tile sit on the CTAs of this
           // cluster, slice z on rank z.  Reduce-scatter through distributed
-          // shared memory: rank z owns CW = bn / kMaxSplits output channels
-          // [CW z, CW (z + 1)); each rank sends every owner its partial of the
-          // owner's channels (16-byte st.async into the owner's receive slots,
-          // counted on the owner's mbarrier), and the owner sums the slices in
-          // slice order and stores its channels in 16-channel TMA boxes.
-          const int CW = S.bn / kMaxSplits;                        // 16
+          // shared memory: rank z owns output channels [16z, 16z + 16); each
+          // rank writes its partial of every owner's channels into its own
+          // shared memory and moves each slot to its owner with one bulk copy
+          // (counted on the owner's mbarrier); the owner sums the slices in
+          // slice order and stores its channels in a 16-channel TMA box.  The
+          // outgoing slots are rewritten only after the next item's
+          // bulk_wait_read_all.
+          constexpr int CW = 16;                                   // bn = 16 * kMaxSplits
           const int z = I.z;
           if (row == 0 && cluster_ctarank() != (uint32_t)z) atomicOr(P.err, ERR_BOUNDS);
-          uint8_t* recv = stage;                                   // [kMaxSplits-1][BM][CW] fp32
-          uint8_t* out16 = stage + (kMaxSplits - 1) * BM * CW * 4; // [BM][16] 16-bit
-          if (row == 0) mbar_arrive_expect_tx(recvbar, (uint32_t)((kMaxSplits - 1) * BM * CW * 4));
-          const uint32_t my_recv = smem_u32(recv), my_bar = smem_u32(recvbar);
+          constexpr int SLOT = BM * CW * 4;                       // one slice of one owner: 8 KB
+          uint8_t* outg = stage;                                   // [kMaxSplits-1][BM][CW] fp32, to peers
+          uint8_t* recv = stage + (kMaxSplits - 1) * SLOT;         // [kMaxSplits-1][BM][CW] fp32, from peers
+          uint8_t* out16 = stage + 2 * (kMaxSplits - 1) * SLOT;    // [BM][16] 16-bit
+          if (row == 0) mbar_arrive_expect_tx(recvbar, (uint32_t)((kMaxSplits - 1) * SLOT));
+          // every rank's 16 columns of this row in one round of TMEM loads
+          uint32_t rq[kMaxSplits][16];
+#pragma unroll
+          for (int q = 0; q < kMaxSplits; ++q) tmem_ld16_issue(taddr + q * CW, rq[q]);
+          tmem_ld_wait();
+#pragma unroll
+          for (int q = 0; q < kMaxSplits; ++q) tmem_reg_fence(rq[q]);
+          // the peers' columns go to this CTA's outgoing slots, then one bulk
+          // copy per peer moves a whole slot into the peer's receive slot
+#pragma unroll
           for (int q = 0; q < kMaxSplits; ++q) {
             if (q == z) continue;                  // uniform over the CTA
-            const int slot = z < q ? z : z - 1;    // this rank's slot at owner q
-            const uint32_t dst = mapa_shared(my_recv + (uint32_t)((slot * BM + row) * CW * 4), q);
-            const uint32_t bar = mapa_shared(my_bar, q);
-            for (int c0 = 0; c0 < CW; c0 += 16) {
-              float v[16];
-              tmem_ld16(taddr + q * CW + c0, v);
+            const int oslot = q < z ? q : q - 1;   // outgoing slot of peer q
+            uint4* o = reinterpret_cast<uint4*>(outg + oslot * SLOT + row * CW * 4);
 #pragma unroll
-              for (int j = 0; j < 4; ++j)
-                st_async_v4(dst + (uint32_t)(c0 + 4 * j) * 4,
-                            make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]), bar);
+            for (int j = 0; j < 4; ++j)
+              o[j] = make_uint4(rq[q][4 * j], rq[q][4 * j + 1], rq[q][4 * j + 2], rq[q][4 * j + 3]);
+          }
+          fence_async_smem();                      // generic writes -> the bulk copies
+          epilogue_sync();
+          if (row == 0) {
+            const uint32_t my_recv = smem_u32(recv), my_bar = smem_u32(recvbar);
+            for (int q = 0; q < kMaxSplits; ++q) {
+              if (q == z) continue;
+              const int oslot = q < z ? q : q - 1;
+              const int slot = z < q ? z : z - 1;  // this rank's receive slot at owner q
+              bulk_copy_to_peer(mapa_shared(my_recv + (uint32_t)(slot * SLOT), q), outg + oslot * SLOT,
+                                (uint32_t)SLOT, mapa_shared(my_bar, q));
             }
+            bulk_commit();
           }
           if (alive && !mbar_wait(recvbar, dsm_phase)) {
             if (lane == 0) atomicOr(P.err, ERR_WAIT_EPILOGUE);
             alive = false;
           }
           dsm_phase ^= 1u;
-          for (int c0 = 0; c0 < CW; c0 += 16) {
-            float own[16];
-            tmem_ld16(taddr + z * CW + c0, own);
-            float sum[16];
+          float sum[16];
 #pragma unroll
-            for (int j = 0; j < 16; ++j) sum[j] = 0.f;
-            for (int zz = 0; zz < kMaxSplits; ++zz) {
-              if (zz == z) {
+          for (int j = 0; j < 16; ++j) sum[j] = 0.f;
 #pragma unroll
-                for (int j = 0; j < 16; ++j) sum[j] += own[j];
-              } else {
-                const int slot = zz < z ? zz : zz - 1;
-                const float4* src =
-                    reinterpret_cast<const float4*>(recv + ((slot * BM + row) * CW + c0) * 4);
+          for (int zz = 0; zz < kMaxSplits; ++zz) {
+            if (zz == z) {
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                  const float4 f = src[q];
-                  sum[4 * q] += f.x;
-                  sum[4 * q + 1] += f.y;
-                  sum[4 * q + 2] += f.z;
-                  sum[4 * q + 3] += f.w;
-                }
+              for (int j = 0; j < 16; ++j) sum[j] += __uint_as_float(rq[zz][j]);
+            } else {
+              const int slot = zz < z ? zz : zz - 1;
+              const float4* src = reinterpret_cast<const float4*>(recv + slot * SLOT + row * CW * 4);
+#pragma unroll
+              for (int q = 0; q < 4; ++q) {
+                const float4 f = src[q];
+                sum[4 * q] += f.x;
+                sum[4 * q + 1] += f.y;
+                sum[4 * q + 2] += f.z;
+                sum[4 * q + 3] += f.w;
               }
             }
-            // bias + ReLU, 16-bit, staged [BM][16] per group (32-byte rows)
-            const float* bz = bias + z * CW + c0;
-            uint32_t pk[8];
-#pragma unroll
-            for (int j = 0; j < 8; ++j)
-              pk[j] = Store<T>::pack2(relu_f(sum[2 * j] + bz[2 * j]), relu_f(sum[2 * j + 1] + bz[2 * j + 1]));
-            uint4* o = reinterpret_cast<uint4*>(out16 + (c0 / 16) * BM * 32 + row * 32);
-            o[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-            o[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
           }
+          // bias + ReLU, 16-bit, staged [BM][16] (32-byte rows, no swizzle)
+          const float* bz = bias + z * CW;
+          uint32_t pk[8];
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            pk[j] = Store<T>::pack2(relu_f(sum[2 * j] + bz[2 * j]), relu_f(sum[2 * j + 1] + bz[2 * j + 1]));
+          uint4* o = reinterpret_cast<uint4*>(out16 + row * 32);
+          o[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+          o[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
           fence_async_smem();
           epilogue_sync();
           if (row == 0) {
-            for (int c0 = 0; c0 < CW; c0 += 16)
-              tma_store_3d(mapC16, out16 + (c0 / 16) * BM * 32, I.n0 + z * CW + c0, I.x0, I.y0);
+            tma_store_3d(mapC16, out16, I.n0 + z * CW, I.x0, I.y0);
             bulk_commit();
           }
           store = false;
