@@ -306,9 +306,10 @@ rtcc_status upload_weights(rtcc_ctx* c, const float* w) {
 // persistent backbone kernel: one tcgen05 MMA instruction costs about the same
 // for every N <= 128, so a k-block costs the same for every N tile; a CTA
 // holds one item at a time, so items beyond the grid take another round; a
-// split into kMaxSplits slices of a 64-wide tile (one item per CTA) is reduced
-// through distributed shared memory at about the cost of 6 k-blocks (the
-// measured cost of 128-wide splits, with twice the exchange, was far higher).
+// split of a 64-wide tile into kMaxSplits slices (one item per CTA) is reduced
+// through distributed shared memory at about the cost of 7 k-blocks.  Measured
+// on the 64x64x128 block, a 2-way split (9 k-blocks per slice) was slower than
+// 32-wide tiles without split (18 k-blocks), so only 4-way splits are used.
 // Ties go to the narrower tile (more CTAs).
 void pick_tile(int m_tiles, int co, int total_kb, int grid, int* bn_out, int* sp_out) {
   double best = 1e30;
@@ -319,7 +320,7 @@ void pick_tile(int m_tiles, int co, int total_kb, int grid, int* bn_out, int* sp
       const int items = m_tiles * (co / bn) * sp;
       if (sp > 1 && (bn != 64 || total_kb / sp < 4 || items > grid)) continue;
       const int rounds = (items + grid - 1) / grid;
-      const double cost = rounds * (double)((total_kb + sp - 1) / sp) + (sp > 1 ? 6.0 : 0.0);
+      const double cost = rounds * (double)((total_kb + sp - 1) / sp) + (sp > 1 ? 7.0 : 0.0);
       if (cost < best - 1e-9) {
         best = cost;
         bb = bn;

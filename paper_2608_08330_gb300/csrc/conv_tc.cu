@@ -411,51 +411,49 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
             }
           }
         } else if (S.dsm && clustered) {
-          // The kMaxSplits K-slices of this tile sit on the CTAs of this
-          // cluster, slice z on rank z.  Reduce-scatter through distributed
-          // shared memory: rank z owns output channels [16z, 16z + 16); each
-          // rank writes its partial of every owner's channels into its own
-          // shared memory and moves each slot to its owner with one bulk copy
-          // (counted on the owner's mbarrier); the owner sums the slices in
-          // slice order and stores its channels in a 16-channel TMA box.  The
-          // outgoing slots are rewritten only after the next item's
-          // bulk_wait_read_all.
-          constexpr int CW = 16;                                   // bn = 16 * kMaxSplits
+          // The Sp = splits (2 or 4) K-slices of this 64-wide tile sit on Sp
+          // consecutive ranks of this cluster of four, slice z on rank gb + z.
+          // Reduce-scatter through distributed shared memory: slice z owns the
+          // CW = 64 / Sp output channels [CW z, CW (z + 1)).  Every rank writes
+          // its 64 partial columns into its own shared memory by owner; one
+          // bulk copy per peer moves the peer's slot into the peer's receive
+          // slot (counted on the peer's mbarrier); each owner sums the slices in
+          // slice order and stores its channels in 16-channel TMA boxes.  The
+          // slots are rewritten only after the next item's bulk_wait_read_all.
+          const int Sp = S.splits;
+          const int CW = 64 / Sp, G16 = CW / 16;
           const int z = I.z;
-          if (row == 0 && cluster_ctarank() != (uint32_t)z) atomicOr(P.err, ERR_BOUNDS);
-          constexpr int SLOT = BM * CW * 4;                       // one slice of one owner: 8 KB
-          uint8_t* outg = stage;                                   // [kMaxSplits-1][BM][CW] fp32, to peers
-          uint8_t* recv = stage + (kMaxSplits - 1) * SLOT;         // [kMaxSplits-1][BM][CW] fp32, from peers
-          uint8_t* out16 = stage + 2 * (kMaxSplits - 1) * SLOT;    // [BM][16] 16-bit
-          if (row == 0) mbar_arrive_expect_tx(recvbar, (uint32_t)((kMaxSplits - 1) * SLOT));
-          // every rank's 16 columns of this row in one round of TMEM loads
-          uint32_t rq[kMaxSplits][16];
+          const uint32_t rank = cluster_ctarank();
+          const uint32_t gb = rank & ~static_cast<uint32_t>(Sp - 1);
+          if (row == 0 && (rank & static_cast<uint32_t>(Sp - 1)) != (uint32_t)z) atomicOr(P.err, ERR_BOUNDS);
+          const int SLOT = BM * CW * 4;                          // one owner's channels, fp32
+          uint8_t* own = stage;                                  // [Sp][BM][CW] fp32, by owner (32 KB)
+          uint8_t* recv = stage + Sp * SLOT;                     // [Sp-1][BM][CW] fp32, from peers
+          uint8_t* out16 = recv + (Sp - 1) * SLOT;               // [G16][BM][16] 16-bit
+          if (row == 0) mbar_arrive_expect_tx(recvbar, (uint32_t)((Sp - 1) * SLOT));
+          // the row's 64 columns in one round of TMEM loads, into the owner slots
+          uint32_t rq[4][16];
 #pragma unroll
-          for (int q = 0; q < kMaxSplits; ++q) tmem_ld16_issue(taddr + q * CW, rq[q]);
+          for (int g = 0; g < 4; ++g) tmem_ld16_issue(taddr + 16 * g, rq[g]);
           tmem_ld_wait();
 #pragma unroll
-          for (int q = 0; q < kMaxSplits; ++q) tmem_reg_fence(rq[q]);
-          // the peers' columns go to this CTA's outgoing slots, then one bulk
-          // copy per peer moves a whole slot into the peer's receive slot
-#pragma unroll
-          for (int q = 0; q < kMaxSplits; ++q) {
-            if (q == z) continue;                  // uniform over the CTA
-            const int oslot = q < z ? q : q - 1;   // outgoing slot of peer q
-            uint4* o = reinterpret_cast<uint4*>(outg + oslot * SLOT + row * CW * 4);
+          for (int g = 0; g < 4; ++g) {
+            tmem_reg_fence(rq[g]);
+            const int q = g / G16, h = g - q * G16;
+            uint4* o = reinterpret_cast<uint4*>(own + q * SLOT + (row * CW + h * 16) * 4);
 #pragma unroll
             for (int j = 0; j < 4; ++j)
-              o[j] = make_uint4(rq[q][4 * j], rq[q][4 * j + 1], rq[q][4 * j + 2], rq[q][4 * j + 3]);
+              o[j] = make_uint4(rq[g][4 * j], rq[g][4 * j + 1], rq[g][4 * j + 2], rq[g][4 * j + 3]);
           }
           fence_async_smem();                      // generic writes -> the bulk copies
           epilogue_sync();
           if (row == 0) {
             const uint32_t my_recv = smem_u32(recv), my_bar = smem_u32(recvbar);
-            for (int q = 0; q < kMaxSplits; ++q) {
+            for (int q = 0; q < Sp; ++q) {
               if (q == z) continue;
-              const int oslot = q < z ? q : q - 1;
-              const int slot = z < q ? z : z - 1;  // this rank's receive slot at owner q
-              bulk_copy_to_peer(mapa_shared(my_recv + (uint32_t)(slot * SLOT), q), outg + oslot * SLOT,
-                                (uint32_t)SLOT, mapa_shared(my_bar, q));
+              const int slot = z < q ? z : z - 1;  // this slice's receive slot at owner q
+              bulk_copy_to_peer(mapa_shared(my_recv + (uint32_t)(slot * SLOT), gb + q), own + q * SLOT,
+                                (uint32_t)SLOT, mapa_shared(my_bar, gb + q));
             }
             bulk_commit();
           }
@@ -464,40 +462,37 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
             alive = false;
           }
           dsm_phase ^= 1u;
-          float sum[16];
+          for (int h = 0; h < G16; ++h) {
+            float sum[16];
 #pragma unroll
-          for (int j = 0; j < 16; ++j) sum[j] = 0.f;
-#pragma unroll
-          for (int zz = 0; zz < kMaxSplits; ++zz) {
-            if (zz == z) {
-#pragma unroll
-              for (int j = 0; j < 16; ++j) sum[j] += __uint_as_float(rq[zz][j]);
-            } else {
-              const int slot = zz < z ? zz : zz - 1;
-              const float4* src = reinterpret_cast<const float4*>(recv + slot * SLOT + row * CW * 4);
+            for (int j = 0; j < 16; ++j) sum[j] = 0.f;
+            for (int zz = 0; zz < Sp; ++zz) {
+              const uint8_t* src = (zz == z) ? own + z * SLOT : recv + (zz < z ? zz : zz - 1) * SLOT;
+              const float4* f4 = reinterpret_cast<const float4*>(src + (row * CW + h * 16) * 4);
 #pragma unroll
               for (int q = 0; q < 4; ++q) {
-                const float4 f = src[q];
+                const float4 f = f4[q];
                 sum[4 * q] += f.x;
                 sum[4 * q + 1] += f.y;
                 sum[4 * q + 2] += f.z;
                 sum[4 * q + 3] += f.w;
               }
             }
-          }
-          // bias + ReLU, 16-bit, staged [BM][16] (32-byte rows, no swizzle)
-          const float* bz = bias + z * CW;
-          uint32_t pk[8];
+            // bias + ReLU, 16-bit, staged [BM][16] per group (32-byte rows)
+            const float* bz = bias + z * CW + h * 16;
+            uint32_t pk[8];
 #pragma unroll
-          for (int j = 0; j < 8; ++j)
-            pk[j] = Store<T>::pack2(relu_f(sum[2 * j] + bz[2 * j]), relu_f(sum[2 * j + 1] + bz[2 * j + 1]));
-          uint4* o = reinterpret_cast<uint4*>(out16 + row * 32);
-          o[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-          o[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+            for (int j = 0; j < 8; ++j)
+              pk[j] = Store<T>::pack2(relu_f(sum[2 * j] + bz[2 * j]), relu_f(sum[2 * j + 1] + bz[2 * j + 1]));
+            uint4* o = reinterpret_cast<uint4*>(out16 + h * BM * 32 + row * 32);
+            o[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            o[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+          }
           fence_async_smem();
           epilogue_sync();
           if (row == 0) {
-            tma_store_3d(mapC16, out16, I.n0 + z * CW, I.x0, I.y0);
+            for (int h = 0; h < G16; ++h)
+              tma_store_3d(mapC16, out16 + h * BM * 32, I.n0 + z * CW + h * 16, I.x0, I.y0);
             bulk_commit();
           }
           store = false;
@@ -768,9 +763,10 @@ cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, unsigned* grid_b
     D.choff = L.choff;
     D.wait_layers = L.wait_layers;
     D.mapC16 = L.mapC16;
-    // a split of kMaxSplits 64-wide tiles with one item per CTA reduces its
-    // slices through distributed shared memory within a cluster
-    D.dsm = (L.kind != DECONV && L.splits == kMaxSplits && L.bn == 16 * kMaxSplits && grid_cl > 0 &&
+    // a split of a 64-wide tile into 2 or kMaxSplits slices, one item per
+    // CTA, reduces its slices through distributed shared memory within a
+    // cluster of kMaxSplits CTAs
+    D.dsm = (L.kind != DECONV && (L.splits == 2 || L.splits == kMaxSplits) && L.bn == 64 && grid_cl > 0 &&
              D.m_tiles * D.n_tiles * L.splits <= grid_cl)
                 ? 1
                 : 0;
