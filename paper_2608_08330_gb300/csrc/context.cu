@@ -54,7 +54,8 @@ struct Branch {
   unsigned long long* stamps = nullptr;   // RTCC_FLAG_LAYER_TIMES: layer start times
   BackboneParams* bb = nullptr;    // backbone kernel parameters (host copy)
   cudaStream_t st = nullptr;
-  cudaGraphExec_t exec = nullptr;
+  cudaGraphExec_t exec = nullptr;       // payload already in the device slot
+  cudaGraphExec_t exec_host = nullptr;  // payload in the pinned staging buffer (zero-copy)
   cudaEvent_t h2d_done = nullptr, done = nullptr;
   cudaEvent_t ev_start = nullptr, ev_bb0 = nullptr, ev_bb1 = nullptr, ev_end = nullptr;
   const float* pend_ptr = nullptr;
@@ -526,7 +527,7 @@ cudaError_t record_node(cudaEvent_t ev, cudaStream_t st) {
   return cudaEventRecordWithFlags(ev, st, cudaEventRecordExternal);
 }
 
-rtcc_status capture_branch(rtcc_ctx* c, int k) {
+rtcc_status capture_branch_graph(rtcc_ctx* c, int k, const PillarBufs& pb, cudaGraphExec_t* out) {
   Branch& b = c->br[k];
   const bool tl = (c->cfg.flags & RTCC_FLAG_TIMELINE) != 0;
   (void)cudaGetLastError();   // no stale error may leak into the launch checks
@@ -537,7 +538,7 @@ rtcc_status capture_branch(rtcc_ctx* c, int k) {
   // one memset of the per-frame words, then kernels only, so that the pillar
   // chain and the backbone are programmatic dependent launches of each other
   if (e == cudaSuccess) e = cudaMemsetAsync(b.frame_zero, 0, kFrameZeroBytes, b.st);
-  if (e == cudaSuccess) e = launch_pillarise(b.pb, gg, c->pfn_w, c->pfn_b, c->bf16, c->d_err, b.st);
+  if (e == cudaSuccess) e = launch_pillarise(pb, gg, c->pfn_w, c->pfn_b, c->bf16, c->d_err, b.st);
   if (e == cudaSuccess && tl) e = record_node(b.ev_bb0, b.st);
   if (e == cudaSuccess) e = launch_backbone(*b.bb, c->bf16, b.st);
   if (e == cudaSuccess && tl) e = record_node(b.ev_bb1, b.st);
@@ -548,9 +549,24 @@ rtcc_status capture_branch(rtcc_ctx* c, int k) {
     if (graph) cudaGraphDestroy(graph);
     return RTCC_E_CUDA;
   }
-  e = cudaGraphInstantiate(&b.exec, graph, 0);
+  e = cudaGraphInstantiate(out, graph, 0);
   cudaGraphDestroy(graph);
   return e == cudaSuccess ? RTCC_OK : RTCC_E_CUDA;
+}
+
+// Two graphs per branch: one for payloads already in the device slot, and
+// one whose first kernel reads the payload from the pinned staging buffer
+// (over the host link) and copies it into the device slot as it goes, so a
+// host payload needs no copy-engine transfer and no cross-stream event.
+rtcc_status capture_branch(rtcc_ctx* c, int k) {
+  Branch& b = c->br[k];
+  RS(capture_branch_graph(c, k, b.pb, &b.exec));
+  PillarBufs ph = b.pb;
+  ph.src_hdr = reinterpret_cast<const int*>(b.staging);
+  ph.src_pts = reinterpret_cast<const float4*>(reinterpret_cast<const uint8_t*>(b.staging) + kHdrBytes);
+  ph.dst_hdr = reinterpret_cast<int*>(b.in_dev);
+  ph.dst_pts = reinterpret_cast<float4*>(b.in_dev + kHdrBytes);
+  return capture_branch_graph(c, k, ph, &b.exec_host);
 }
 
 rtcc_status capture_post(rtcc_ctx* c) {
@@ -643,6 +659,7 @@ void free_all(rtcc_ctx* c) {
     Branch& b = c->br[k];
     if (b.st) cudaStreamSynchronize(b.st);
     if (b.exec) cudaGraphExecDestroy(b.exec);
+    if (b.exec_host) cudaGraphExecDestroy(b.exec_host);
     for (cudaEvent_t ev : {b.h2d_done, b.done, b.ev_start, b.ev_bb0, b.ev_bb1, b.ev_end})
       if (ev) cudaEventDestroy(ev);
     delete b.bb;
@@ -702,6 +719,7 @@ rtcc_status init_impl(rtcc_ctx* c, const float* weights) {
   RS(capture_post(c));
   // warm-up: every graph once on empty payloads (pays first-launch costs)
   for (int k = 0; k < c->K; ++k) CK(cudaGraphLaunch(c->br[k].exec, c->br[k].st));
+  for (int k = 0; k < c->K; ++k) CK(cudaGraphLaunch(c->br[k].exec_host, c->br[k].st));
   for (int k = 0; k < c->K; ++k) CK(cudaStreamSynchronize(c->br[k].st));
   CK(cudaGraphLaunch(c->post_exec, c->post));
   CK(cudaStreamSynchronize(c->post));
@@ -716,16 +734,17 @@ rtcc_status init_impl(rtcc_ctx* c, const float* weights) {
 rtcc_status launch_branch(rtcc_ctx* c, int k) {
   Branch& b = c->br[k];
   if (!b.pend_resident) {
+    // the branch's first kernel reads the payload from the pinned staging
+    // buffer and copies it to the device slot (no copy engine, no event)
     const int n = b.pend_n;
     float* pts = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(b.staging) + kHdrBytes);
     if (n > 0 && b.pend_ptr != pts) std::memcpy(pts, b.pend_ptr, (size_t)n * 16);
-    *reinterpret_cast<int*>(b.staging) = n;
-    CK(cudaMemcpyAsync(b.in_dev, b.staging, kHdrBytes + (size_t)n * 16, cudaMemcpyHostToDevice,
-                       c->xfer));
-    CK(cudaEventRecord(b.h2d_done, c->xfer));
-    CK(cudaStreamWaitEvent(b.st, b.h2d_done, 0));
+    *reinterpret_cast<volatile int*>(b.staging) = n;
+    std::atomic_thread_fence(std::memory_order_seq_cst);
+    CK(cudaGraphLaunch(b.exec_host, b.st));
+  } else {
+    CK(cudaGraphLaunch(b.exec, b.st));
   }
-  CK(cudaGraphLaunch(b.exec, b.st));
   CK(cudaEventRecord(b.done, b.st));
   b.launched = true;
   c->ctrl.mark(k, RTCC_RUNNING);

@@ -63,6 +63,13 @@ struct PillarBufs {
   int* cell2pillar;      // [H*W]     -1 where no kept pillar
   void* image;           // [H][W][C] storage type, zeros where no kept pillar
   int* present_flag;     // optional: set to 1 by the pass (the agent's slot is filled)
+  // optional zero-copy payload: the first kernel reads the header and points
+  // from src_* (e.g. pinned host memory) and writes them to dst_* (= n_hdr,
+  // pts) for the later kernels
+  const int* src_hdr;
+  const float4* src_pts;
+  int* dst_hdr;
+  float4* dst_pts;
   int cap, P, N, C;
   int clear_all;         // 1: the pass clears all of image and cell2pillar (their
                          // content is unknown); 0: they hold the previous pass's

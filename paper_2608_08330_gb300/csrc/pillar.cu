@@ -44,11 +44,19 @@ __global__ void k_pillar_cells(const float4* __restrict__ pts, const int* __rest
                                int* __restrict__ first_cell, int* __restrict__ stats,
                                const int* __restrict__ prev_cell, const int* __restrict__ np_prev,
                                int clear_all, uint4* __restrict__ image,
-                               int* __restrict__ cell2pillar, int* __restrict__ present_flag) {
+                               int* __restrict__ cell2pillar, int* __restrict__ present_flag,
+                               const int* __restrict__ src_hdr, const float4* __restrict__ src_pts,
+                               int* __restrict__ dst_hdr, float4* __restrict__ dst_pts) {
+  __shared__ int s_n;
   pdl_trigger();
   pdl_wait();
-  const int n = *n_hdr;
+  // zero-copy payload: one read of the header per block, every point read
+  // once from the source and copied to the device slot the later kernels use
+  if (threadIdx.x == 0) s_n = src_hdr ? *src_hdr : *n_hdr;
+  __syncthreads();
+  const int n = s_n;
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i == 0 && dst_hdr) *dst_hdr = n;
   if (i == 0 && present_flag) *present_flag = 1;     // this agent's slot is filled this frame
   // clear what the previous pass wrote (CH 16-byte chunks per cell)
   {
@@ -71,7 +79,8 @@ __global__ void k_pillar_cells(const float4* __restrict__ pts, const int* __rest
   if (i == 0) stats[0] = n;
   bool ok = false;
   if (i < n) {
-    const float4 p = pts[i];
+    const float4 p = src_pts ? src_pts[i] : pts[i];
+    if (dst_pts) dst_pts[i] = p;
     // IEEE float32 subtraction and division with round-to-nearest.
     const float fx = __fdiv_rn(__fsub_rn(p.x, g.x_min), g.v);
     const float fy = __fdiv_rn(__fsub_rn(p.y, g.y_min), g.v);
@@ -389,7 +398,8 @@ cudaError_t launch_all(const PillarBufs& b, const GridGeom& g, const float* pfn_
   e = launch_pdl(k_pillar_cells<CH>, dim3((b.cap + 255) / 256), dim3(256), 0, st, b.pts, b.n_hdr,
                  g, b.cell_of, b.cnt_cell, b.first_cell, b.stats,
                  static_cast<const int*>(b.pillar_cell), static_cast<const int*>(b.np_prev),
-                 b.clear_all, static_cast<uint4*>(b.image), b.cell2pillar, b.present_flag);
+                 b.clear_all, static_cast<uint4*>(b.image), b.cell2pillar, b.present_flag,
+                 b.src_hdr, b.src_pts, b.dst_hdr, b.dst_pts);
   if (e != cudaSuccess) return e;
   e = launch_pdl(k_pillar_blocksum, dim3(nblk), dim3(kScanThreads), 0, st, b.n_hdr, b.cell_of,
                  b.cnt_cell, b.first_cell, b.items, b.blocksum);
