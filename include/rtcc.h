@@ -90,8 +90,9 @@ typedef enum {
 #define RTCC_FLAG_KEEP_FUSED  2  /* also store the fused BEV map (parity)      */
 #define RTCC_FLAG_KEEP_LAYERS 4  /* give every conv layer its own output buffer
                                     so each can be read back (parity)         */
-#define RTCC_FLAG_LAYER_TIMES 8  /* record the GPU time at which the backbone
-                                    kernel starts each conv/deconv layer       */
+#define RTCC_FLAG_LAYER_TIMES 8  /* record the GPU times at which the backbone
+                                    kernel starts and ends each conv/deconv
+                                    layer                                     */
 #define RTCC_FLAG_NO_CLUSTERS 16 /* launch the backbone without thread-block
                                     clusters: split-K slices then reduce
                                     through global memory instead of
@@ -253,11 +254,21 @@ rtcc_status rtcc_get_frame_info(struct rtcc_ctx* ctx, rtcc_frame_info* info);
 
 /* Per-layer GPU times (ms) of `agent`'s conv and deconv layers in the last
  * closed frame, in order (13 convs then 3 deconvs for the PointPillars
- * backbone): the time between the backbone kernel starting consecutive layers
- * (the last layer: until every CTA finished it).  Needs
- * RTCC_FLAG_LAYER_TIMES.  *n_out receives the layer count. */
+ * backbone): for each layer, from the moment the backbone kernel's CTA that
+ * holds its first item has seen every input item stored, to the moment its
+ * last output item is counted.  Layers may overlap (the neck deconvs of the
+ * first two blocks run beside the deeper blocks), so the times do not add up
+ * to the backbone's time.  Needs RTCC_FLAG_LAYER_TIMES.  *n_out receives the
+ * layer count; entries beyond it are not written; -1 where a stamp is
+ * missing.  RTCC_E_STATE without the flag. */
 rtcc_status rtcc_get_layer_times(struct rtcc_ctx* ctx, int32_t agent, float* host_ms,
                                  int32_t cap, int32_t* n_out);
+
+/* The same stamps as start and end offsets (ms) from the earliest layer start
+ * of the backbone launch, so that overlapping layers can be laid out on one
+ * time axis.  Either array may be NULL. */
+rtcc_status rtcc_get_layer_spans(struct rtcc_ctx* ctx, int32_t agent, float* start_ms,
+                                 float* end_ms, int32_t cap, int32_t* n_out);
 
 /* State z_k of a branch in the open (or last) frame, and its release time
  * r_k in the caller's timebase (NaN while WAITING). */

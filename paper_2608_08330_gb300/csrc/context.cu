@@ -51,7 +51,7 @@ struct Branch {
   int* splitk_cnt = nullptr;       // split-K per-tile arrival counters
   unsigned* grid_bar = nullptr;      // inside frame_zero
   void* frame_zero = nullptr;         // [kFrameZeroBytes] cleared at the start of every branch graph    // backbone per-layer arrival counters
-  unsigned long long* stamps = nullptr;   // RTCC_FLAG_LAYER_TIMES: layer start times
+  unsigned long long* stamps = nullptr;   // RTCC_FLAG_LAYER_TIMES: layer starts, then ends
   BackboneParams* bb = nullptr;    // backbone kernel parameters (host copy)
   cudaStream_t st = nullptr;
   cudaGraphExec_t exec = nullptr;       // payload already in the device slot
@@ -503,8 +503,8 @@ rtcc_status build_branch(rtcc_ctx* c, int k) {
   }
   b.grid_bar = reinterpret_cast<unsigned*>(static_cast<uint8_t*>(b.frame_zero) + 8 * sizeof(int));
   if (g.flags & RTCC_FLAG_LAYER_TIMES) {
-    RS(dalloc(c, &b.stamps, (b.layers.size() + 1) * sizeof(unsigned long long)));
-    CK(cudaMemset(b.stamps, 0, (b.layers.size() + 1) * sizeof(unsigned long long)));
+    RS(dalloc(c, &b.stamps, 2 * b.layers.size() * sizeof(unsigned long long)));
+    CK(cudaMemset(b.stamps, 0, 2 * b.layers.size() * sizeof(unsigned long long)));
   }
   b.bb = new (std::nothrow) BackboneParams;
   if (!b.bb) return RTCC_E_NOMEM;
@@ -1006,8 +1006,8 @@ rtcc_status rtcc_get_frame_info(rtcc_ctx* c, rtcc_frame_info* info) {
   return RTCC_OK;
 }
 
-rtcc_status rtcc_get_layer_times(rtcc_ctx* c, int32_t agent, float* host_ms, int32_t cap,
-                                 int32_t* n_out) {
+rtcc_status rtcc_get_layer_spans(rtcc_ctx* c, int32_t agent, float* start_ms, float* end_ms,
+                                 int32_t cap, int32_t* n_out) {
   if (!c) return RTCC_E_ARG;
   std::lock_guard<std::mutex> lk(c->mu);
   if (agent < 0 || agent >= c->K) return RTCC_E_AGENT;
@@ -1015,12 +1015,30 @@ rtcc_status rtcc_get_layer_times(rtcc_ctx* c, int32_t agent, float* host_ms, int
   if (!b.stamps) return RTCC_E_STATE;
   const int n = (int)b.layers.size();
   if (n_out) *n_out = n;
-  if (!host_ms) return RTCC_OK;
+  if (!start_ms && !end_ms) return RTCC_OK;
   CK(cudaStreamSynchronize(b.st));
-  std::vector<unsigned long long> t(n + 1);
-  CK(cudaMemcpy(t.data(), b.stamps, (n + 1) * sizeof(unsigned long long), cudaMemcpyDeviceToHost));
-  for (int i = 0; i < n && i < cap; ++i)
-    host_ms[i] = (t[i + 1] >= t[i] && t[i] > 0) ? (float)((t[i + 1] - t[i]) * 1e-6) : -1.f;
+  std::vector<unsigned long long> t(2 * n);
+  CK(cudaMemcpy(t.data(), b.stamps, 2 * n * sizeof(unsigned long long), cudaMemcpyDeviceToHost));
+  unsigned long long t0 = 0;
+  for (int i = 0; i < 2 * n; ++i)
+    if (t[i] > 0 && (t0 == 0 || t[i] < t0)) t0 = t[i];
+  for (int i = 0; i < n && i < cap; ++i) {
+    const bool ok = t0 > 0 && t[i] > 0 && t[n + i] >= t[i];
+    if (start_ms) start_ms[i] = ok ? (float)((t[i] - t0) * 1e-6) : -1.f;
+    if (end_ms) end_ms[i] = ok ? (float)((t[n + i] - t0) * 1e-6) : -1.f;
+  }
+  return RTCC_OK;
+}
+
+rtcc_status rtcc_get_layer_times(rtcc_ctx* c, int32_t agent, float* host_ms, int32_t cap,
+                                 int32_t* n_out) {
+  if (!host_ms || cap <= 0) return rtcc_get_layer_spans(c, agent, nullptr, nullptr, 0, n_out);
+  std::vector<float> a(cap), e(cap);
+  int32_t n = 0;
+  const rtcc_status r = rtcc_get_layer_spans(c, agent, a.data(), e.data(), cap, &n);
+  if (r != RTCC_OK) return r;
+  if (n_out) *n_out = n;
+  for (int i = 0; i < n && i < cap; ++i) host_ms[i] = (a[i] >= 0.f && e[i] >= 0.f) ? e[i] - a[i] : -1.f;
   return RTCC_OK;
 }
 

@@ -35,6 +35,7 @@
 // a tile sums them in slice order, so results do not depend on timing.  Every
 // wait is bounded; one that runs out sets a bit in the error word and the CTA
 // winds down instead of hanging.
+#include <algorithm>
 #include <cstring>
 #include <mutex>
 #include <type_traits>
@@ -111,6 +112,8 @@ struct LayerScalars {
   int n_items, total_kb;
   int ncb_log2;            // log2(cin / bk): k-block kb = (tap << ncb_log2) + channel block
   int dsm;                 // split-K slices reduced through distributed shared memory
+  int cta_lo, cta_hi;      // CTAs the items are dealt to
+  int wait_items;          // target of the awaited layer's counter
 };
 __device__ __forceinline__ LayerScalars layer_scalars(const LayerDesc& D) {
   LayerScalars S;
@@ -130,10 +133,21 @@ __device__ __forceinline__ LayerScalars layer_scalars(const LayerDesc& D) {
   S.choff = D.choff;
   S.wait_layers = D.wait_layers;
   S.dsm = D.dsm;
+  S.cta_lo = D.cta_lo;
+  S.cta_hi = D.cta_hi;
+  S.wait_items = D.wait_items;
   S.n_items = S.m_tiles * S.n_tiles * S.splits;
   S.ncb_log2 = __ffs(S.cin / S.bk) - 1;            // cin / bk is a power of two
   S.total_kb = (S.kind == DECONV ? 1 : 9) << S.ncb_log2;
   return S;
+}
+
+// This CTA's first item of a layer (-1: none); its later items follow every
+// cta_hi - cta_lo items.
+__device__ __forceinline__ int first_item(const LayerScalars& S) {
+  const int b = (int)blockIdx.x;
+  if (b < S.cta_lo || b >= S.cta_hi) return -1;
+  return b - S.cta_lo < S.n_items ? b - S.cta_lo : -1;
 }
 
 // Work item t of a layer -> (tile = (m tile, n tile), K slice z), its tile
@@ -215,7 +229,6 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const unsigned G = gridDim.x;
   // The DSMEM reduction needs the launch to be in clusters of kMaxSplits CTAs;
   // the cluster size is read from the hardware, not trusted from the
   // parameters, and without such clusters split layers reduce through global
@@ -254,7 +267,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
     if (lane == 0) {
       // ---------------- TMA producer ----------------
       uint32_t it = 0;
-      bool alive = true;
+      bool alive = true, waited_pdl = false;
       for (int l = 0; l < P.n_layers && alive; ++l) {
         const LayerDesc& D = P.L[l];
         const LayerScalars S = layer_scalars(D);
@@ -266,10 +279,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
         // The weights do not depend on the previous layer: load the B boxes
         // of the first k-blocks of this CTA's first item before waiting for
         // the layer's input, so only the A boxes remain after the wait.
+        const int t0 = first_item(S), tstep = S.cta_hi - S.cta_lo;
+        if (t0 < 0) continue;                  // no items here: no wait, no count
         int npre = 0;
         Item I0{};
-        if ((int)blockIdx.x < S.n_items) {
-          I0 = item_of(S, blockIdx.x);
+        {
+          I0 = item_of(S, t0);
           npre = I0.kb1 - I0.kb0;
           if (npre > kStages) npre = kStages;
           for (int j = 0; j < npre; ++j) {
@@ -285,24 +300,26 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
           }
           if (!alive) break;
         }
-        if (l == 0) pdl_wait();
+        if (!waited_pdl) {                     // the pseudo-image is the previous kernel's output
+          pdl_wait();
+          waited_pdl = true;
+        }
         if (S.wait_layers > 0) {
-          // every CTA has finished layer wait_layers - 1 (and, as each CTA
-          // runs its layers in order, every layer before it)
-          if (!grid_wait(&P.grid_bar[S.wait_layers - 1], G)) {
+          // every item of the layer this one reads has been stored
+          if (!grid_wait(&P.grid_bar[S.wait_layers - 1], (unsigned)S.wait_items)) {
             atomicOr(P.err, ERR_WAIT_PRODUCER);
             alive = false;
             break;
           }
           fence_async_global();
         }
-        if (P.stamps && blockIdx.x == 0) P.stamps[l] = global_ns();
-        for (int t = blockIdx.x; t < S.n_items && alive; t += G) {
-          const Item I = (t == (int)blockIdx.x) ? I0 : item_of(S, t);
+        if (P.stamps && t0 == 0) P.stamps[l] = global_ns();
+        for (int t = t0; t < S.n_items && alive; t += tstep) {
+          const Item I = (t == t0) ? I0 : item_of(S, t);
           for (int kb = I.kb0; kb < I.kb1; ++kb, ++it) {
             const int s = it % kStages;
             uint8_t* dA = smem + s * kStageBytes;
-            if (t == (int)blockIdx.x && kb - I.kb0 < npre) {
+            if (t == t0 && kb - I.kb0 < npre) {
               load_a(S, mapA, dA, &full[s], I, kb);    // B already in flight
               continue;
             }
@@ -330,7 +347,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
         const bool bk64 = S.bk == 64;
         const uint32_t swz = bk64 ? 2u : 4u;          // 128B : 64B swizzle
         const uint32_t sbo = 8u * S.bk * 2u;          // bytes between 8-row atoms
-        for (int t = blockIdx.x; t < S.n_items && alive; t += G, ++tc) {
+        const int t0 = first_item(S), tstep = S.cta_hi - S.cta_lo;
+        for (int t = t0; t >= 0 && t < S.n_items && alive; t += tstep, ++tc) {
           const Item I = item_of(S, t);
           const int acc = tc & 1;
           if (!mbar_wait(&accempty[acc], ((tc >> 1) & 1) ^ 1)) {
@@ -373,7 +391,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
       const CUtensorMap* mapC = &D.mapC;
       const CUtensorMap* mapC16 = &D.mapC16;
       const int sg = S.bn < 64 ? S.bn : 64;    // channels per staged store box
-      for (int t = blockIdx.x; t < S.n_items; t += G, ++tc) {
+      const int t0 = first_item(S), tstep = S.cta_hi - S.cta_lo;
+      if (t0 < 0) continue;                    // no items here: no count
+      int mine = 0;
+      for (int t = t0; t < S.n_items; t += tstep, ++tc, ++mine) {
         const Item I = item_of(S, t);
         const int acc = tc & 1;
         // bias of this tile, read while the MMAs run (the slot was last read
@@ -582,16 +603,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
           }
         }
       }
-      // this CTA's part of layer l is written: count it in the grid barrier
+      // this CTA's items of layer l are stored: count them
       if (row == 0) {
         bulk_wait_all();
         fence_async_global();
         __threadfence();
-        atomicAdd(&P.grid_bar[l], 1u);
+        const unsigned before = atomicAdd(&P.grid_bar[l], (unsigned)mine);
+        // the CTA completing the layer's count stamps its end
+        if (P.stamps && before + (unsigned)mine == (unsigned)S.n_items)
+          P.stamps[P.n_layers + l] = global_ns();
       }
-    }
-    if (row == 0 && P.stamps && blockIdx.x == 0) {
-      if (grid_wait(&P.grid_bar[P.n_layers - 1], G)) P.stamps[P.n_layers] = global_ns();
     }
   }
 
@@ -774,6 +795,33 @@ cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, unsigned* grid_b
   }
   P->cluster = any_dsm ? kMaxSplits : 1;
   P->grid = any_dsm ? grid_cl : grid_sm;
+  // Item ranges.  Every layer's items are dealt round-robin over all CTAs,
+  // except the deconvs of the shallower blocks (those that do not read the
+  // deepest block): when the conv layers leave at least 8 CTAs without items,
+  // those CTAs take the early deconvs, which then run alongside the deeper
+  // conv blocks instead of after them.  A layer waits for the items of the
+  // one layer it reads.
+  int main_max = 0, last_conv = -1;
+  for (int i = 0; i < P->n_layers; ++i) {
+    const LayerDesc& D = P->L[i];
+    if (D.kind != DECONV) {
+      main_max = std::max(main_max, D.m_tiles * D.n_tiles * D.splits);
+      last_conv = i;
+    }
+  }
+  const bool background = P->grid - main_max >= 8;
+  for (int i = 0; i < P->n_layers; ++i) {
+    LayerDesc& D = P->L[i];
+    D.cta_lo = 0;
+    D.cta_hi = P->grid;
+    if (background && D.kind == DECONV && D.wait_layers - 1 != last_conv) D.cta_lo = main_max;
+    if (D.wait_layers > P->n_layers || D.wait_layers > (int)i) return cudaErrorInvalidValue;
+    D.wait_items = 0;
+    if (D.wait_layers > 0) {
+      const LayerDesc& W = P->L[D.wait_layers - 1];
+      D.wait_items = W.m_tiles * W.n_tiles * W.splits;
+    }
+  }
   return cudaSuccess;
 }
 

@@ -132,13 +132,16 @@ struct alignas(128) LayerDesc {   // CUtensorMap is 128-byte aligned
   int tiles_x, m_tiles, n_tiles, choff;
   int wait_layers;
   int dsm;                       // split-K slices reduced through distributed shared memory
+  int cta_lo, cta_hi;            // the CTAs this layer's items are dealt to (round-robin)
+  int wait_items;                // items of layer wait_layers - 1 (its counter's target)
 };
 struct BackboneParams {
   LayerDesc L[kMaxLayers];
   int n_layers;
-  unsigned* grid_bar;            // [kMaxLayers] per-layer arrival counters, zero before each launch
+  unsigned* grid_bar;            // [kMaxLayers] per-layer counts of finished items, zero before each launch
   int* err;
-  unsigned long long* stamps;    // optional [n_layers + 1] layer-start times (ns)
+  unsigned long long* stamps;    // optional [2 * n_layers] global-timer ns: layer starts
+                                 // (first item's wait passed), then layer ends (last item counted)
   int cluster;                   // 1, or kMaxSplits when some layer reduces through DSMEM
   int grid;                      // CTAs of the launch
 };

@@ -107,6 +107,8 @@ def load(path: Optional[str] = None) -> C.CDLL:
                                       C.POINTER(C.c_double)]),
         "rtcc_get_layer_times": (S, [_ctx_p, C.c_int32, C.c_void_p, C.c_int32,
                                      C.POINTER(C.c_int32)]),
+        "rtcc_get_layer_spans": (S, [_ctx_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_int32,
+                                     C.POINTER(C.c_int32)]),
         "rtcc_get_head": (S, [_ctx_p, C.c_void_p, C.c_size_t]),
         "rtcc_get_pillars": (S, [_ctx_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p,
                                  C.c_void_p]),
@@ -257,7 +259,8 @@ def rtcc_get_frame_info(ctx) -> rtcc_frame_info:
 
 
 def rtcc_get_layer_times(ctx, agent: int) -> np.ndarray:
-    """Per-layer ms of the agent's conv/deconv launches in the last frame."""
+    """Per-layer ms (first input-ready to last item counted) of the agent's
+    conv/deconv layers in the last frame."""
     lib = load()
     n = C.c_int32(0)
     _chk(lib.rtcc_get_layer_times(ctx, agent, None, 0, C.byref(n)), "rtcc_get_layer_times")
@@ -265,6 +268,19 @@ def rtcc_get_layer_times(ctx, agent: int) -> np.ndarray:
     _chk(lib.rtcc_get_layer_times(ctx, agent, _ptr(out), out.size, C.byref(n)),
          "rtcc_get_layer_times")
     return out
+
+
+def rtcc_get_layer_spans(ctx, agent: int):
+    """(start_ms, end_ms) of each conv/deconv layer of the agent's backbone in
+    the last frame, from the earliest layer start."""
+    lib = load()
+    n = C.c_int32(0)
+    _chk(lib.rtcc_get_layer_spans(ctx, agent, None, None, 0, C.byref(n)), "rtcc_get_layer_spans")
+    a = np.empty(n.value, dtype=np.float32)
+    e = np.empty(n.value, dtype=np.float32)
+    _chk(lib.rtcc_get_layer_spans(ctx, agent, _ptr(a), _ptr(e), a.size, C.byref(n)),
+         "rtcc_get_layer_spans")
+    return a, e
 
 
 def rtcc_get_branch_state(ctx, agent: int):

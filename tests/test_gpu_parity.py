@@ -277,3 +277,41 @@ def test_pointpillars_full_size(R):
     cfg = synth.get_config("pp3")
     ctx, *_ = _end_to_end(R, cfg, frame=1)
     R.rtcc_destroy(ctx)
+
+
+def test_layer_spans_follow_dependencies(R):
+    # With layer stamps on, the backbone records when each layer's first item
+    # passed its wait and when its last item was counted.  Every conv reads
+    # the conv before it and the neck deconv of block b reads that block's
+    # last conv, so no layer may start before the layers it reads have ended
+    # (up to the global timer's resolution).  The stamps must not change the
+    # results.
+    cfg = synth.get_config("pp3")
+    pts = [synth.points_for(cfg, 2, k) for k in range(cfg.n_agents)]
+    heads, spans = [], None
+    for flags in (U.DEBUG_FLAGS, U.DEBUG_FLAGS | R.FLAG_LAYER_TIMES):
+        ctx, _ = U.make_ctx(cfg, flags=flags)
+        try:
+            U.run_frame(ctx, cfg, pts, [0.0, 1.0, 2.0], R.MODE_RTCC)
+            heads.append(R.rtcc_get_head(ctx, cfg.feat_h, cfg.feat_w).copy())
+            if flags & R.FLAG_LAYER_TIMES:
+                spans = [R.rtcc_get_layer_spans(ctx, k) for k in range(cfg.n_agents)]
+                dur = R.rtcc_get_layer_times(ctx, 0)
+        finally:
+            R.rtcc_destroy(ctx)
+    assert heads[0].tobytes() == heads[1].tobytes()
+    last_of_block, n_conv = [], 0
+    for n, _, _ in cfg.blocks:
+        n_conv += n
+        last_of_block.append(n_conv - 1)
+    deps = [[l - 1] if 0 < l < n_conv else [] for l in range(n_conv)]
+    deps += [[last_of_block[b]] for b in range(len(cfg.up_strides))]
+    tol = 2e-3                                  # ms
+    for start, end in spans:
+        assert len(start) == len(deps)
+        assert np.all(start >= 0) and np.all(end >= start)
+        assert np.min(start) == 0.0
+        for l, dl in enumerate(deps):
+            for d in dl:
+                assert start[l] >= end[d] - tol, (l, d, start[l], end[d])
+    np.testing.assert_allclose(dur, spans[0][1] - spans[0][0], rtol=0, atol=1e-6)
