@@ -48,18 +48,26 @@ namespace rtcc {
 
 namespace {
 
-constexpr int TW = 32;                       // tile width in pixels
-constexpr int TH = 4;                        // tile height
+constexpr int TW = 8;                        // tile width in pixels: one 8-row MMA atom per image row
+constexpr int TH = 16;                       // tile height
 constexpr int BM = TW * TH;                  // 128 = MMA M
 constexpr int kThreads = 192;
 constexpr int kStages = 5;
 constexpr int kABytes = BM * 64 * 2;         // A slot (BK <= 64)
 constexpr int kBBytes = 128 * 64 * 2;        // B slot (BN <= 128, BK <= 64)
-constexpr int kStageBytes = kABytes + kBBytes;
+constexpr int kBOff = kStages * kABytes;     // the A slots, then the B slots
+// Halo tiles (3x3 stride-1 convs with 64-channel k-blocks): the (TW+2) x
+// (TH+2) input pixels of a tile for one 64-channel chunk, 128 bytes each in
+// the 128-byte swizzle; kHalo slots reuse the A area.
+constexpr int kHaloW = TW + 2, kHaloH = TH + 2;
+constexpr int kHaloBytes = kHaloW * kHaloH * 128;
+constexpr int kHaloSlot = 24 * 1024;
+constexpr int kHalo = 3;
+static_assert(kHaloBytes <= kHaloSlot && kHalo * kHaloSlot <= kBOff, "halo slots must fit the A area");
 constexpr int kStagingBytes = 64 * 1024;     // output tile (BN <= 128: 32 KB), or for a DSMEM
                                              // split the outgoing and receive slots (2 x 3 x
                                              // 128 x 16 fp32) + the 16-channel output tile
-constexpr int kSmem = kStages * kStageBytes + kStagingBytes + 1024 + 256;
+constexpr int kSmem = kStages * (kABytes + kBBytes) + kStagingBytes + 1024 + 256;
 constexpr uint32_t kTmemCols = 256;          // two 128-column accumulators
 
 // bias + ReLU of 16 fp32 columns [c0, c0+16) of tile row `row`, packed to
@@ -114,6 +122,11 @@ struct LayerScalars {
   int dsm;                 // split-K slices reduced through distributed shared memory
   int cta_lo, cta_hi;      // CTAs the items are dealt to
   int wait_items;          // target of the awaited layer's counter
+  int halo;                // A from halo tiles; k-blocks chunk-major (kb = 9 chunk + tap)
+  int kpb;                 // k-blocks per pipeline stage: halo layers put the weight boxes of
+                           // kBBytes / (bn * 128) taps into one stage, others 1 (A + B)
+  int spc;                 // halo layers: stages per 64-channel chunk (a stage never spans
+                           // two chunks)
 };
 __device__ __forceinline__ LayerScalars layer_scalars(const LayerDesc& D) {
   LayerScalars S;
@@ -136,6 +149,9 @@ __device__ __forceinline__ LayerScalars layer_scalars(const LayerDesc& D) {
   S.cta_lo = D.cta_lo;
   S.cta_hi = D.cta_hi;
   S.wait_items = D.wait_items;
+  S.halo = D.halo;
+  S.kpb = S.halo ? kBBytes / (S.bn * 128) : 1;
+  S.spc = (9 + S.kpb - 1) / S.kpb;
   S.n_items = S.m_tiles * S.n_tiles * S.splits;
   S.ncb_log2 = __ffs(S.cin / S.bk) - 1;            // cin / bk is a power of two
   S.total_kb = (S.kind == DECONV ? 1 : 9) << S.ncb_log2;
@@ -171,6 +187,23 @@ __device__ __forceinline__ Item item_of(const LayerScalars& S, int t) {
   return it;
 }
 
+// Pipeline stages of an item and the k-blocks [*k0, *k0 + *n) of its stage j.
+// Tap-box layers: one k-block per stage.  Halo layers: the item holds whole
+// 64-channel chunks, each split into spc stages of up to kpb taps.
+__device__ __forceinline__ int item_stages(const LayerScalars& S, const Item& I) {
+  return S.halo ? (I.kb1 - I.kb0) / 9 * S.spc : I.kb1 - I.kb0;
+}
+__device__ __forceinline__ void stage_kbs(const LayerScalars& S, const Item& I, int j, int* k0, int* n) {
+  if (!S.halo) {
+    *k0 = I.kb0 + j;
+    *n = 1;
+    return;
+  }
+  const int c = j / S.spc, q = j - c * S.spc;
+  *k0 = I.kb0 + 9 * c + q * S.kpb;
+  *n = min(S.kpb, 9 - q * S.kpb);
+}
+
 // TMA load of the activation (A) box of k-block kb of item I.
 __device__ __forceinline__ void load_a(const LayerScalars& S, const CUtensorMap* map, uint8_t* dA,
                                        uint64_t* bar, const Item& I, int kb) {
@@ -192,23 +225,68 @@ __device__ __forceinline__ void load_a(const LayerScalars& S, const CUtensorMap*
   }
 }
 
-// TMA load of the weight (B) box of k-block kb of item I.
+// TMA load of the weight (B) box of k-block kb of item I.  The packed
+// weights are [Cout][tap][Cin]: K index = tap * cin + cb * bk, which is kb * bk
+// for tap-major k-blocks.
 __device__ __forceinline__ void load_b(const LayerScalars& S, const CUtensorMap* map, uint8_t* dB,
                                        uint64_t* bar, const Item& I, int kb) {
-  // K index of k-block kb = tap * cin + cb * bk = kb * bk
-  tma_load_2d(dB, map, bar, kb * S.bk, I.n0);
+  int k = kb * S.bk;
+  if (S.halo) {
+    const int cb = kb / 9, tap = kb - 9 * cb;
+    k = tap * S.cin + cb * 64;
+  }
+  tma_load_2d(dB, map, bar, k, I.n0);
 }
 
-// One k-block of MMAs (BK = 64 or 32 -> 4 or 2 MMAs of K = 16) from
-// precomputed descriptors; advancing K by 16 elements = 32 bytes = +2 in the
-// descriptors' 16-byte address field (the start stays inside the stage).
-__device__ __forceinline__ void mma_kblock(uint32_t d_tmem, uint64_t ad, uint64_t bd, uint32_t idesc,
-                                           uint32_t acc0, bool bk64) {
-  umma_f16(d_tmem, ad, bd, idesc, acc0);
-  umma_f16(d_tmem, ad + 2, bd + 2, idesc, 1u);
+// TMA load of the halo tile of 64-channel chunk cb of item I: input pixels
+// [x0 - 1, x0 + TW] x [y0 - 1, y0 + TH]; out-of-image pixels read as zero,
+// which is the zero padding.  Tap (dy, dx) of the tile is then the A operand
+// starting (dy * kHaloW + dx) rows into it, with kHaloW rows between the
+// 8-row atoms: the hardware applies the 128-byte swizzle to the final shared
+// memory address, so a start at any 128-byte row matches the TMA placement.
+__device__ __forceinline__ void load_halo(const CUtensorMap* map, uint8_t* dH, uint64_t* bar,
+                                          const Item& I, int cb) {
+  tma_load_4d(dH, map, bar, cb * 64, I.x0 - 1, I.y0 - 1, 0);
+}
+
+// One k-block of MMAs (BK = 64 or 32 -> 4 or 2 MMAs of K = 16).  The
+// issuing thread cannot issue an MMA before the tensor pipe takes the
+// previous one, so every instruction between them adds to the k-block's time;
+// one asm statement keeps that to one add per operand.  The descriptors come
+// as 32-bit halves: advancing K by 16 elements = 32 bytes is +2 in the
+// 16-byte address field of the low half (the start stays inside its stage,
+// so the field does not overflow), and the high half (stride, swizzle) is the
+// same for every MMA of an operand.
+__device__ __forceinline__ void mma_kblock(uint32_t d_tmem, uint32_t a_lo, uint32_t a_hi, uint32_t b_lo,
+                                           uint32_t b_hi, uint32_t idesc, uint32_t acc0, bool bk64) {
   if (bk64) {
-    umma_f16(d_tmem, ad + 4, bd + 4, idesc, 1u);
-    umma_f16(d_tmem, ad + 6, bd + 6, idesc, 1u);
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\t.reg .b64 a, b;\n\t.reg .b32 al, bl;\n\t"
+        "setp.ne.b32 p, %5, 0;\n\t"
+        "setp.eq.b32 q, %5, %5;\n\t"
+        "mov.b64 a, {%1, %2};\n\tmov.b64 b, {%3, %4};\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %6, p;\n\t"
+        "add.u32 al, %1, 2;\n\tadd.u32 bl, %3, 2;\n\t"
+        "mov.b64 a, {al, %2};\n\tmov.b64 b, {bl, %4};\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %6, q;\n\t"
+        "add.u32 al, %1, 4;\n\tadd.u32 bl, %3, 4;\n\t"
+        "mov.b64 a, {al, %2};\n\tmov.b64 b, {bl, %4};\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %6, q;\n\t"
+        "add.u32 al, %1, 6;\n\tadd.u32 bl, %3, 6;\n\t"
+        "mov.b64 a, {al, %2};\n\tmov.b64 b, {bl, %4};\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %6, q;\n\t}" ::"r"(d_tmem),
+        "r"(a_lo), "r"(a_hi), "r"(b_lo), "r"(b_hi), "r"(acc0), "r"(idesc));
+  } else {
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\t.reg .b64 a, b;\n\t.reg .b32 al, bl;\n\t"
+        "setp.ne.b32 p, %5, 0;\n\t"
+        "setp.eq.b32 q, %5, %5;\n\t"
+        "mov.b64 a, {%1, %2};\n\tmov.b64 b, {%3, %4};\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %6, p;\n\t"
+        "add.u32 al, %1, 2;\n\tadd.u32 bl, %3, 2;\n\t"
+        "mov.b64 a, {al, %2};\n\tmov.b64 b, {bl, %4};\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], a, b, %6, q;\n\t}" ::"r"(d_tmem),
+        "r"(a_lo), "r"(a_hi), "r"(b_lo), "r"(b_hi), "r"(acc0), "r"(idesc));
   }
 }
 
@@ -217,13 +295,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint8_t* stage = smem + kStages * kStageBytes;
+  uint8_t* stage = smem + kStages * (kABytes + kBBytes);
   uint64_t* full = reinterpret_cast<uint64_t*>(stage + kStagingBytes);
   uint64_t* empty = full + kStages;
   uint64_t* accfull = empty + kStages;         // [2]
   uint64_t* accempty = accfull + 2;            // [2]
   uint64_t* recvbar = accempty + 2;            // partials received through DSMEM
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(recvbar + 1);
+  uint64_t* hfull = recvbar + 1;               // [kHalo] halo tiles
+  uint64_t* hempty = hfull + kHalo;            // [kHalo]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(hempty + kHalo);
   __shared__ int s_last;
   __shared__ float s_bias[2][128];             // bias of the tile in each accumulator
 
@@ -246,6 +326,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
       mbar_init(&accempty[a], 4);              // one arrival per epilogue warp
     }
     mbar_init(recvbar, 1);                     // the owner's arrival + the peers' bytes
+    for (int h = 0; h < kHalo; ++h) {
+      mbar_init(&hfull[h], 1);
+      mbar_init(&hempty[h], 1);
+    }
     fence_barrier_init();
     if (ncl > 1) fence_mbar_init_cluster();
   }
@@ -265,8 +349,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
 
   if (warp == 0) {
     if (lane == 0) {
-      // ---------------- TMA producer ----------------
-      uint32_t it = 0;
+      // ---------------- TMA producer (one thread) ----------------
+      uint32_t it = 0, hc = 0;                   // stages (B ring) and halo tiles issued
+      int a_mode = 0;                            // last user of the A area: 1 tap boxes, 2 halo tiles
       bool alive = true, waited_pdl = false;
       for (int l = 0; l < P.n_layers && alive; ++l) {
         const LayerDesc& D = P.L[l];
@@ -275,17 +360,21 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
         const CUtensorMap* mapB = &D.mapB;
         tma_prefetch_desc(mapA);
         tma_prefetch_desc(mapB);
-        const uint32_t bytes = (uint32_t)(BM + S.bn) * S.bk * 2;
+        // bytes landing on a stage's barrier: the tap box and the weight box,
+        // or for a layer that reads halo tiles (they have their own barriers)
+        // the weight boxes of the stage's kpb k-blocks
+        const uint32_t bbox = (uint32_t)S.bn * S.bk * 2;
+        const uint32_t bytes = S.halo ? bbox * S.kpb : (uint32_t)(BM * S.bk * 2) + bbox;
         // The weights do not depend on the previous layer: load the B boxes
         // of the first k-blocks of this CTA's first item before waiting for
         // the layer's input, so only the A boxes remain after the wait.
         const int t0 = first_item(S), tstep = S.cta_hi - S.cta_lo;
-        if (t0 < 0) continue;                  // no items here: no wait, no count
+        if (t0 < 0) continue;                    // no items here: no wait, no count
         int npre = 0;
         Item I0{};
         {
           I0 = item_of(S, t0);
-          npre = I0.kb1 - I0.kb0;
+          npre = item_stages(S, I0);
           if (npre > kStages) npre = kStages;
           for (int j = 0; j < npre; ++j) {
             const uint32_t u = it + j;
@@ -295,12 +384,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
               alive = false;
               break;
             }
-            mbar_arrive_expect_tx(&full[s], bytes);
-            load_b(S, mapB, smem + s * kStageBytes + kABytes, &full[s], I0, I0.kb0 + j);
+            int k0, n;
+            stage_kbs(S, I0, j, &k0, &n);
+            mbar_arrive_expect_tx(&full[s], S.halo ? bbox * n : bytes);
+            for (int i = 0; i < n; ++i)
+              load_b(S, mapB, smem + kBOff + s * kBBytes + i * bbox, &full[s], I0, k0 + i);
           }
           if (!alive) break;
         }
-        if (!waited_pdl) {                     // the pseudo-image is the previous kernel's output
+        if (!waited_pdl) {                       // the pseudo-image is the previous kernel's output
           pdl_wait();
           waited_pdl = true;
         }
@@ -313,40 +405,100 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
           }
           fence_async_global();
         }
+        // Tap boxes and halo tiles share the A area: before it changes use,
+        // the MMAs that read it must be done.  The issuer commits every stage
+        // after its MMAs, halo tiles included, so the release of the last stage
+        // issued implies the rest (a wait costs about a hundred clocks even
+        // when the phase has long completed, so one wait, not one per slot).
+        const int mode = S.halo ? 2 : 1;
+        if (a_mode != 0 && a_mode != mode && it > 0) {
+          if (!mbar_wait(&empty[(it - 1) % kStages], ((it - 1) / kStages) & 1)) {
+            atomicOr(P.err, ERR_WAIT_PRODUCER);
+            break;
+          }
+        }
+        a_mode = mode;
         if (P.stamps && t0 == 0) P.stamps[l] = global_ns();
-        for (int t = t0; t < S.n_items && alive; t += tstep) {
-          const Item I = (t == t0) ? I0 : item_of(S, t);
-          for (int kb = I.kb0; kb < I.kb1; ++kb, ++it) {
-            const int s = it % kStages;
-            uint8_t* dA = smem + s * kStageBytes;
-            if (t == t0 && kb - I.kb0 < npre) {
-              load_a(S, mapA, dA, &full[s], I, kb);    // B already in flight
-              continue;
+        if (S.halo) {
+          for (int t = t0; t < S.n_items && alive; t += tstep) {
+            const Item I = (t == t0) ? I0 : item_of(S, t);
+            // The item's chunks: the first kHalo halo tiles go out at once;
+            // from then on, reaching chunk c issues chunk c + 1's halo tile
+            // into the slot of chunk c + 1 - kHalo (released when its MMAs are
+            // done), a chunk of MMAs ahead of its use.
+            const int c0 = I.kb0 / 9, nch = (I.kb1 - I.kb0) / 9;
+            int issued = 0;
+            for (int c = 0; c < nch && alive; ++c) {
+              while (issued < nch && (issued < kHalo ? c == 0 : issued == c + kHalo - 2)) {
+                const int h = hc % kHalo;
+                if (!mbar_wait(&hempty[h], ((hc / kHalo) & 1) ^ 1)) {
+                  atomicOr(P.err, ERR_WAIT_PRODUCER);
+                  alive = false;
+                  break;
+                }
+                mbar_arrive_expect_tx(&hfull[h], (uint32_t)kHaloBytes);
+                load_halo(mapA, smem + h * kHaloSlot, &hfull[h], I, c0 + issued);
+                ++hc;
+                ++issued;
+              }
+              for (int q = 0; q < S.spc && alive; ++q, ++it) {
+                const int j = c * S.spc + q;
+                if (t == t0 && j < npre) continue;               // weights already in flight
+                int k0, n;
+                stage_kbs(S, I, j, &k0, &n);
+                const int s = it % kStages;
+                if (!mbar_wait(&empty[s], ((it / kStages) & 1) ^ 1)) {
+                  atomicOr(P.err, ERR_WAIT_PRODUCER);
+                  alive = false;
+                  break;
+                }
+                mbar_arrive_expect_tx(&full[s], bbox * n);
+                for (int i = 0; i < n; ++i)
+                  load_b(S, mapB, smem + kBOff + s * kBBytes + i * bbox, &full[s], I, k0 + i);
+              }
             }
-            if (!mbar_wait(&empty[s], ((it / kStages) & 1) ^ 1)) {
-              atomicOr(P.err, ERR_WAIT_PRODUCER);
-              alive = false;
-              break;
+          }
+        } else {
+          for (int t = t0; t < S.n_items && alive; t += tstep) {
+            const Item I = (t == t0) ? I0 : item_of(S, t);
+            for (int kb = I.kb0; kb < I.kb1; ++kb, ++it) {
+              const int s = it % kStages;
+              uint8_t* dA = smem + s * kABytes;
+              if (t == t0 && kb - I.kb0 < npre) {
+                load_a(S, mapA, dA, &full[s], I, kb);         // B already in flight
+                continue;
+              }
+              if (!mbar_wait(&empty[s], ((it / kStages) & 1) ^ 1)) {
+                atomicOr(P.err, ERR_WAIT_PRODUCER);
+                alive = false;
+                break;
+              }
+              mbar_arrive_expect_tx(&full[s], bytes);
+              load_a(S, mapA, dA, &full[s], I, kb);
+              load_b(S, mapB, smem + kBOff + s * kBBytes, &full[s], I, kb);
             }
-            mbar_arrive_expect_tx(&full[s], bytes);
-            load_a(S, mapA, dA, &full[s], I, kb);
-            load_b(S, mapB, dA + kABytes, &full[s], I, kb);
           }
         }
       }
     }
   } else if (warp == 1) {
     if (lane == 0) {
-      // ---------------- MMA issuer ----------------
-      uint32_t it = 0, tc = 0;
+      // ---------------- MMA issuer (one thread) ----------------
+      uint32_t it = 0, tc = 0, hc = 0;
       bool alive = true;
       const uint32_t smem0 = smem_u32(smem);
       for (int l = 0; l < P.n_layers && alive; ++l) {
         const LayerScalars S = layer_scalars(P.L[l]);
         const uint32_t idesc = idesc_f16(BM, S.bn, std::is_same<T, __nv_bfloat16>::value);
         const bool bk64 = S.bk == 64;
-        const uint32_t swz = bk64 ? 2u : 4u;          // 128B : 64B swizzle
-        const uint32_t sbo = 8u * S.bk * 2u;          // bytes between 8-row atoms
+        const uint32_t swz = bk64 ? 2u : 4u;            // 128B : 64B swizzle
+        const uint32_t sbo = 8u * S.bk * 2u;            // bytes between 8-row atoms
+        // descriptor halves of the first A and B slots (the slots of a stage
+        // s are kABytes / kBBytes further on) and of the halo slots
+        const uint64_t ad0 = smem_desc(smem0, sbo, swz), bd0 = smem_desc(smem0 + kBOff, sbo, swz);
+        const uint32_t a_lo0 = (uint32_t)ad0, a_hi = (uint32_t)(ad0 >> 32);
+        const uint32_t b_lo0 = (uint32_t)bd0, b_hi = (uint32_t)(bd0 >> 32);
+        const uint32_t a_hi_halo = (uint32_t)(smem_desc(smem0, kHaloW * 128, 2u) >> 32);
         const int t0 = first_item(S), tstep = S.cta_hi - S.cta_lo;
         for (int t = t0; t >= 0 && t < S.n_items && alive; t += tstep, ++tc) {
           const Item I = item_of(S, t);
@@ -358,18 +510,60 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
           }
           tc_fence_after();
           const uint32_t d_tmem = tmem + acc * 128;
-          for (int kb = I.kb0; kb < I.kb1; ++kb, ++it) {
-            const int s = it % kStages;
-            if (!mbar_wait(&full[s], (it / kStages) & 1)) {
-              atomicOr(P.err, ERR_WAIT_MMA);
-              alive = false;
-              break;
+          if (S.halo) {
+            // Chunk by chunk: wait for the halo tile, then the 9 taps fully
+            // unrolled, so every descriptor offset is an immediate and the
+            // MMAs issue back to back; a stage of kpb taps starts with a wait
+            // on its weight boxes and ends with a commit that frees it.
+            const int nch = (I.kb1 - I.kb0) / 9;
+            const int km = S.kpb - 1;
+            const uint32_t bstep = (uint32_t)(S.bn * 8);        // one weight box, 16-byte units
+            for (int c = 0; c < nch && alive; ++c) {
+              const int h = hc % kHalo;
+              if (!mbar_wait(&hfull[h], (hc / kHalo) & 1)) {
+                atomicOr(P.err, ERR_WAIT_MMA);
+                alive = false;
+                break;
+              }
+              ++hc;
+              const uint32_t a_lo = (uint32_t)smem_desc(smem0 + h * kHaloSlot, kHaloW * 128, 2u);
+              uint32_t b_lo = 0;
+              int s = 0;
+#pragma unroll
+              for (int tap = 0; tap < 9; ++tap) {
+                if ((tap & km) == 0) {
+                  s = it % kStages;
+                  if (!mbar_wait(&full[s], (it / kStages) & 1)) {
+                    atomicOr(P.err, ERR_WAIT_MMA);
+                    alive = false;
+                    break;
+                  }
+                  tc_fence_after();
+                  b_lo = b_lo0 + (uint32_t)(s * (kBBytes >> 4));
+                }
+                mma_kblock(d_tmem, a_lo + (uint32_t)(((tap / 3) * kHaloW + tap % 3) * 8), a_hi_halo,
+                           b_lo + (uint32_t)(tap & km) * bstep, b_hi, idesc, (c > 0 || tap > 0) ? 1u : 0u,
+                           true);
+                if (((tap + 1) & km) == 0 || tap == 8) {
+                  umma_commit(&empty[s]);
+                  ++it;
+                }
+              }
+              umma_commit(&hempty[h]);
             }
-            tc_fence_after();
-            const uint32_t aa = smem0 + s * kStageBytes;
-            mma_kblock(d_tmem, smem_desc(aa, sbo, swz), smem_desc(aa + kABytes, sbo, swz), idesc,
-                       kb > I.kb0 ? 1u : 0u, bk64);
-            umma_commit(&empty[s]);
+          } else {
+            for (int kb = I.kb0; kb < I.kb1; ++kb, ++it) {
+              const int s = it % kStages;
+              if (!mbar_wait(&full[s], (it / kStages) & 1)) {
+                atomicOr(P.err, ERR_WAIT_MMA);
+                alive = false;
+                break;
+              }
+              tc_fence_after();
+              mma_kblock(d_tmem, a_lo0 + (uint32_t)(s * (kABytes >> 4)), a_hi,
+                         b_lo0 + (uint32_t)(s * (kBBytes >> 4)), b_hi, idesc, kb > I.kb0 ? 1u : 0u, bk64);
+              umma_commit(&empty[s]);
+            }
           }
           umma_commit(&accfull[acc]);
         }
@@ -694,7 +888,9 @@ cudaError_t conv_make_maps(ConvLayer& L, bool bf16) {
   } else {
     cuuint64_t dims[4] = {C, W, H, 1};
     cuuint64_t strides[3] = {C * 2, W * C * 2, H * W * C * 2};
-    cuuint32_t box[4] = {(cuuint32_t)L.bk, (cuuint32_t)TW, (cuuint32_t)TH, 1};
+    const bool halo = conv_uses_halo(L);
+    cuuint32_t box[4] = {(cuuint32_t)L.bk, (cuuint32_t)(halo ? kHaloW : TW),
+                         (cuuint32_t)(halo ? kHaloH : TH), 1};
     cuuint32_t es[4] = {1, 1, 1, 1};
     r = enc(&L.mapA, dt, 4, const_cast<void*>(L.in), dims, strides, box, es,
             CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
@@ -784,6 +980,7 @@ cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, unsigned* grid_b
     D.choff = L.choff;
     D.wait_layers = L.wait_layers;
     D.mapC16 = L.mapC16;
+    D.halo = conv_uses_halo(L) ? 1 : 0;
     // a split of a 64-wide tile into 2 or kMaxSplits slices, one item per
     // CTA, reduces its slices through distributed shared memory within a
     // cluster of kMaxSplits CTAs

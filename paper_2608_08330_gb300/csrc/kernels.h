@@ -115,6 +115,12 @@ struct ConvLayer {
 
 // Encode the layer's tensor maps (input activations, packed weights, output).
 cudaError_t conv_make_maps(ConvLayer& L, bool bf16);
+// Whether the layer reads its A operand as halo tiles (one box per tile and
+// 64-channel chunk, shared by the 9 taps) instead of one box per tap: 3x3
+// stride-1 convs with 64-channel k-blocks whose K slices hold whole chunks.
+inline bool conv_uses_halo(const ConvLayer& L) {
+  return L.kind == CONV3_S1 && L.bk == 64 && L.splits >= 1 && (L.cin / 64) % L.splits == 0;
+}
 int conv_tile_w();
 int conv_tile_h();
 int conv_tile_m();
@@ -134,6 +140,7 @@ struct alignas(128) LayerDesc {   // CUtensorMap is 128-byte aligned
   int dsm;                       // split-K slices reduced through distributed shared memory
   int cta_lo, cta_hi;            // the CTAs this layer's items are dealt to (round-robin)
   int wait_items;                // items of layer wait_layers - 1 (its counter's target)
+  int halo;                      // 3x3 stride-1 with 64-channel k-blocks: A from halo tiles
 };
 struct BackboneParams {
   LayerDesc L[kMaxLayers];
