@@ -29,10 +29,11 @@
 // Roles (192 threads): warp 0 = TMA producer, warp 1 = tensor-memory owner and
 // MMA issuer, warps 2..5 = epilogue.  Tensor memory holds two 128-column
 // accumulators, so the epilogue of one tile overlaps the MMAs of the next.
-// The epilogue adds bias, applies ReLU, rounds to 16 bits, stages the tile in
-// shared memory in the store map's swizzle and writes it with TMA tensor
-// stores.  Split-K slices publish fp32 partials and the last-arriving slice of
-// a tile sums them in slice order, so results do not depend on timing.  Every
+// The epilogue adds bias, applies ReLU, rounds to 16 bits and writes each
+// pixel's channels from registers (16-byte stores; a CTA's stores are then
+// published by one release-ordered count).  Split-K slices of a tile are
+// summed in slice order (through distributed shared memory, else global
+// memory), so results do not depend on timing.  Every
 // wait is bounded; one that runs out sets a bit in the error word and the CTA
 // winds down instead of hanging.
 #include <algorithm>
@@ -64,34 +65,60 @@ constexpr int kHaloBytes = kHaloW * kHaloH * 128;
 constexpr int kHaloSlot = 24 * 1024;
 constexpr int kHalo = 3;
 static_assert(kHaloBytes <= kHaloSlot && kHalo * kHaloSlot <= kBOff, "halo slots must fit the A area");
-constexpr int kStagingBytes = 64 * 1024;     // output tile (BN <= 128: 32 KB), or for a DSMEM
-                                             // split the outgoing and receive slots (2 x 3 x
-                                             // 128 x 16 fp32) + the 16-channel output tile
+constexpr int kStagingBytes = 64 * 1024;     // DSMEM split-K exchange: the outgoing slots
+                                             // (4 x 128 x 16 fp32) and the receive slots
+                                             // (3 x 128 x 16 fp32); deconvs: the output
+                                             // tile (128 x 128 channels, 16-bit)
 constexpr int kSmem = kStages * (kABytes + kBBytes) + kStagingBytes + 1024 + 256;
 constexpr uint32_t kTmemCols = 256;          // two 128-column accumulators
 
-// bias + ReLU of 16 fp32 columns [c0, c0+16) of tile row `row`, packed to
-// 16 bits and written to the staging tile.  Channels are staged in groups of
-// sg (64 or 32): group g is a [BM][sg] block with sg*2-byte rows in the
-// 128-byte (sg = 64) or 64-byte (sg = 32) swizzle of the store tensor map, so
-// a warp's 16-byte writes spread over all banks.
+// bias + ReLU of 16 fp32 values, packed to 16 bits and written as two
+// 16-byte stores to dst (16-byte aligned: the channel offset is a multiple of
+// 16 and the pixel stride a multiple of 8 channels); nothing for a pixel
+// outside the image (dst null).
 template <typename T>
-__device__ __forceinline__ void stage16(uint8_t* stage, int sg, int row, int c0, const float* v,
-                                        const float* bias) {
+__device__ __forceinline__ void store16(T* dst, const float* v, const float* bias) {
+  if (!dst) return;
   uint32_t pk[8];
 #pragma unroll
   for (int j = 0; j < 8; ++j)
     pk[j] = Store<T>::pack2(relu_f(v[2 * j] + bias[2 * j]), relu_f(v[2 * j + 1] + bias[2 * j + 1]));
-  const int rb = sg * 2;                               // bytes per staged row
-  uint8_t* base = stage + (c0 / sg) * (BM * rb) + row * rb;
-  const int j0 = (c0 % sg) / 8;                        // 16-byte chunk within the row
-  const int x = (sg == 64) ? (row & 7) : ((row >> 1) & 3);
+  uint4* o = reinterpret_cast<uint4*>(dst);
+  o[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+  o[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+}
+
+// bias + ReLU of 16 fp32 columns [c0, c0+16) of tile row `row`, packed to
+// 16 bits and written to the staging tile: a [BM][64]-channel block per 64
+// columns, 128-byte rows in the 128-byte swizzle of the deconv store map, so
+// a warp's 16-byte writes spread over all banks.
+template <typename T>
+__device__ __forceinline__ void stage16(uint8_t* stage, int row, int c0, const float* v, const float* bias) {
+  uint32_t pk[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j)
+    pk[j] = Store<T>::pack2(relu_f(v[2 * j] + bias[2 * j]), relu_f(v[2 * j + 1] + bias[2 * j + 1]));
+  uint8_t* base = stage + (c0 / 64) * (BM * 128) + row * 128;
+  const int j0 = (c0 % 64) / 8;                        // 16-byte chunk within the row
+  const int x = row & 7;
   *reinterpret_cast<uint4*>(base + ((j0 ^ x) << 4)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
   *reinterpret_cast<uint4*>(base + (((j0 + 1) ^ x) << 4)) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
 }
 
 // barrier among the 4 epilogue warps only (named barrier 1, 128 threads)
 __device__ __forceinline__ void epilogue_sync() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+
+// Release-ordered additions to a grid-wide counter: the writes this thread
+// made before are visible to any thread that reads the new value with acquire
+// semantics.  The reduction form does not wait for the old value.
+__device__ __forceinline__ void red_add_release_gpu(unsigned* ctr, unsigned v) {
+  asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(ctr), "r"(v) : "memory");
+}
+__device__ __forceinline__ unsigned atom_add_release_gpu(unsigned* ctr, unsigned v) {
+  unsigned old;
+  asm volatile("atom.release.gpu.global.add.u32 %0, [%1], %2;" : "=r"(old) : "l"(ctr), "r"(v) : "memory");
+  return old;
+}
 
 // Wait until the grid-wide arrival counter reaches `target` (bounded).
 __device__ __forceinline__ bool grid_wait(const unsigned* ctr, unsigned target) {
@@ -127,6 +154,8 @@ struct LayerScalars {
                            // kBBytes / (bn * 128) taps into one stage, others 1 (A + B)
   int spc;                 // halo layers: stages per 64-channel chunk (a stage never spans
                            // two chunks)
+  void* out;               // output [.][ow][ldc], 16-bit
+  int ow, ldc, gw, gh;     // output row length (pixels), pixel stride (channels), tile grid extent
 };
 __device__ __forceinline__ LayerScalars layer_scalars(const LayerDesc& D) {
   LayerScalars S;
@@ -150,6 +179,11 @@ __device__ __forceinline__ LayerScalars layer_scalars(const LayerDesc& D) {
   S.cta_hi = D.cta_hi;
   S.wait_items = D.wait_items;
   S.halo = D.halo;
+  S.out = D.out;
+  S.ow = D.ow;
+  S.ldc = D.ldc;
+  S.gw = D.gw;
+  S.gh = D.gh;
   S.kpb = S.halo ? kBBytes / (S.bn * 128) : 1;
   S.spc = (9 + S.kpb - 1) / S.kpb;
   S.n_items = S.m_tiles * S.n_tiles * S.splits;
@@ -582,9 +616,6 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
     for (int l = 0; l < P.n_layers; ++l) {
       const LayerDesc& D = P.L[l];
       const LayerScalars S = layer_scalars(D);
-      const CUtensorMap* mapC = &D.mapC;
-      const CUtensorMap* mapC16 = &D.mapC16;
-      const int sg = S.bn < 64 ? S.bn : 64;    // channels per staged store box
       const int t0 = first_item(S), tstep = S.cta_hi - S.cta_lo;
       if (t0 < 0) continue;                    // no items here: no count
       int mine = 0;
@@ -601,10 +632,32 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
         tc_fence_after();
         const float* bias = s_bias[acc];
         const uint32_t taddr = tmem + acc * 128 + (static_cast<uint32_t>(qd * 32) << 16);
-        // the previous tile's stores must have read the staging buffer
-        if (row == 0) bulk_wait_read_all();
+        // This row's output pixel (the tile's row-th pixel; for a deconv one
+        // sub-pixel position of its input pixel), written straight from
+        // registers: channels [n0, n0 + bn) of a conv, [choff, choff + cout)
+        // of a deconv.  Null outside the image (ragged tiles).
+        T* orow = nullptr;
+        {
+          const int px = I.x0 + row % TW, py = I.y0 + row / TW;
+          if (px < S.gw && py < S.gh) {
+            size_t pix;
+            int c0;
+            if (S.kind == DECONV) {
+              const int sub = I.n0 / S.cout;
+              const int sy = sub / S.s, sx = sub - sy * S.s;
+              pix = (size_t)(py * S.s + sy) * S.ow + (size_t)(px * S.s + sx);
+              c0 = S.choff;
+            } else {
+              pix = (size_t)py * S.ow + px;
+              c0 = S.choff + I.n0;
+            }
+            orow = static_cast<T*>(S.out) + pix * S.ldc + c0;
+          }
+        }
+        // the previous item's bulk copies (DSMEM exchange) or tile stores
+        // (deconv) must have read the shared memory they came from
+        if ((S.dsm || S.kind == DECONV) && row == 0) bulk_wait_read_all();
         epilogue_sync();
-        bool store = true;
         if (S.splits == 1) {
           // up to 64 columns per round: issue all TMEM loads, wait once
           for (int c0 = 0; c0 < S.bn; c0 += 64) {
@@ -621,7 +674,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
                 float v[16];
 #pragma unroll
                 for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[g][i]);
-                stage16<T>(stage, sg, row, c0 + 16 * g, v, bias + c0 + 16 * g);
+                if (S.kind == DECONV)
+                  stage16<T>(stage, row, c0 + 16 * g, v, bias + c0 + 16 * g);
+                else
+                  store16<T>(orow ? orow + c0 + 16 * g : nullptr, v, bias + c0 + 16 * g);
               }
             }
           }
@@ -644,7 +700,6 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
           const int SLOT = BM * CW * 4;                          // one owner's channels, fp32
           uint8_t* own = stage;                                  // [Sp][BM][CW] fp32, by owner (32 KB)
           uint8_t* recv = stage + Sp * SLOT;                     // [Sp-1][BM][CW] fp32, from peers
-          uint8_t* out16 = recv + (Sp - 1) * SLOT;               // [G16][BM][16] 16-bit
           if (row == 0) mbar_arrive_expect_tx(recvbar, (uint32_t)((Sp - 1) * SLOT));
           // the row's 64 columns in one round of TMEM loads, into the owner slots
           uint32_t rq[4][16];
@@ -693,24 +748,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
                 sum[4 * q + 3] += f.w;
               }
             }
-            // bias + ReLU, 16-bit, staged [BM][16] per group (32-byte rows)
-            const float* bz = bias + z * CW + h * 16;
-            uint32_t pk[8];
-#pragma unroll
-            for (int j = 0; j < 8; ++j)
-              pk[j] = Store<T>::pack2(relu_f(sum[2 * j] + bz[2 * j]), relu_f(sum[2 * j + 1] + bz[2 * j + 1]));
-            uint4* o = reinterpret_cast<uint4*>(out16 + h * BM * 32 + row * 32);
-            o[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-            o[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+            // bias + ReLU, 16-bit, the owner's 16 channels of this row
+            store16<T>(orow ? orow + z * CW + h * 16 : nullptr, sum, bias + z * CW + h * 16);
           }
-          fence_async_smem();
-          epilogue_sync();
-          if (row == 0) {
-            for (int h = 0; h < G16; ++h)
-              tma_store_3d(mapC16, out16 + h * BM * 32, I.n0 + z * CW + h * 16, I.x0, I.y0);
-            bulk_commit();
-          }
-          store = false;
         } else {
           // publish this slice's fp32 partial ([bn/4][BM][4] per (slice, tile),
           // so a warp's float4 stores cover 512 contiguous bytes), then the
@@ -733,8 +773,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
             s_last = (old == S.splits - 1);
           }
           epilogue_sync();
-          store = s_last != 0;
-          if (store) {
+          if (s_last != 0) {
             __threadfence();
             for (int c0 = 0; c0 < S.bn; c0 += 16) {
               // all other slices' loads of this column group in flight at once
@@ -771,7 +810,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
                   }
                 }
               }
-              stage16<T>(stage, sg, row, c0, sum, bias + c0);
+              store16<T>(orow ? orow + c0 : nullptr, sum, bias + c0);
             }
             if (row == 0) S.counters[tile_id] = 0;     // ready for the next launch
           }
@@ -779,33 +818,39 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
         // the accumulator has been read: hand it back to the MMA issuer
         tc_fence_before();
         if (lane == 0) mbar_arrive(&accempty[acc]);
-        if (store) {
+        if (S.kind == DECONV) {
+          // A deconv row is 128 channels at a strided sub-pixel position:
+          // one 5-D TMA box store per 64 channels beats 16 stores per thread.
           fence_async_smem();
           epilogue_sync();
           if (row == 0) {
-            const int GB = BM * sg * 2;                // bytes of one staged channel group
-            if (S.kind == DECONV) {
-              const int sub = I.n0 / S.cout;
-              const int sy = sub / S.s, sx = sub - sy * S.s;
-              for (int g = 0; g < S.bn / sg; ++g)
-                tma_store_5d(mapC, stage + g * GB, S.choff + g * sg, sx, I.x0, sy, I.y0);
-            } else {
-              for (int g = 0; g < S.bn / sg; ++g)
-                tma_store_3d(mapC, stage + g * GB, I.n0 + g * sg, I.x0, I.y0);
-            }
+            const int sub = I.n0 / S.cout;
+            const int sy = sub / S.s, sx = sub - sy * S.s;
+            for (int g = 0; g < S.bn / 64; ++g)
+              tma_store_5d(&D.mapC, stage + g * BM * 128, S.choff + g * 64, sx, I.x0, sy, I.y0);
             bulk_commit();
           }
         }
       }
-      // this CTA's items of layer l are stored: count them
+      // This CTA's items of layer l are stored: count them.  The epilogue
+      // threads' stores are ordered before the count by the barrier and the
+      // count's release semantics (cumulative over what the barrier made
+      // visible to this thread), so a consumer that acquires the counter
+      // sees them.  (With TMA stores, waiting for their completion and a
+      // full __threadfence here cost about a microsecond per layer.)
+      epilogue_sync();
       if (row == 0) {
-        bulk_wait_all();
-        fence_async_global();
-        __threadfence();
-        const unsigned before = atomicAdd(&P.grid_bar[l], (unsigned)mine);
-        // the CTA completing the layer's count stamps its end
-        if (P.stamps && before + (unsigned)mine == (unsigned)S.n_items)
-          P.stamps[P.n_layers + l] = global_ns();
+        if (S.kind == DECONV) {                // TMA stores: complete, then ordered
+          bulk_wait_all();
+          fence_async_global();
+        }
+        if (P.stamps) {
+          const unsigned before = atom_add_release_gpu(&P.grid_bar[l], (unsigned)mine);
+          // the CTA completing the layer's count stamps its end
+          if (before + (unsigned)mine == (unsigned)S.n_items) P.stamps[P.n_layers + l] = global_ns();
+        } else {
+          red_add_release_gpu(&P.grid_bar[l], (unsigned)mine);
+        }
       }
     }
   }
@@ -907,34 +952,18 @@ cudaError_t conv_make_maps(ConvLayer& L, bool bf16) {
           CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
-  // output store map: conv [out_h][out_w][ldc]; deconv viewed as
-  // [in_h][s][in_w][s][ldc] so one sub-pixel position of a tile is one box
-  const int sg = L.bn < 64 ? L.bn : 64;
-  const CUtensorMapSwizzle osw = (sg == 64) ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
-  const cuuint64_t LD = (cuuint64_t)L.ldc;
   if (L.kind == DECONV) {
-    const cuuint64_t S = (cuuint64_t)L.s, IW = (cuuint64_t)L.in_w, IH = (cuuint64_t)L.in_h;
-    const cuuint64_t OW = (cuuint64_t)L.out_w;
+    // output store map: [in_h][s][in_w][s][ldc] view of the output, so one
+    // sub-pixel position of a tile is one box of 64 channels
+    if (L.bn % 64) return cudaErrorInvalidValue;
+    const cuuint64_t LD = (cuuint64_t)L.ldc, S = (cuuint64_t)L.s;
+    const cuuint64_t IW = (cuuint64_t)L.in_w, IH = (cuuint64_t)L.in_h, OW = (cuuint64_t)L.out_w;
     cuuint64_t dims[5] = {LD, S, IW, S, IH};
     cuuint64_t strides[4] = {LD * 2, S * LD * 2, OW * LD * 2, S * OW * LD * 2};
-    cuuint32_t box[5] = {(cuuint32_t)sg, 1, (cuuint32_t)TW, 1, (cuuint32_t)TH};
+    cuuint32_t box[5] = {64, 1, (cuuint32_t)TW, 1, (cuuint32_t)TH};
     cuuint32_t es[5] = {1, 1, 1, 1, 1};
-    r = enc(&L.mapC, dt, 5, L.out, dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, osw,
-            CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  } else {
-    cuuint64_t dims[3] = {LD, (cuuint64_t)L.out_w, (cuuint64_t)L.out_h};
-    cuuint64_t strides[2] = {LD * 2, (cuuint64_t)L.out_w * LD * 2};
-    cuuint32_t box[3] = {(cuuint32_t)sg, (cuuint32_t)TW, (cuuint32_t)TH};
-    cuuint32_t es[3] = {1, 1, 1};
-    r = enc(&L.mapC, dt, 3, L.out, dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, osw,
-            CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
-    // 16-channel boxes, unswizzled 32-byte rows: one owner's share of a
-    // split-K tile reduced through distributed shared memory
-    cuuint32_t box16[3] = {16, (cuuint32_t)TW, (cuuint32_t)TH};
-    r = enc(&L.mapC16, dt, 3, L.out, dims, strides, box16, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
-            CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_NONE,
-            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    r = enc(&L.mapC, dt, 5, L.out, dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+            CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   }
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
@@ -963,7 +992,6 @@ cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, unsigned* grid_b
     LayerDesc& D = P->L[i];
     D.mapA = L.mapA;
     D.mapB = L.mapB;
-    D.mapC = L.mapC;
     D.bias = L.bias;
     D.ws = L.ws;
     D.counters = L.counters;
@@ -979,7 +1007,12 @@ cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, unsigned* grid_b
     D.n_tiles = L.n_tiles_n;
     D.choff = L.choff;
     D.wait_layers = L.wait_layers;
-    D.mapC16 = L.mapC16;
+    D.mapC = L.mapC;
+    D.out = L.out;
+    D.ow = L.out_w;
+    D.ldc = L.ldc;
+    D.gw = L.gw;
+    D.gh = L.gh;
     D.halo = conv_uses_halo(L) ? 1 : 0;
     // a split of a 64-wide tile into 2 or kMaxSplits slices, one item per
     // CTA, reduces its slices through distributed shared memory within a

@@ -109,11 +109,11 @@ struct ConvLayer {
   void* out;             // device [out_h][out_w][ldc]
   const void* wpacked;   // device, K-major: conv [Cout][9][Cin]; deconv [s*s*Cout][Cin]
   const float* bias;     // device [Cout]
-  CUtensorMap mapA, mapB, mapC;   // input, packed weights, output (store)
-  CUtensorMap mapC16;             // output with 16-channel boxes (convs)
+  CUtensorMap mapA, mapB;         // input (tap boxes or halo tiles), packed weights
+  CUtensorMap mapC;               // deconvs: output store map
 };
 
-// Encode the layer's tensor maps (input activations, packed weights, output).
+// Encode the layer's tensor maps (input activations, packed weights).
 cudaError_t conv_make_maps(ConvLayer& L, bool bf16);
 // Whether the layer reads its A operand as halo tiles (one box per tile and
 // 64-channel chunk, shared by the 9 taps) instead of one box per tap: 3x3
@@ -129,8 +129,8 @@ int conv_tile_m();
 constexpr int kMaxLayers = 20;
 constexpr int kMaxSplits = 4;     // split-K slices per tile (the reducing slice keeps one load per slice in flight)
 struct alignas(128) LayerDesc {   // CUtensorMap is 128-byte aligned
-  CUtensorMap mapA, mapB, mapC;
-  CUtensorMap mapC16;            // output map with 16-channel boxes (split-K through DSMEM)
+  CUtensorMap mapA, mapB;
+  CUtensorMap mapC;              // deconvs: output store map (convs store from registers)
   const float* bias;
   float* ws;
   int* counters;
@@ -141,6 +141,8 @@ struct alignas(128) LayerDesc {   // CUtensorMap is 128-byte aligned
   int cta_lo, cta_hi;            // the CTAs this layer's items are dealt to (round-robin)
   int wait_items;                // items of layer wait_layers - 1 (its counter's target)
   int halo;                      // 3x3 stride-1 with 64-channel k-blocks: A from halo tiles
+  void* out;                     // output [out_h][ow][ldc], channels from choff
+  int ow, ldc, gw, gh;           // output row length, pixel stride, tile grid extent
 };
 struct BackboneParams {
   LayerDesc L[kMaxLayers];
