@@ -44,7 +44,7 @@ METRIC = "complete-detection latency p50/p99 ms RTCC vs barrier; conv TFLOP/s, f
 # without its cluster dimension, so block 3 reduced its split-K partials
 # through global memory; they stay in L2 either way); None once the kernel
 # changes and until it is captured again
-BACKBONE_TRAFFIC = 16_635_136
+BACKBONE_TRAFFIC = 16_597_504
 WORKLOAD = "pp3"
 DATA = ("synthetic: seeded uniform + Gaussian-cluster point clouds, He-normal fp32 weights "
         "rounded to fp16, seeded arrival traces (OPV2V and the trained OpenCOOD model are not "
