@@ -78,15 +78,14 @@ __global__ void k_pillar_cells(const float4* __restrict__ pts, const int* __rest
     }
   }
   if (i == 0) stats[0] = n;
-  bool ok = false;
   if (i < n) {
     const float4 p = src_pts ? src_pts[i] : pts[i];
     if (dst_pts) dst_pts[i] = p;
     // IEEE float32 subtraction and division with round-to-nearest.
     const float fx = __fdiv_rn(__fsub_rn(p.x, g.x_min), g.v);
     const float fy = __fdiv_rn(__fsub_rn(p.y, g.y_min), g.v);
-    ok = (p.z >= g.z_min) && (p.z < g.z_max) && (fx >= 0.f) && (fx < (float)g.W) &&
-         (fy >= 0.f) && (fy < (float)g.H);
+    const bool ok = (p.z >= g.z_min) && (p.z < g.z_max) && (fx >= 0.f) && (fx < (float)g.W) &&
+                    (fy >= 0.f) && (fy < (float)g.H);
     int cell = -1;
     if (ok) {
       const int ix = (int)floorf(fx);
@@ -97,8 +96,6 @@ __global__ void k_pillar_cells(const float4* __restrict__ pts, const int* __rest
     }
     cell_of[i] = cell;
   }
-  const unsigned in_range = __ballot_sync(kFull, ok);
-  if ((threadIdx.x & 31) == 0 && in_range) atomicAdd(&stats[1], __popc(in_range));
 }
 
 // Flag and count of point i for the pillar scan.
@@ -152,21 +149,28 @@ constexpr int kScanThreads = 256;
 constexpr int kItems = kScanTile / kScanThreads;   // 4 consecutive points per thread
 static_assert(kItems == 4, "the item loads below move 4 points per thread");
 
+// Same-address atomics serialise in L2, so the pass's counters are summed per
+// block and added once per block (here and in the scan), not per point, warp
+// or pillar.
 __global__ void __launch_bounds__(kScanThreads)
 k_pillar_blocksum(const int* __restrict__ n_hdr, const int* __restrict__ cell_of,
                   const int* __restrict__ cnt_cell, const int* __restrict__ first_cell,
-                  int2* __restrict__ items, int2* __restrict__ blocksum) {
+                  int2* __restrict__ items, int2* __restrict__ blocksum, int* __restrict__ stats) {
   pdl_trigger();
   pdl_wait();
   const int n = *n_hdr;
   const int base = blockIdx.x * kScanTile + threadIdx.x * kItems;
   int2 s = make_int2(0, 0);
   int2 it[kItems];
+  int inr = 0;                                 // points inside the grid
 #pragma unroll
   for (int q = 0; q < kItems; ++q) {
     it[q] = first_point_item(base + q, n, cell_of, cnt_cell, first_cell);
     s = add2(s, it[q]);
+    inr += (base + q < n && cell_of[base + q] >= 0) ? 1 : 0;
   }
+#pragma unroll
+  for (int d = 16; d > 0; d >>= 1) inr += __shfl_xor_sync(kFull, inr, d);
   if (base < n) {
     int4* dst = reinterpret_cast<int4*>(items + base);
     dst[0] = make_int4(it[0].x, it[0].y, it[1].x, it[1].y);
@@ -175,20 +179,31 @@ k_pillar_blocksum(const int* __restrict__ n_hdr, const int* __restrict__ cell_of
 #pragma unroll
   for (int d = 16; d > 0; d >>= 1) s = add2(s, shfl_xor2(s, d));
   __shared__ int2 ws[32];
+  __shared__ int wi[32];
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-  if (lane == 0) ws[wid] = s;
+  if (lane == 0) {
+    ws[wid] = s;
+    wi[wid] = inr;
+  }
   __syncthreads();
   if (wid == 0) {
     int2 t = lane < (int)(blockDim.x >> 5) ? ws[lane] : make_int2(0, 0);
+    int ti = lane < (int)(blockDim.x >> 5) ? wi[lane] : 0;
 #pragma unroll
-    for (int d = 16; d > 0; d >>= 1) t = add2(t, shfl_xor2(t, d));
-    if (lane == 0) blocksum[blockIdx.x] = t;
+    for (int d = 16; d > 0; d >>= 1) {
+      t = add2(t, shfl_xor2(t, d));
+      ti += __shfl_xor_sync(kFull, ti, d);
+    }
+    if (lane == 0) {
+      blocksum[blockIdx.x] = t;
+      if (ti) atomicAdd(&stats[1], ti);
+    }
   }
 }
 
 __global__ void __launch_bounds__(kScanThreads)
 k_pillar_scan(const int* __restrict__ n_hdr, const int* __restrict__ cell_of,
-              const int2* __restrict__ items, const int2* __restrict__ blocksum, int P,
+              const int2* __restrict__ items, const int2* __restrict__ blocksum, int P, int N,
               int* __restrict__ c2p,
               int* __restrict__ pillar_cell, int* __restrict__ pcnt_raw, int* __restrict__ poff,
               int* __restrict__ cursor, int* __restrict__ stats) {
@@ -221,6 +236,7 @@ k_pillar_scan(const int* __restrict__ n_hdr, const int* __restrict__ cell_of,
   for (int q = 0; q < kItems; ++q) own = add2(own, it[q]);
   int2 run = block_excl_scan(own, &tot);
   run = add2(run, pre);
+  int kept = 0, raw = 0;                       // points of this thread's kept pillars
 #pragma unroll
   for (int q = 0; q < kItems; ++q) {
     if (it[q].x) {
@@ -233,9 +249,30 @@ k_pillar_scan(const int* __restrict__ n_hdr, const int* __restrict__ cell_of,
         pcnt_raw[pid] = it[q].y;
         poff[pid] = run.y;
         cursor[pid] = 0;
+        kept += it[q].y < N ? it[q].y : N;
+        raw += it[q].y;
       }
     }
     run = add2(run, it[q]);
+  }
+  // the PFN keeps min(raw, N) points of a pillar: stats 3 (kept), 6 (dropped
+  // by the per-pillar cap), 7 (points of kept pillars), summed per block
+  __shared__ int2 wk[32];
+#pragma unroll
+  for (int d = 16; d > 0; d >>= 1) {
+    kept += __shfl_xor_sync(kFull, kept, d);
+    raw += __shfl_xor_sync(kFull, raw, d);
+  }
+  if (lane == 0) wk[threadIdx.x >> 5] = make_int2(kept, raw);
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int2 t = make_int2(0, 0);
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t = add2(t, wk[w]);
+    if (t.y) {
+      atomicAdd(&stats[3], t.x);
+      atomicAdd(&stats[6], t.y - t.x);
+      atomicAdd(&stats[7], t.y);
+    }
   }
   if (blockIdx.x == gridDim.x - 1 && threadIdx.x == 0) {
     const int total = pre.x + tot.x;
@@ -302,15 +339,13 @@ k_pfn(const float4* __restrict__ pts, const int* __restrict__ stats_in,
       const int* __restrict__ list, const int* __restrict__ pillar_cell,
       const float* __restrict__ w, const float* __restrict__ b, GridGeom g, int N,
       T* __restrict__ image, int* __restrict__ cell2pillar, int* __restrict__ np_prev,
-      int* __restrict__ pcount, int* __restrict__ stats) {
+      int* __restrict__ pcount) {
   __shared__ float sw[C * 9];
   __shared__ float sb[C];
-  __shared__ int s_stat[3];                   // kept, capped, raw (block partial sums)
   pdl_trigger();
   for (int j = threadIdx.x; j < C * 9; j += blockDim.x) sw[j] = w[j];   // weights: constant
   pdl_wait();
   for (int j = threadIdx.x; j < C; j += blockDim.x) sb[j] = b[j];
-  if (threadIdx.x < 3) s_stat[threadIdx.x] = 0;
   __syncthreads();
   const int lane = threadIdx.x & 31;
   const int p = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -394,18 +429,7 @@ k_pfn(const float4* __restrict__ pts, const int* __restrict__ stats_in,
     if (lane == 0) {
       cell2pillar[cell] = p;
       pcount[p] = m;
-      atomicAdd(&s_stat[0], m);
-      atomicAdd(&s_stat[1], raw - m);
-      atomicAdd(&s_stat[2], raw);
     }
-  }
-  // one global update per block (same-address atomics from every pillar
-  // serialise in L2)
-  __syncthreads();
-  if (threadIdx.x == 0 && s_stat[2] > 0) {
-    atomicAdd(&stats[3], s_stat[0]);
-    atomicAdd(&stats[6], s_stat[1]);
-    atomicAdd(&stats[7], s_stat[2]);
   }
 }
 
@@ -422,10 +446,10 @@ cudaError_t launch_all(const PillarBufs& b, const GridGeom& g, const float* pfn_
                  b.src_hdr, b.src_pts, b.dst_hdr, b.dst_pts);
   if (e != cudaSuccess) return e;
   e = launch_pdl(k_pillar_blocksum, dim3(nblk), dim3(kScanThreads), 0, st, b.n_hdr, b.cell_of,
-                 b.cnt_cell, b.first_cell, b.items, b.blocksum);
+                 b.cnt_cell, b.first_cell, b.items, b.blocksum, b.stats);
   if (e != cudaSuccess) return e;
   e = launch_pdl(k_pillar_scan, dim3(nblk), dim3(kScanThreads), 0, st, b.n_hdr, b.cell_of,
-                 b.items, b.blocksum, b.P, b.c2p, b.pillar_cell, b.pcnt_raw, b.poff, b.cursor,
+                 b.items, b.blocksum, b.P, b.N, b.c2p, b.pillar_cell, b.pcnt_raw, b.poff, b.cursor,
                  b.stats);
   if (e != cudaSuccess) return e;
   e = launch_pdl(k_pillar_fill, dim3((b.cap + 255) / 256), dim3(256), 0, st, b.n_hdr, b.cell_of,
@@ -433,7 +457,7 @@ cudaError_t launch_all(const PillarBufs& b, const GridGeom& g, const float* pfn_
   if (e != cudaSuccess) return e;
   e = launch_pdl(k_pfn<T, C>, dim3((b.P + 7) / 8), dim3(256), 0, st, b.pts, b.stats, b.pcnt_raw,
                  b.poff, b.list, b.pillar_cell, pfn_w, pfn_b, g, b.N, static_cast<T*>(b.image),
-                 b.cell2pillar, b.np_prev, b.pcount, b.stats);
+                 b.cell2pillar, b.np_prev, b.pcount);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
