@@ -79,7 +79,7 @@ __device__ int block_scan_excl(int v, int* total) {
 // The thread's contiguous chunk of keys, 16 bytes at a time (the key array is
 // padded with invalid keys to kThreads * chunk entries).  f(key, index).
 template <typename F>
-__device__ __forceinline__ void for_chunk(const uint32_t* __restrict__ keys, int lo, int chunk4,
+__device__ __forceinline__ void for_chunk(const uint32_t* keys, int lo, int chunk4,
                                           F f) {
   const uint4* v = reinterpret_cast<const uint4*>(keys + lo);
   constexpr int B = 8;                                   // loads in flight per thread
@@ -104,7 +104,7 @@ __device__ __forceinline__ void for_chunk(const uint32_t* __restrict__ keys, int
 // Coalesced pass over the (padded) key array: thread t takes the 16-byte
 // vectors t, t + kThreads, ...; f(key, index).
 template <typename F>
-__device__ __forceinline__ void for_strided(const uint32_t* __restrict__ keys, int n4, F f) {
+__device__ __forceinline__ void for_strided(const uint32_t* keys, int n4, F f) {
   const uint4* v = reinterpret_cast<const uint4*>(keys);
   constexpr int B = 8;                                   // loads in flight per thread
   for (int base = threadIdx.x; base < n4; base += B * kThreads) {
@@ -205,7 +205,7 @@ __device__ __forceinline__ void merge_level(const unsigned long long* src, unsig
 }
 
 // Box of the selected pair v (anchor = its low 32 bits), written to out.
-__device__ __forceinline__ void decode_box(unsigned long long v, const float* __restrict__ head,
+__device__ __forceinline__ void decode_box(unsigned long long v, const float* head,
                                            const AnchorGeo& g, rtcc_box* out) {
   const int a = static_cast<int>(v & 0xFFFFFFFFull);
   const int cell = a / g.anchors, an = a - cell * g.anchors;
@@ -229,11 +229,9 @@ __device__ __forceinline__ void decode_box(unsigned long long v, const float* __
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
-k_decode_select(const uint32_t* __restrict__ keys, uint32_t* __restrict__ hist0,
-                const float* __restrict__ head, int chunk4, int max_boxes, AnchorGeo g,
-                const int* __restrict__ err, DetResultHeader* __restrict__ hdr,
-                rtcc_box* __restrict__ boxes, int* __restrict__ present, int K,
-                volatile int* __restrict__ done) {
+k_decode_select(const uint32_t* keys, uint32_t* hist0, const float* head, int chunk4, int max_boxes,
+                AnchorGeo g, const int* err, DetResultHeader* __restrict__ hdr,
+                rtcc_box* __restrict__ boxes, int* present, int K, volatile int* __restrict__ done) {
   extern __shared__ unsigned long long bnd[];        // [kBndCap] keys of bin b0
   __shared__ int hist[kThreads];                     // level-1/2 histograms (10 bits)
   __shared__ unsigned long long sel[kDecodeKeep];    // selected, unordered

@@ -175,7 +175,7 @@ struct Group {
 
 template <typename T, int C, bool ATTN>
 __global__ void __launch_bounds__(kThreads, 1)
-k_fuse_head(const void* const* __restrict__ feats, const int* __restrict__ present, int K,
+k_fuse_head(const void* const* __restrict__ feats, const int* present, int K,
             int cells, float inv_sqrt_c, const float* __restrict__ head_wp,
             const float* __restrict__ head_b, float* __restrict__ head_out, T* __restrict__ fused,
             uint32_t* __restrict__ keys, uint32_t* __restrict__ hist0, float cls_thresh,

@@ -39,15 +39,21 @@ namespace {
 
 constexpr unsigned kFull = 0xFFFFFFFFu;
 
+// Pointers to data an earlier kernel of the chain writes are not __restrict__:
+// a read through a const __restrict__ pointer may be scheduled above
+// griddepcontrol.wait (the qualifier promises the data does not change while
+// the kernel runs), and would then read the predecessor's output before it is
+// complete.  Only the constant PFN weights keep the qualifier.
+
 template <int CH>
-__global__ void k_pillar_cells(const float4* __restrict__ pts, const int* __restrict__ n_hdr,
-                               GridGeom g, int* __restrict__ cell_of, int* __restrict__ cnt_cell,
-                               int* __restrict__ first_cell, int* __restrict__ stats,
-                               const int* __restrict__ prev_cell, const int* __restrict__ np_prev,
-                               int clear_all, uint4* __restrict__ image,
-                               int* __restrict__ cell2pillar, int* __restrict__ present_flag,
-                               const int* __restrict__ src_hdr, const float4* __restrict__ src_pts,
-                               int* __restrict__ dst_hdr, float4* __restrict__ dst_pts) {
+__global__ void k_pillar_cells(const float4* pts, const int* n_hdr,
+                               GridGeom g, int* cell_of, int* cnt_cell,
+                               int* first_cell, int* stats,
+                               const int* prev_cell, const int* np_prev,
+                               int clear_all, uint4* image,
+                               int* cell2pillar, int* present_flag,
+                               const int* src_hdr, const float4* src_pts,
+                               int* dst_hdr, float4* dst_pts) {
   __shared__ int s_n;
   pdl_trigger();
   pdl_wait();
@@ -153,9 +159,9 @@ static_assert(kItems == 4, "the item loads below move 4 points per thread");
 // block and added once per block (here and in the scan), not per point, warp
 // or pillar.
 __global__ void __launch_bounds__(kScanThreads)
-k_pillar_blocksum(const int* __restrict__ n_hdr, const int* __restrict__ cell_of,
-                  const int* __restrict__ cnt_cell, const int* __restrict__ first_cell,
-                  int2* __restrict__ items, int2* __restrict__ blocksum, int* __restrict__ stats) {
+k_pillar_blocksum(const int* n_hdr, const int* cell_of,
+                  const int* cnt_cell, const int* first_cell,
+                  int2* items, int2* blocksum, int* stats) {
   pdl_trigger();
   pdl_wait();
   const int n = *n_hdr;
@@ -202,11 +208,11 @@ k_pillar_blocksum(const int* __restrict__ n_hdr, const int* __restrict__ cell_of
 }
 
 __global__ void __launch_bounds__(kScanThreads)
-k_pillar_scan(const int* __restrict__ n_hdr, const int* __restrict__ cell_of,
-              const int2* __restrict__ items, const int2* __restrict__ blocksum, int P, int N,
-              int* __restrict__ c2p,
-              int* __restrict__ pillar_cell, int* __restrict__ pcnt_raw, int* __restrict__ poff,
-              int* __restrict__ cursor, int* __restrict__ stats) {
+k_pillar_scan(const int* n_hdr, const int* cell_of,
+              const int2* items, const int2* blocksum, int P, int N,
+              int* c2p,
+              int* pillar_cell, int* pcnt_raw, int* poff,
+              int* cursor, int* stats) {
   __shared__ int2 pre;
   __shared__ int2 tot;
   pdl_trigger();
@@ -280,10 +286,10 @@ k_pillar_scan(const int* __restrict__ n_hdr, const int* __restrict__ cell_of,
   }
 }
 
-__global__ void k_pillar_fill(const int* __restrict__ n_hdr, const int* __restrict__ cell_of,
-                              const int* __restrict__ c2p, int P, const int* __restrict__ poff,
-                              int* __restrict__ cursor, int* __restrict__ list,
-                              int* __restrict__ cnt_cell, int* __restrict__ first_cell) {
+__global__ void k_pillar_fill(const int* n_hdr, const int* cell_of,
+                              const int* c2p, int P, const int* poff,
+                              int* cursor, int* list,
+                              int* cnt_cell, int* first_cell) {
   pdl_trigger();
   pdl_wait();
   const int n = *n_hdr;
@@ -334,12 +340,12 @@ __device__ __forceinline__ float warp_sum(float v) {
 
 template <typename T, int C>
 __global__ void __launch_bounds__(256)
-k_pfn(const float4* __restrict__ pts, const int* __restrict__ stats_in,
-      const int* __restrict__ pcnt_raw, const int* __restrict__ poff,
-      const int* __restrict__ list, const int* __restrict__ pillar_cell,
+k_pfn(const float4* pts, const int* stats_in,
+      const int* pcnt_raw, const int* poff,
+      const int* list, const int* pillar_cell,
       const float* __restrict__ w, const float* __restrict__ b, GridGeom g, int N,
-      T* __restrict__ image, int* __restrict__ cell2pillar, int* __restrict__ np_prev,
-      int* __restrict__ pcount) {
+      T* image, int* cell2pillar, int* np_prev,
+      int* pcount) {
   __shared__ float sw[C * 9];
   __shared__ float sb[C];
   pdl_trigger();
