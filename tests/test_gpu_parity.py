@@ -315,3 +315,19 @@ def test_layer_spans_follow_dependencies(R):
             for d in dl:
                 assert start[l] >= end[d] - tol, (l, d, start[l], end[d])
     np.testing.assert_allclose(dur, spans[0][1] - spans[0][0], rtol=0, atol=1e-6)
+
+
+def test_long_range_attention_bf16_full_size(R):
+    # 5 agents, 704x200 grid, 120k points each, per-cell attention fusion with
+    # the ego agent as query, bf16 storage; one agent masked out
+    cfg = synth.get_config("lr5")
+    ctx, *_ = _end_to_end(R, cfg, frame=1, absent=(2,))
+    R.rtcc_destroy(ctx)
+
+
+def test_eight_agent_stress_full_size(R):
+    # 8 agents, 704x200 grid, 150k points each, max fusion; all eight payloads
+    # complete at once (branches contend for the GPU)
+    cfg = synth.get_config("stress8")
+    ctx, *_ = _end_to_end(R, cfg, frame=1, arrivals=[0.0] * cfg.n_agents)
+    R.rtcc_destroy(ctx)
