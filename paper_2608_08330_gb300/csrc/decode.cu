@@ -12,18 +12,22 @@
 //      the count of keys in lower bins;
 //   2. one coalesced pass over the keys selects the keys of lower bins and
 //      lists the keys of bin b0 in shared memory;
-//   3. a histogram of the listed keys' next 10 bits splits them into selected
-//      ones, the few of the bin b1 that holds the K-th pair, and the rest;
-//   4. the selected pairs are ordered (warp bitonic runs of 32, then merge
-//      levels that place each pair by one binary search in its partner run;
-//      the pairs are distinct) and the lowest pairs of bin b1 complete the K;
-//   5. each ranked pair is decoded into the box of its rank (staged in shared
+//   3. when both lists together fit one pair per thread (the usual case),
+//      each pair's rank is the count of smaller pairs in its own list: the
+//      lower bins' pairs take ranks 0 .. below-1, bin b0's pairs of rank
+//      below K - below complete the K;
+//   4. each ranked pair is decoded into the box of its rank (staged in shared
 //      memory, then stored into the pinned host result block).
-// When bin b0 or b1 is too full for the shared-memory lists (e.g. many equal
-// logits), a radix select over the global keys (next 10 + 10 bits) finds the
-// exact K-th key instead, the keys below it are collected, and an ordered pass
-// (each thread owns a contiguous range of anchors, a block scan ranks its
-// ties) adds the lowest-index keys equal to it.
+// Larger lists take two more steps instead of 3: a histogram of the listed
+// keys' next 10 bits splits them into selected ones, the few of the bin b1
+// that holds the K-th pair, and the rest; the selected pairs are ordered (warp
+// bitonic runs of 32, then merge levels that place each pair by one binary
+// search in its partner run; the pairs are distinct) and the lowest pairs of
+// bin b1 complete the K.  When bin b0 or b1 is too full for the shared-memory
+// lists (e.g. many equal logits), a radix select over the global keys (next
+// 10 + 10 bits) finds the exact K-th key instead, the keys below it are
+// collected, and an ordered pass (each thread owns a contiguous range of
+// anchors, a block scan ranks its ties) adds the lowest-index keys equal to it.
 #include <cmath>
 
 #include "common.cuh"
@@ -140,6 +144,27 @@ __device__ __forceinline__ void warp_append(bool pred, unsigned long long e, int
   if (pred) arr[base + __popc(m & ((1u << lane) - 1u))] = e;
 }
 
+// Count of the pairs of a shared-memory list[0..n) (16-byte aligned) below v,
+// shared by the S lanes q = 0..S-1 of a group (S a power of two): lane q
+// reads the 16-byte chunks q, q + S, ... (two pairs each) and lane 0 the odd
+// last pair.  The lanes of a group read consecutive chunks and the groups of
+// a warp the same ones.  The caller sums the lanes.  (The count is bound by
+// the shared-memory bandwidth: every compare's operand is delivered to its
+// lane; explicit 16-byte loads halve the load instructions.)
+__device__ __forceinline__ int count_below(const unsigned long long* list, int n, int q, int S,
+                                           unsigned long long v) {
+  const ulonglong2* l2 = reinterpret_cast<const ulonglong2*>(list);
+  const int n2 = n >> 1;
+  int cnt = 0;
+#pragma unroll 4
+  for (int j = q; j < n2; j += S) {
+    const ulonglong2 x = l2[j];
+    cnt += (x.x < v ? 1 : 0) + (x.y < v ? 1 : 0);
+  }
+  if ((n & 1) && q == 0) cnt += list[n - 1] < v ? 1 : 0;
+  return cnt;
+}
+
 // Ascending bitonic sort of one value per lane across a warp.
 __device__ __forceinline__ unsigned long long warp_sort32(unsigned long long v, int lane) {
 #pragma unroll
@@ -167,18 +192,9 @@ __device__ __forceinline__ int sort_width(int n) {
   return p;
 }
 __device__ __forceinline__ void sort_phase1(const unsigned long long* in, int n, int t0, int P,
-                                            unsigned long long* run, const float* head, int anchors) {
+                                            unsigned long long* run) {
   const int t = threadIdx.x - t0;
-  if (t >= 0 && t < P) {
-    const unsigned long long v = t < n ? in[t] : ~0ull;
-    if (t < n) {
-      // the head row of this pair is read when its box is decoded: fetch it
-      // into L1 while the pairs are ranked
-      const int cell = static_cast<int>(v & 0xFFFFFFFFull) / anchors;
-      asm volatile("prefetch.global.L1 [%0];" ::"l"(head + (size_t)cell * 16));
-    }
-    run[t] = warp_sort32(v, threadIdx.x & 31);
-  }
+  if (t >= 0 && t < P) run[t] = warp_sort32(t < n ? in[t] : ~0ull, threadIdx.x & 31);
 }
 // One level of the merge sort over warp-sorted runs, by the threads
 // [t0, t0 + P): the runs of R pairs in src[0..P) merge pairwise into runs of
@@ -232,9 +248,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 k_decode_select(const uint32_t* keys, uint32_t* hist0, const float* head, int chunk4, int max_boxes,
                 AnchorGeo g, const int* err, DetResultHeader* __restrict__ hdr,
                 rtcc_box* __restrict__ boxes, int* present, int K, volatile int* __restrict__ done) {
-  extern __shared__ unsigned long long bnd[];        // [kBndCap] keys of bin b0
+  extern __shared__ __align__(16) unsigned long long bnd[];  // [kBndCap] keys of bin b0
   __shared__ int hist[kThreads];                     // level-1/2 histograms (10 bits)
-  __shared__ unsigned long long sel[kDecodeKeep];    // selected, unordered
+  __shared__ __align__(16) unsigned long long sel[kDecodeKeep];  // selected, unordered
   __shared__ unsigned long long tie[kTieCap];
   __shared__ __align__(16) rtcc_box sbox[kDecodeKeep];  // boxes in rank order
   __shared__ int s_total, s_bin, s_below, s_nsel, s_nb, s_nl, s_nt;
@@ -295,57 +311,84 @@ k_decode_select(const uint32_t* keys, uint32_t* hist0, const float* head, int ch
         }
       });
       __syncthreads();                                   // every thread has read nb0
-      // ---- 3. level 1 over bnd (key bits 10..19 = pair bits 42..51) ---------
-      for (int i = tid; i < 1024; i += kThreads) hist[i] = 0;
-      __syncthreads();
-      // many listed keys share their next 10 bits: lanes with the same bin add
-      // their count with one atomic (uniform trip count: warps stay converged)
-      for (int i0 = 0; i0 < nb0; i0 += kThreads) {
-        const int i = i0 + tid;
-        const int bin1 = i < nb0 ? (int)((bnd[i] >> 42) & 1023) : -1;
-        const unsigned peers = __match_any_sync(0xFFFFFFFFu, bin1);
-        if (bin1 >= 0 && (tid & 31) == __ffs(peers) - 1) atomicAdd(&hist[bin1], __popc(peers));
-      }
-      __syncthreads();
-      {
-        int run = block_scan_excl(hist[tid], &s_total);  // 1024 bins, one per thread
-        const int h = hist[tid];
-        if (below0 + run < need && below0 + run + h >= need) {
-          s_bin = tid;
-          s_below = below0 + run;
+      if (below0 + nb0 <= kThreads) {
+        // ---- 3. the candidates fit one per thread: rank each pair within its
+        // list by counting the smaller pairs there (pairs are distinct, so the
+        // ranks are a permutation).  The lower bins' pairs are all selected
+        // and come first in rank order; a pair of bin b0 is selected when its
+        // rank is below need - below0.  S lanes share a pair, each counting a
+        // strided part of the list (broadcast shared-memory reads), and the
+        // rank is the box slot: the box is decoded at once.
+        const int nc = below0 + nb0;
+        int S = 1;
+        while (S < 32 && nc * 2 * S <= kThreads) S <<= 1;
+        const int c = tid / S, q = tid & (S - 1);
+        const bool lower = c < below0;
+        unsigned long long v = 0;
+        int cnt = 0;
+        if (c < nc) {
+          v = lower ? sel[c] : bnd[c - below0];
+          cnt = lower ? count_below(sel, below0, q, S, v) : count_below(bnd, nb0, q, S, v);
         }
-        __syncthreads();
-      }
-      const int b1 = s_bin, below1 = s_below, nb1 = hist[b1];
-      if (nb1 <= kTieCap) {
-        // bin-1 entries below b1 are selected; those in b1 compete for the rest
-        for (int i = tid; i < nb0; i += kThreads) {
-          const unsigned long long e = bnd[i];
-          const int bin1 = (int)((e >> 42) & 1023);
-          warp_append(bin1 < b1, e, &s_nsel, sel);
-          warp_append(bin1 == b1, e, &s_nt, tie);
+        for (int o = S >> 1; o > 0; o >>= 1) cnt += __shfl_xor_sync(0xFFFFFFFFu, cnt, o);
+        if (c < nc && q == 0) {
+          const int slot = lower ? cnt : below0 + cnt;
+          if (slot < need) decode_box(v, head, g, sbox + slot);
         }
-        __syncthreads();
-        // ---- 4. order sel (below1 pairs) and tie (nb1 pairs, all above);
-        // ---- 5. each ranked pair is decoded straight into its box slot
-        // (bnd is free again and serves as the run buffer)
-        const int P1 = sort_width(below1), P2 = sort_width(nb1);
-        unsigned long long *a = bnd, *a2 = bnd + 2 * kDecodeKeep;              // sel runs
-        unsigned long long *b = bnd + kDecodeKeep, *b2 = bnd + kDecodeKeep + kTieCap;  // tie runs
-        sort_phase1(sel, below1, 0, P1, a, head, g.anchors);
-        sort_phase1(tie, nb1, kDecodeKeep, P2, b, head, g.anchors);
-        __syncthreads();
-        for (int R = 32; R < (P1 > P2 ? P1 : P2); R *= 2) {
-          merge_level(a, a2, 0, P1, R);
-          merge_level(b, b2, kDecodeKeep, P2, R);
-          __syncthreads();
-          if (R < P1) { unsigned long long* x = a; a = a2; a2 = x; }
-          if (R < P2) { unsigned long long* x = b; b = b2; b2 = x; }
-        }
-        if (tid < below1) decode_box(a[tid], head, g, sbox + tid);
-        const int tt = tid - kDecodeKeep;
-        if (tt >= 0 && tt < need - below1) decode_box(b[tt], head, g, sbox + below1 + tt);
         ranked = true;
+      } else {
+        // ---- 3'. level 1 over bnd (key bits 10..19 = pair bits 42..51) --------
+        for (int i = tid; i < 1024; i += kThreads) hist[i] = 0;
+        __syncthreads();
+        // many listed keys share their next 10 bits: lanes with the same bin add
+        // their count with one atomic (uniform trip count: warps stay converged)
+        for (int i0 = 0; i0 < nb0; i0 += kThreads) {
+          const int i = i0 + tid;
+          const int bin1 = i < nb0 ? (int)((bnd[i] >> 42) & 1023) : -1;
+          const unsigned peers = __match_any_sync(0xFFFFFFFFu, bin1);
+          if (bin1 >= 0 && (tid & 31) == __ffs(peers) - 1) atomicAdd(&hist[bin1], __popc(peers));
+        }
+        __syncthreads();
+        {
+          int run = block_scan_excl(hist[tid], &s_total);  // 1024 bins, one per thread
+          const int h = hist[tid];
+          if (below0 + run < need && below0 + run + h >= need) {
+            s_bin = tid;
+            s_below = below0 + run;
+          }
+          __syncthreads();
+        }
+        const int b1 = s_bin, below1 = s_below, nb1 = hist[b1];
+        if (nb1 <= kTieCap) {
+          // bin-1 entries below b1 are selected; those in b1 compete for the rest
+          for (int i = tid; i < nb0; i += kThreads) {
+            const unsigned long long e = bnd[i];
+            const int bin1 = (int)((e >> 42) & 1023);
+            warp_append(bin1 < b1, e, &s_nsel, sel);
+            warp_append(bin1 == b1, e, &s_nt, tie);
+          }
+          __syncthreads();
+          // ---- 4'. order sel (below1 pairs) and tie (nb1 pairs, all above);
+          // each ranked pair is decoded straight into its box slot
+          // (bnd is free again and serves as the run buffer)
+          const int P1 = sort_width(below1), P2 = sort_width(nb1);
+          unsigned long long *a = bnd, *a2 = bnd + 2 * kDecodeKeep;              // sel runs
+          unsigned long long *b = bnd + kDecodeKeep, *b2 = bnd + kDecodeKeep + kTieCap;  // tie runs
+          sort_phase1(sel, below1, 0, P1, a);
+          sort_phase1(tie, nb1, kDecodeKeep, P2, b);
+          __syncthreads();
+          for (int R = 32; R < (P1 > P2 ? P1 : P2); R *= 2) {
+            merge_level(a, a2, 0, P1, R);
+            merge_level(b, b2, kDecodeKeep, P2, R);
+            __syncthreads();
+            if (R < P1) { unsigned long long* x = a; a = a2; a2 = x; }
+            if (R < P2) { unsigned long long* x = b; b = b2; b2 = x; }
+          }
+          if (tid < below1) decode_box(a[tid], head, g, sbox + tid);
+          const int tt = tid - kDecodeKeep;
+          if (tt >= 0 && tt < need - below1) decode_box(b[tt], head, g, sbox + below1 + tt);
+          ranked = true;
+        }
       }
     }
 
@@ -404,7 +447,7 @@ k_decode_select(const uint32_t* keys, uint32_t* hist0, const float* head, int ch
       __syncthreads();
       const int P = sort_width(need);
       unsigned long long *a = bnd, *a2 = bnd + 2 * kDecodeKeep;
-      sort_phase1(sel, need, 0, P, a, head, g.anchors);
+      sort_phase1(sel, need, 0, P, a);
       __syncthreads();
       for (int R = 32; R < P; R *= 2) {
         merge_level(a, a2, 0, P, R);
