@@ -192,7 +192,7 @@ def oracle_step(cfg, w, pts_agent, arrivals_list):
     feats = [enc["feat"]] * cfg.n_agents
     F = of.fuse_max(feats) if cfg.fusion == "max" else of.fuse_attn(feats)
     hd = of.head(F, of.store_round(w["head.w"], cfg.dtype), of.store_round(w["head.b"], cfg.dtype))
-    of.decode(hd, cfg)
+    of.detect(hd, cfg)
     t2 = time.perf_counter()
     c_enc = int((t1 - t0) * 1e9)
     c_post = int((t2 - t1) * 1e9)

@@ -23,6 +23,8 @@ from typing import Dict, List, Optional, Sequence
 
 import numpy as np
 
+from . import nms
+
 # --------------------------------------------------------------------------
 # storage rounding
 # --------------------------------------------------------------------------
@@ -368,6 +370,21 @@ def decode(hd: np.ndarray, cfg, cls_thresh: Optional[float] = None,
     return {"idx": idx, "boxes": boxes}
 
 
+def detect(hd: np.ndarray, cfg) -> Dict[str, np.ndarray]:
+    """The final detections: the decode's top-K, then greedy rotated BEV NMS
+    at ``cfg.nms_iou`` (see :mod:`oracle.nms`); ``nms_iou <= 0`` skips it.
+
+    The paper's T^det ends after box decoding, score thresholding and rotated
+    NMS (Sec. V-A-3).
+    """
+    det = decode(hd, cfg)
+    thr = getattr(cfg, "nms_iou", 0.0)
+    if thr > 0 and len(det["idx"]):
+        keep = nms.nms(nms.bev(det["boxes"]), thr)
+        det = {"idx": det["idx"][keep], "boxes": det["boxes"][keep]}
+    return det
+
+
 # --------------------------------------------------------------------------
 # whole frame
 # --------------------------------------------------------------------------
@@ -375,7 +392,7 @@ def decode(hd: np.ndarray, cfg, cls_thresh: Optional[float] = None,
 
 def forward(points: Sequence[Optional[np.ndarray]], weights: Dict[str, np.ndarray], cfg,
             store: Optional[str] = None) -> Dict[str, object]:
-    """One frame: every present agent's encoder, then fusion, head and decode.
+    """One frame: every present agent's encoder, then fusion, head, decode and NMS.
 
     ``points[k] is None`` marks agent k absent (masked out of the fusion).  The
     result does not depend on the order or time at which encoders run: each
@@ -388,5 +405,5 @@ def forward(points: Sequence[Optional[np.ndarray]], weights: Dict[str, np.ndarra
     hw = store_round(weights["head.w"], store)
     hb = store_round(weights["head.b"], store)
     hd = head(F, hw, hb)
-    det = decode(hd, cfg)
+    det = detect(hd, cfg)
     return {"enc": enc, "fused": F, "head": hd, "det": det}

@@ -64,6 +64,7 @@ class ModelConfig:
     point_seed: int
     arrival: str                  # "fixed", "uniform", "lognormal", "slots", "zero"
     arrival_args: Tuple[float, ...] = ()
+    nms_iou: float = 0.15         # rotated BEV NMS: suppress IoU > nms_iou (0: no NMS)
 
     # ---- derived shapes (no arithmetic of the method, only bookkeeping) ----
     @property

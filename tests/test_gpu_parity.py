@@ -192,6 +192,54 @@ def test_decode_all_equal_logits(R, grid):
         R.rtcc_destroy(ctx)
 
 
+def _decode_path_sizes(hd, cls_thresh, max_boxes):
+    """The decode's list sizes for a head output, recomputed on the host: the
+    count below0 of keys in level-0 bins below the bin b0 that holds the K-th
+    key, that bin's size nb0, and the size nb1 of the level-1 bin (next 10 key
+    bits) that holds it.  Keys order the class logits descending as 32-bit
+    unsigned integers (the fusion kernel's encoding)."""
+    A = 2
+    logit = (hd[:A].transpose(1, 2, 0).reshape(-1).astype(np.float32) + np.float32(0.0))
+    u = logit.view(np.uint32)
+    asc = np.where(u & np.uint32(0x80000000), ~u, u | np.uint32(0x80000000))
+    key = (~asc)[logit >= np.float32(cls_thresh)]
+    need = min(max_boxes, key.size)
+    cum = np.cumsum(np.bincount(key >> 20, minlength=4096))
+    b0 = int(np.searchsorted(cum, need))
+    below0 = int(cum[b0 - 1]) if b0 > 0 else 0
+    inb = key[(key >> 20) == b0]
+    cum1 = np.cumsum(np.bincount((inb >> 10) & 1023, minlength=1024))
+    b1 = int(np.searchsorted(cum1, need - below0))
+    return below0, inb.size, int(cum1[b1] - (cum1[b1 - 1] if b1 > 0 else 0))
+
+
+def test_decode_level1_list_path(R):
+    # Class logits crowded into one level-0 key bin (logits about 1.03 +- 0.02)
+    # but spread over its next 10 bits: more candidates than the decode's
+    # threads, so it takes the level-1 histogram and warp-sort path instead of
+    # ranking by counting (which the other workloads take).
+    cfg = dataclasses.replace(_small_pp(grid=(96, 64)), cls_thresh=-1.0, max_boxes=500)
+    w = dict(synth.weights_for(cfg))
+    pts = [synth.points_for(cfg, 0, k) for k in range(cfg.n_agents)]
+    F = of.forward(pts, w, cfg, store=cfg.dtype)["fused"]
+    z = np.tensordot(of.store_round(w["head.w"], cfg.dtype)[:2], F, axes=(1, 0))
+    hw = w["head.w"].copy()
+    hw[:2] *= np.float32(0.02 / max(float(z.std()), 1e-6))
+    hb = w["head.b"].copy()
+    hb[:2] = 1.03
+    w["head.w"], w["head.b"] = hw, hb
+    ctx = R.rtcc_init(R.model_config(cfg, flags=U.DEBUG_FLAGS), synth.weight_blob(w))
+    try:
+        boxes = U.run_frame(ctx, cfg, pts, [0.0] * cfg.n_agents, R.MODE_RTCC)
+        hd = U.head_to_oracle_layout(R.rtcc_get_head(ctx, cfg.feat_h, cfg.feat_w))
+        below0, nb0, nb1 = _decode_path_sizes(hd, cfg.cls_thresh, cfg.max_boxes)
+        assert below0 + nb0 > 1024 and nb0 <= 4096 and nb1 <= 64, (below0, nb0, nb1)
+        assert len(boxes) == cfg.max_boxes
+        _check_decode(cfg, hd, boxes)
+    finally:
+        R.rtcc_destroy(ctx)
+
+
 def test_split_k_without_clusters_bit_identical(R):
     # The deepest block's 4-way split-K reduces through distributed shared
     # memory when the backbone runs in clusters of four CTAs, and through
