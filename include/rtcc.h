@@ -105,7 +105,7 @@ typedef enum {
  * stride-2 block must have even sizes); up_stride[b] in {1, 2, 4} for every
  * block, or all 0 for "no neck" (then n_blocks == 1 and the features are the
  * block's output); up_ch == 128 when a neck exists; anchors == 2;
- * 1 <= max_boxes <= 512.
+ * 1 <= max_boxes <= 512; 0 <= nms_iou <= 1.
  */
 typedef struct {
   int32_t n_agents;
@@ -130,6 +130,10 @@ typedef struct {
   int32_t max_boxes;                /* top-K after thresholding              */
   float cls_thresh;                 /* keep anchors whose class logit is
                                        >= cls_thresh                         */
+  float nms_iou;                    /* rotated BEV NMS after the top-K: a box
+                                       is dropped when its IoU with a kept
+                                       higher-ranked box exceeds nms_iou;
+                                       0 = no NMS; 0 <= nms_iou <= 1         */
   int32_t flags;                    /* RTCC_FLAG_*                           */
 } rtcc_model_config;
 
@@ -238,7 +242,9 @@ rtcc_status rtcc_frame_abort(struct rtcc_ctx* ctx);
 
 /*
  * Wait (host-side, up to timeout_ms; < 0 = no limit) until the frame's
- * detections are ready, then copy up to `cap` boxes (score-descending) to
+ * detections are ready -- decoded, thresholded, cut to max_boxes and, with
+ * nms_iou > 0, passed through rotated BEV NMS: the endpoint of T^det
+ * (Sec. V-A-3) -- then copy up to `cap` boxes (score-descending) to
  * out, their number to *n_out and the ready time to *t_ready_ms (any of the
  * three may be NULL).  Closes the frame.  RTCC_E_TIMEOUT leaves the frame
  * open (call again); RTCC_E_INFEASIBLE after rtcc_frame_abort;
@@ -282,6 +288,12 @@ rtcc_status rtcc_get_branch_state(struct rtcc_ctx* ctx, int32_t agent,
 
 /* Head output float32 [H'][W'][8A]. */
 rtcc_status rtcc_get_head(struct rtcc_ctx* ctx, float* host_out, size_t cap);
+
+/* The decode's top-K boxes before NMS (rank order: score descending, anchor
+ * index ascending), up to `cap` of them; *n_out = their count.  Without NMS
+ * (nms_iou == 0) these are the frame's result boxes. */
+rtcc_status rtcc_get_decoded(struct rtcc_ctx* ctx, rtcc_box* host_out, int32_t cap,
+                             int32_t* n_out);
 
 /* Pillarisation of `agent`: cell2pillar int32 [H*W] (-1 = empty),
  * pillar_cell int32 [P_max] (-1 pad), count int32 [P_max] (kept points), and
@@ -387,6 +399,18 @@ double rtcc_now_ms(void);
 /* Number of kernel launches one frame makes (branches + post-join), for the
  * given number of present agents. */
 int32_t rtcc_kernels_per_frame(struct rtcc_ctx* ctx, int32_t n_present);
+
+/*
+ * Rotated BEV NMS of n <= 512 boxes already in rank order (the frame's own
+ * post-join step, run on the caller's boxes on the current device): a box is
+ * dropped when its IoU with a kept earlier box exceeds iou (0 <= iou <= 1).
+ * Writes the kept boxes in order to host_out (room for n) and their number to
+ * *n_out.  Boxes are rectangles in x-y: centre (x, y), length l along
+ * (cos yaw, sin yaw), width w across it; z, h and score are carried along.
+ * Synchronous; allocates and frees its own device scratch.
+ */
+rtcc_status rtcc_nms(const rtcc_box* host_in, int32_t n, float iou, rtcc_box* host_out,
+                     int32_t* n_out);
 
 #ifdef __cplusplus
 }

@@ -91,7 +91,11 @@ struct rtcc_ctx {
   void* fused = nullptr;
   uint32_t* keys = nullptr;           // decode key per anchor (padded)
   uint32_t* hist0 = nullptr;          // decode level-0 histogram
-  uint8_t* det_host = nullptr;        // pinned; the decode kernel writes it directly
+  rtcc_box* dec_boxes = nullptr;      // NMS on: the decode's boxes (device), NMS input
+  int* dec_n = nullptr;               //         and their count
+  uint32_t* nms_mask = nullptr;       //         suppression bitmask scratch
+  unsigned* nms_ticket = nullptr;     //         last-block counter
+  uint8_t* det_host = nullptr;        // pinned; the decode (or NMS) kernel writes it directly
   size_t det_bytes = 0;
   volatile int* h_done = nullptr;     // pinned; the decode kernel sets it to 1 when det_host is complete
   bool present_dirty = false;         // a branch set its presence flag and no post-join cleared it
@@ -174,6 +178,7 @@ rtcc_status validate_config(const rtcc_model_config& c) {
   if (!pow2_in(c.pfn_ch, {32, 64})) return RTCC_E_ARG;
   if (c.n_blocks < 1 || c.n_blocks > RTCC_MAX_BLOCKS) return RTCC_E_ARG;
   if (c.anchors != 2 || c.max_boxes < 1 || c.max_boxes > 512) return RTCC_E_ARG;
+  if (!(c.nms_iou >= 0.f && c.nms_iou <= 1.f)) return RTCC_E_ARG;
   if (c.max_points < 0 || c.max_points > (1 << 24)) return RTCC_E_ARG;
   if (c.fusion != RTCC_FUSE_MAX && c.fusion != RTCC_FUSE_ATTN) return RTCC_E_ARG;
   if (c.dtype != RTCC_FP16 && c.dtype != RTCC_BF16) return RTCC_E_ARG;
@@ -629,6 +634,18 @@ rtcc_status capture_post(rtcc_ctx* c) {
   da.present = c->d_present;
   da.K = c->K;
   da.done = c->h_done;
+  da.dev_boxes = c->dec_boxes;                    // null without NMS
+  da.dev_n = c->dec_n;
+  NmsArgs na{};
+  na.in = c->dec_boxes;
+  na.n_in = c->dec_n;
+  na.mask = c->nms_mask;
+  na.ticket = c->nms_ticket;
+  na.max_boxes = c->cfg.max_boxes;
+  na.iou = c->cfg.nms_iou;
+  na.err = c->d_err;
+  na.out = c->det_host;
+  na.done = c->h_done;
   (void)cudaGetLastError();
   CK(cudaStreamBeginCapture(c->post, cudaStreamCaptureModeRelaxed));
   cudaError_t e = cudaSuccess;
@@ -642,6 +659,7 @@ rtcc_status capture_post(rtcc_ctx* c) {
   }
   if (e == cudaSuccess && tl) e = record_node(c->ev_fuse1, c->post);
   if (e == cudaSuccess) e = launch_decode(da, c->post);
+  if (e == cudaSuccess && c->dec_boxes) e = launch_nms(na, c->post);
   if (e == cudaSuccess && tl) e = record_node(c->ev_post1, c->post);
   cudaGraph_t graph = nullptr;
   cudaError_t e2 = cudaStreamEndCapture(c->post, &graph);
@@ -699,6 +717,14 @@ rtcc_status init_impl(rtcc_ctx* c, const float* weights) {
   CK(cudaMemset(c->keys, 0xFF, nkeys * sizeof(uint32_t)));   // padding stays invalid
   RS(dalloc(c, &c->hist0, kDecodeHistBins * sizeof(uint32_t)));
   CK(cudaMemset(c->hist0, 0, kDecodeHistBins * sizeof(uint32_t)));
+  if (g.nms_iou > 0.f) {
+    RS(dalloc(c, &c->dec_boxes, (size_t)g.max_boxes * sizeof(rtcc_box)));
+    RS(dalloc(c, &c->dec_n, sizeof(int)));
+    CK(cudaMemset(c->dec_n, 0, sizeof(int)));
+    RS(dalloc(c, &c->nms_mask, nms_mask_words(g.max_boxes) * sizeof(uint32_t)));
+    RS(dalloc(c, &c->nms_ticket, sizeof(unsigned)));
+    CK(cudaMemset(c->nms_ticket, 0, sizeof(unsigned)));
+  }
   c->det_bytes = sizeof(DetResultHeader) + (size_t)g.max_boxes * sizeof(rtcc_box);
   RS(halloc(c, &c->det_host, c->det_bytes));
   std::memset(c->det_host, 0, c->det_bytes);
@@ -1068,6 +1094,28 @@ rtcc_status rtcc_get_head(rtcc_ctx* c, float* host_out, size_t cap) {
   return RTCC_OK;
 }
 
+rtcc_status rtcc_get_decoded(rtcc_ctx* c, rtcc_box* host_out, int32_t cap, int32_t* n_out) {
+  if (!c || (!host_out && cap > 0) || cap < 0) return RTCC_E_ARG;
+  std::lock_guard<std::mutex> lk(c->mu);
+  CK(cudaStreamSynchronize(c->post));
+  int n = 0;
+  if (c->dec_boxes) {
+    CK(cudaMemcpy(&n, c->dec_n, sizeof(int), cudaMemcpyDeviceToHost));
+    n = std::max(0, std::min(n, c->cfg.max_boxes));
+    if (cap > 0 && n > 0)
+      CK(cudaMemcpy(host_out, c->dec_boxes, sizeof(rtcc_box) * (size_t)std::min(n, cap),
+                    cudaMemcpyDeviceToHost));
+  } else {
+    // without NMS the decode's boxes are the result block's
+    const DetResultHeader* hdr = reinterpret_cast<const DetResultHeader*>(c->det_host);
+    n = std::max(0, std::min(hdr->n_boxes, c->cfg.max_boxes));
+    if (cap > 0 && n > 0)
+      std::memcpy(host_out, hdr + 1, sizeof(rtcc_box) * (size_t)std::min(n, cap));
+  }
+  if (n_out) *n_out = n;
+  return RTCC_OK;
+}
+
 rtcc_status rtcc_get_pillars(rtcc_ctx* c, int32_t agent, int32_t* host_cell2pillar,
                              int32_t* host_pillar_cell, int32_t* host_count, int32_t* host_stats) {
   if (!c) return RTCC_E_ARG;
@@ -1163,7 +1211,56 @@ double rtcc_now_ms(void) { return now_ms(); }
 
 int32_t rtcc_kernels_per_frame(rtcc_ctx* c, int32_t n_present) {
   if (!c) return 0;
-  return n_present * (5 + 1) + 2;     // pillar chain + backbone per branch; fusion, decode
+  // pillar chain + backbone per branch; fusion, decode (and NMS)
+  return n_present * (5 + 1) + 2 + (c->dec_boxes ? 1 : 0);
+}
+
+rtcc_status rtcc_nms(const rtcc_box* host_in, int32_t n, float iou, rtcc_box* host_out,
+                     int32_t* n_out) {
+  if (n < 0 || n > kDecodeKeep || (n > 0 && (!host_in || !host_out)) || !n_out ||
+      !(iou >= 0.f && iou <= 1.f))
+    return RTCC_E_ARG;
+  const int mb = n > 0 ? n : 1;
+  // one scratch block: boxes in, count, ticket, error word, done word,
+  // result block (header + boxes), bitmask
+  const size_t in_b = (size_t)mb * sizeof(rtcc_box), res_b = sizeof(DetResultHeader) + in_b;
+  const size_t off_n = (in_b + 15) / 16 * 16, off_res = off_n + 64,
+               off_mask = off_res + (res_b + 15) / 16 * 16;
+  const size_t total = off_mask + nms_mask_words(mb) * sizeof(uint32_t);
+  uint8_t* d = nullptr;
+  if (cudaMalloc(&d, total) != cudaSuccess) return RTCC_E_NOMEM;
+  cudaStream_t st = nullptr;
+  rtcc_status r = RTCC_E_CUDA;
+  int* ints = reinterpret_cast<int*>(d + off_n);       // [0] n, [1] ticket, [2] err, [3] done
+  do {
+    if (cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking) != cudaSuccess) break;
+    if (cudaMemsetAsync(d + off_n, 0, 64, st) != cudaSuccess) break;
+    if (n > 0 && cudaMemcpyAsync(d, host_in, in_b, cudaMemcpyHostToDevice, st) != cudaSuccess) break;
+    if (cudaMemcpyAsync(ints, &n, sizeof(int), cudaMemcpyHostToDevice, st) != cudaSuccess) break;
+    NmsArgs a{};
+    a.in = reinterpret_cast<const rtcc_box*>(d);
+    a.n_in = ints;
+    a.ticket = reinterpret_cast<unsigned*>(ints + 1);
+    a.err = ints + 2;
+    a.done = ints + 3;
+    a.mask = reinterpret_cast<uint32_t*>(d + off_mask);
+    a.max_boxes = mb;
+    a.iou = iou;
+    a.out = d + off_res;
+    if (launch_nms(a, st) != cudaSuccess) break;
+    DetResultHeader h{};
+    if (cudaMemcpyAsync(&h, d + off_res, sizeof(h), cudaMemcpyDeviceToHost, st) != cudaSuccess) break;
+    if (cudaStreamSynchronize(st) != cudaSuccess) break;
+    const int k = std::max(0, std::min(h.n_boxes, n));
+    if (k > 0 && cudaMemcpy(host_out, d + off_res + sizeof(DetResultHeader), (size_t)k * sizeof(rtcc_box),
+                            cudaMemcpyDeviceToHost) != cudaSuccess)
+      break;
+    *n_out = k;
+    r = RTCC_OK;
+  } while (false);
+  if (st) cudaStreamDestroy(st);
+  cudaFree(d);
+  return r;
 }
 
 }  // extern "C"

@@ -1,6 +1,6 @@
 // Anchor decode, threshold and deterministic top-K of the head output (the
 // detection post-processing that ends the complete-detection latency, Sec.
-// V-A-3).  Rotated NMS is not part of this step.
+// V-A-3).  Rotated NMS, when enabled, follows in its own kernel (nms.cu).
 //
 // Order: class logit descending, then anchor index ascending; threshold on the
 // logit (score = sigmoid(logit) is monotone), so the selection is an exact
@@ -247,7 +247,8 @@ __device__ __forceinline__ void decode_box(unsigned long long v, const float* he
 __global__ void __launch_bounds__(kThreads, 1)
 k_decode_select(const uint32_t* keys, uint32_t* hist0, const float* head, int chunk4, int max_boxes,
                 AnchorGeo g, const int* err, DetResultHeader* __restrict__ hdr,
-                rtcc_box* __restrict__ boxes, int* present, int K, volatile int* __restrict__ done) {
+                rtcc_box* __restrict__ boxes, int* present, int K, volatile int* __restrict__ done,
+                int* dev_n) {
   extern __shared__ __align__(16) unsigned long long bnd[];  // [kBndCap] keys of bin b0
   __shared__ int hist[kThreads];                     // level-1/2 histograms (10 bits)
   __shared__ __align__(16) unsigned long long sel[kDecodeKeep];  // selected, unordered
@@ -288,8 +289,12 @@ k_decode_select(const uint32_t* keys, uint32_t* hist0, const float* head, int ch
     __syncthreads();
   }
   if (tid == 0) {
-    hdr->n_boxes = need;
-    hdr->err = *err;
+    if (dev_n) {                                        // NMS follows: it writes the header
+      *dev_n = need;
+    } else {
+      hdr->n_boxes = need;
+      hdr->err = *err;
+    }
   }
   if (need > 0) {
     const uint32_t b0 = static_cast<uint32_t>(s_bin);
@@ -459,7 +464,7 @@ k_decode_select(const uint32_t* keys, uint32_t* hist0, const float* head, int ch
       if (tid < need) decode_box(a[tid], head, g, sbox + tid);
     }
     // the boxes leave shared memory in 16-byte pieces (coalesced stores into
-    // the pinned host block)
+    // the pinned host block, or into device memory when NMS follows)
     __syncthreads();
     const int nbytes = need * (int)sizeof(rtcc_box);
     const uint4* src = reinterpret_cast<const uint4*>(sbox);
@@ -470,11 +475,14 @@ k_decode_select(const uint32_t* keys, uint32_t* hist0, const float* head, int ch
   }  // need > 0
 
   // the fusion kernel has read the presence flags: clear them for the next
-  // frame, then publish the result block to the host
+  // frame, then publish the result block to the host (unless NMS follows: its
+  // dependency wait makes this kernel's writes visible to it)
   if (tid < K) present[tid] = 0;
-  __threadfence_system();                          // this thread's box writes, system-wide
-  __syncthreads();
-  if (tid == 0) *done = 1;
+  if (!dev_n) {
+    __threadfence_system();                        // this thread's box writes, system-wide
+    __syncthreads();
+    if (tid == 0) *done = 1;
+  }
 }
 
 
@@ -486,7 +494,8 @@ cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t st) {
   const int n = a.feat_w * a.feat_h * a.anchors;
   if (a.max_boxes < 1 || a.max_boxes > kDecodeKeep) return cudaErrorInvalidValue;
   DetResultHeader* hdr = static_cast<DetResultHeader*>(a.out);
-  rtcc_box* boxes = reinterpret_cast<rtcc_box*>(hdr + 1);
+  rtcc_box* boxes = a.dev_boxes ? a.dev_boxes : reinterpret_cast<rtcc_box*>(hdr + 1);
+  if ((a.dev_boxes == nullptr) != (a.dev_n == nullptr)) return cudaErrorInvalidValue;
   AnchorGeo g;
   g.x_min = a.x_min;
   g.y_min = a.y_min;
@@ -506,7 +515,7 @@ cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t st) {
   if (!a.present || !a.done || a.K < 1 || a.K > RTCC_MAX_AGENTS) return cudaErrorInvalidValue;
   return launch_pdl(k_decode_select, dim3(1), dim3(kThreads), dyn, st, a.keys, a.hist0, a.head,
                     decode_key_chunk4(n), a.max_boxes, g, a.err, hdr, boxes, a.present, a.K,
-                    a.done);
+                    a.done, a.dev_n);
 }
 
 }  // namespace rtcc

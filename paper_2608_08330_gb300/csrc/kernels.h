@@ -230,6 +230,9 @@ struct DecodeArgs {
   int* present;              // device [K] per-agent presence flags: cleared for the next frame
   int K;
   volatile int* done;        // pinned host word: set to 1 once `out` is complete
+  rtcc_box* dev_boxes;       // non-null when NMS follows: the boxes and their count go
+  int* dev_n;                // to these device buffers instead, and neither `out` nor
+                             // `done` is written
 };
 constexpr int kDecodeKeep = 512;     // largest supported max_boxes
 constexpr int kDecodeHistBins = 4096;
@@ -239,11 +242,26 @@ inline size_t decode_key_capacity(int n_anchors) {
 }
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t st);
 
-// Result block the decode kernel writes into pinned host memory.
+// Result block the decode (or NMS) kernel writes into pinned host memory.
 struct DetResultHeader {
   int n_boxes;
   int err;
   int pad[2];
 };
+
+// Rotated BEV NMS of the decoded boxes (see nms.cu).
+struct NmsArgs {
+  const rtcc_box* in;        // device [max_boxes] decoded boxes in rank order
+  const int* n_in;           // device: their count
+  uint32_t* mask;            // device scratch, nms_mask_words(max_boxes) words
+  unsigned* ticket;          // device counter, 0 between launches
+  int max_boxes;
+  float iou;                 // suppress when IoU > iou, 0 <= iou <= 1
+  const int* err;            // device error word, copied into the result header
+  void* out;                 // pinned host result block DetResultHeader + rtcc_box[max_boxes]
+  volatile int* done;        // pinned host word: set to 1 once `out` is complete
+};
+size_t nms_mask_words(int max_boxes);
+cudaError_t launch_nms(const NmsArgs& a, cudaStream_t st);
 
 }  // namespace rtcc

@@ -43,7 +43,7 @@ class rtcc_model_config(C.Structure):
         ("block_stride", C.c_int32 * MAX_BLOCKS), ("up_stride", C.c_int32 * MAX_BLOCKS),
         ("up_ch", C.c_int32), ("fusion", C.c_int32), ("anchors", C.c_int32),
         ("dtype", C.c_int32), ("max_points", C.c_int32), ("max_boxes", C.c_int32),
-        ("cls_thresh", C.c_float), ("flags", C.c_int32),
+        ("cls_thresh", C.c_float), ("nms_iou", C.c_float), ("flags", C.c_int32),
     ]
 
 
@@ -110,6 +110,8 @@ def load(path: Optional[str] = None) -> C.CDLL:
         "rtcc_get_layer_spans": (S, [_ctx_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_int32,
                                      C.POINTER(C.c_int32)]),
         "rtcc_get_head": (S, [_ctx_p, C.c_void_p, C.c_size_t]),
+        "rtcc_get_decoded": (S, [_ctx_p, C.c_void_p, C.c_int32, C.POINTER(C.c_int32)]),
+        "rtcc_nms": (S, [C.c_void_p, C.c_int32, C.c_float, C.c_void_p, C.POINTER(C.c_int32)]),
         "rtcc_get_pillars": (S, [_ctx_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p,
                                  C.c_void_p]),
         "rtcc_get_tensor": (S, [_ctx_p, C.c_int32, C.c_int32, C.c_void_p, C.c_size_t,
@@ -161,7 +163,7 @@ def model_config(cfg, max_points: Optional[int] = None, flags: int = 0) -> rtcc_
     """Fill the C config from any object with the workload fields
     (n_agents, grid_w, grid_h, ranges, pillar, max_pillars, max_pts, pfn_ch,
     blocks = [(n_conv, channels, stride)], up_strides, up_ch, fusion, anchors,
-    dtype, max_boxes, cls_thresh)."""
+    dtype, max_boxes, cls_thresh; nms_iou, absent = 0, no NMS)."""
     c = rtcc_model_config()
     c.n_agents = cfg.n_agents
     c.grid_w, c.grid_h = cfg.grid_w, cfg.grid_h
@@ -181,6 +183,7 @@ def model_config(cfg, max_points: Optional[int] = None, flags: int = 0) -> rtcc_
     c.max_points = cfg.max_points_per_agent if max_points is None else max_points
     c.max_boxes = cfg.max_boxes
     c.cls_thresh = cfg.cls_thresh
+    c.nms_iou = float(getattr(cfg, "nms_iou", 0.0))
     c.flags = flags
     return c
 
@@ -294,6 +297,23 @@ def rtcc_get_head(ctx, feat_h: int, feat_w: int) -> np.ndarray:
     out = np.empty((feat_h, feat_w, 16), dtype=np.float32)
     _chk(load().rtcc_get_head(ctx, _ptr(out), out.size), "rtcc_get_head")
     return out
+
+
+def rtcc_get_decoded(ctx, cap: int = 512) -> np.ndarray:
+    """The decode's top-K boxes before NMS, in rank order."""
+    out = np.zeros(cap, dtype=BOX_DTYPE)
+    n = C.c_int32(0)
+    _chk(load().rtcc_get_decoded(ctx, _ptr(out), cap, C.byref(n)), "rtcc_get_decoded")
+    return out[:min(n.value, cap)]
+
+
+def rtcc_nms(boxes: np.ndarray, iou: float) -> np.ndarray:
+    """Rotated BEV NMS of boxes (BOX_DTYPE, rank order) on the GPU."""
+    b = np.ascontiguousarray(boxes, dtype=BOX_DTYPE)
+    out = np.zeros(max(len(b), 1), dtype=BOX_DTYPE)
+    n = C.c_int32(0)
+    _chk(load().rtcc_nms(_ptr(b) if len(b) else None, len(b), iou, _ptr(out), C.byref(n)), "rtcc_nms")
+    return out[:n.value]
 
 
 def rtcc_get_pillars(ctx, agent: int, grid_h: int, grid_w: int, max_pillars: int) -> dict:

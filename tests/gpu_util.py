@@ -6,6 +6,7 @@ import numpy as np
 
 import synth
 from oracle import forward as of
+from oracle import nms as onms
 from paper_2608_08330_gb300 import build as B
 from paper_2608_08330_gb300 import rtcc as R
 
@@ -112,3 +113,26 @@ def oracle_neck(blocks, weights, cfg, store):
 
 def head_to_oracle_layout(head_hwc):
     return np.asarray(head_hwc, dtype=np.float64).transpose(2, 0, 1)
+
+
+def check_nms(dec, out, thr, band=1e-4):
+    """Rotated NMS parity on the GPU's own input boxes: the output is a
+    subsequence of them copied bit for bit, and each keep/drop decision, taken
+    against the boxes the GPU kept before it, matches the oracle's float64 IoU
+    test -- except where that IoU lies within `band` of the threshold (the
+    kernel decides in float32).  Returns the kept positions."""
+    pos = {int(a): i for i, a in enumerate(dec["anchor"])}
+    assert len(pos) == len(dec), "anchors identify the boxes"
+    kept = [pos[int(a)] for a in out["anchor"]]
+    assert kept == sorted(kept) and len(set(kept)) == len(kept)
+    assert out.tobytes() == dec[kept].tobytes()
+    bev = np.stack([dec[f] for f in ("x", "y", "l", "w", "yaw")], axis=1).astype(np.float64)
+    ks = set(kept)
+    before = []
+    for i in range(len(dec)):
+        worst = max((onms.rotated_iou(bev[i], bev[j]) for j in before), default=-1.0)
+        if (worst > thr) == (i in ks):                  # the decisions differ
+            assert abs(worst - thr) < band, (i, worst, thr)
+        if i in ks:
+            before.append(i)
+    return kept

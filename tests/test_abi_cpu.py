@@ -59,6 +59,24 @@ def test_init_rejects_bad_config_without_touching_gpu(R):
     assert R.load().rtcc_init(None, w, 4, ctypes.byref(out)) == R.E_ARG
 
 
+def test_nms_arguments_are_checked_before_any_gpu_work(R):
+    import numpy as np
+    import synth
+    cfg = R.model_config(synth.get_config("tiny"))
+    out = ctypes.c_void_p()
+    wp = (ctypes.c_float * 4)()
+    for bad in (-0.1, 1.5, float("nan")):
+        cfg.nms_iou = bad
+        assert R.load().rtcc_init(ctypes.byref(cfg), wp, 4, ctypes.byref(out)) == R.E_ARG
+    box = np.zeros(4, dtype=R.BOX_DTYPE)
+    n = ctypes.c_int32(0)
+    lib = R.load()
+    assert lib.rtcc_nms(R._ptr(box), -1, 0.15, R._ptr(box), ctypes.byref(n)) == R.E_ARG
+    assert lib.rtcc_nms(R._ptr(box), 513, 0.15, R._ptr(box), ctypes.byref(n)) == R.E_ARG
+    assert lib.rtcc_nms(R._ptr(box), 4, float("nan"), R._ptr(box), ctypes.byref(n)) == R.E_ARG
+    assert lib.rtcc_nms(None, 4, 0.15, R._ptr(box), ctypes.byref(n)) == R.E_ARG
+
+
 def test_rtcc_releases_on_completion_in_event_order(R):
     c = R.rtcc_ctrl_create(3, 100)
     assert R.rtcc_ctrl_begin(c, 1, 0.0) == R.OK

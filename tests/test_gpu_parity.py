@@ -95,11 +95,22 @@ def _check_frame(R, ctx, cfg, w, pts, absent=()):
     return hd_g
 
 
-def _check_decode(cfg, hd_g, boxes):
+_BOX_FIELDS = ("x", "y", "z", "l", "w", "h", "yaw", "score")
+
+
+def _check_decode(cfg, hd_g, boxes, R=None, ctx=None):
+    """The decode's selection and order exact given the GPU head, its boxes
+    within tolerance; with NMS, the decoded list comes from the read-back and
+    the result must be its NMS (see gpu_util.check_nms)."""
     det = of.decode(hd_g, cfg)
-    assert boxes["anchor"].tolist() == det["idx"].tolist()      # exact selection + order
-    got = np.stack([boxes[f] for f in ("x", "y", "z", "l", "w", "h", "yaw", "score")], axis=1)
+    nms_on = getattr(cfg, "nms_iou", 0.0) > 0
+    dec = R.rtcc_get_decoded(ctx) if nms_on else boxes
+    assert dec["anchor"].tolist() == det["idx"].tolist()        # exact selection + order
+    got = np.stack([dec[f] for f in _BOX_FIELDS], axis=1)
     U.assert_close(got, det["boxes"], "boxes")
+    if nms_on:
+        U.check_nms(dec, boxes, cfg.nms_iou)
+        assert 0 < len(boxes) <= len(dec) or len(dec) == 0
 
 
 def _end_to_end(R, cfg, frame=0, absent=(), flags=None, arrivals=None):
@@ -109,7 +120,7 @@ def _end_to_end(R, cfg, frame=0, absent=(), flags=None, arrivals=None):
         a = synth.arrivals_for(cfg, frame) if arrivals is None else arrivals
         boxes = U.run_frame(ctx, cfg, pts, a, R.MODE_RTCC, absent=absent)
         hd_g = _check_frame(R, ctx, cfg, w, pts, absent=absent)
-        _check_decode(cfg, hd_g, boxes)
+        _check_decode(cfg, hd_g, boxes, R, ctx)
         # whole-path parity: the oracle forward from the points
         full = of.forward([None if k in absent else pts[k] for k in range(cfg.n_agents)], w, cfg,
                           store=cfg.dtype)
@@ -178,7 +189,7 @@ def test_decode_all_equal_logits(R, grid):
     # then decided by anchor index alone (ties), and at 256x256 the threshold
     # bin holds 16384 keys, more than the decode's shared-memory list takes
     # (its radix-select fallback); at 96x64 it holds 1536 (the list path).
-    cfg = dataclasses.replace(_small_pp(grid=grid), cls_thresh=-1.0)
+    cfg = dataclasses.replace(_small_pp(grid=grid), cls_thresh=-1.0, nms_iou=0.0)
     w = dict(synth.weights_for(cfg))
     w["head.w"] = np.zeros_like(w["head.w"])
     ctx = R.rtcc_init(R.model_config(cfg, flags=U.DEBUG_FLAGS), synth.weight_blob(w))
@@ -187,7 +198,7 @@ def test_decode_all_equal_logits(R, grid):
         boxes = U.run_frame(ctx, cfg, pts, [0.0] * cfg.n_agents, R.MODE_RTCC)
         hd = U.head_to_oracle_layout(R.rtcc_get_head(ctx, cfg.feat_h, cfg.feat_w))
         assert len(boxes) == cfg.max_boxes
-        _check_decode(cfg, hd, boxes)
+        _check_decode(cfg, hd, boxes, R, ctx)
     finally:
         R.rtcc_destroy(ctx)
 
@@ -218,7 +229,7 @@ def test_decode_level1_list_path(R):
     # but spread over its next 10 bits: more candidates than the decode's
     # threads, so it takes the level-1 histogram and warp-sort path instead of
     # ranking by counting (which the other workloads take).
-    cfg = dataclasses.replace(_small_pp(grid=(96, 64)), cls_thresh=-1.0, max_boxes=500)
+    cfg = dataclasses.replace(_small_pp(grid=(96, 64)), cls_thresh=-1.0, max_boxes=500, nms_iou=0.0)
     w = dict(synth.weights_for(cfg))
     pts = [synth.points_for(cfg, 0, k) for k in range(cfg.n_agents)]
     F = of.forward(pts, w, cfg, store=cfg.dtype)["fused"]
@@ -235,7 +246,7 @@ def test_decode_level1_list_path(R):
         below0, nb0, nb1 = _decode_path_sizes(hd, cfg.cls_thresh, cfg.max_boxes)
         assert below0 + nb0 > 1024 and nb0 <= 4096 and nb1 <= 64, (below0, nb0, nb1)
         assert len(boxes) == cfg.max_boxes
-        _check_decode(cfg, hd, boxes)
+        _check_decode(cfg, hd, boxes, R, ctx)
     finally:
         R.rtcc_destroy(ctx)
 
@@ -317,7 +328,7 @@ def test_abort_is_infeasible_and_next_frame_clean(R):
     assert R.rtcc_wait_detection(ctx, 100)[0] == R.E_INFEASIBLE
     boxes = U.run_frame(ctx, cfg, pts, [0.0, 5.0], R.MODE_RTCC, frame_id=2)
     hd = _check_frame(R, ctx, cfg, w, pts)
-    _check_decode(cfg, hd, boxes)
+    _check_decode(cfg, hd, boxes, R, ctx)
     R.rtcc_destroy(ctx)
 
 
