@@ -722,6 +722,9 @@ rtcc_status init_impl(rtcc_ctx* c, const float* weights) {
     RS(dalloc(c, &c->dec_n, sizeof(int)));
     CK(cudaMemset(c->dec_n, 0, sizeof(int)));
     RS(dalloc(c, &c->nms_mask, nms_mask_words(g.max_boxes) * sizeof(uint32_t)));
+    // all ones: a word the kernel read without writing it this frame would
+    // suppress boxes (and show in the parity tests) instead of passing as 0
+    CK(cudaMemset(c->nms_mask, 0xFF, nms_mask_words(g.max_boxes) * sizeof(uint32_t)));
     RS(dalloc(c, &c->nms_ticket, sizeof(unsigned)));
     CK(cudaMemset(c->nms_ticket, 0, sizeof(unsigned)));
   }
@@ -1235,6 +1238,8 @@ rtcc_status rtcc_nms(const rtcc_box* host_in, int32_t n, float iou, rtcc_box* ho
   do {
     if (cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking) != cudaSuccess) break;
     if (cudaMemsetAsync(d + off_n, 0, 64, st) != cudaSuccess) break;
+    // bitmask scratch all ones (see the context's allocation)
+    if (cudaMemsetAsync(d + off_mask, 0xFF, nms_mask_words(mb) * sizeof(uint32_t), st) != cudaSuccess) break;
     if (n > 0 && cudaMemcpyAsync(d, host_in, in_b, cudaMemcpyHostToDevice, st) != cudaSuccess) break;
     if (cudaMemcpyAsync(ints, &n, sizeof(int), cudaMemcpyHostToDevice, st) != cudaSuccess) break;
     NmsArgs a{};
