@@ -466,10 +466,124 @@ def run_ours(args):
                           "tflops_span": round(flops / (span_us * 1e-6) / 1e12, 1),
                           "rows": rows}
         line["other_configs"] = other_configs(R)
+        line["gain_validation"] = gain_validation(R, cfg, w, frames, flush)
         print(json.dumps(line, default=_json_num), flush=True)
     if dist is not None:
         dist.destroy_process_group()
     return 0
+
+
+def predicted_gain(a, c_enc, c_post):
+    """T_B - T_R of one arrival trace on the single-stream timeline of the
+    paper's execution model (Eqs. 20-22): RTCC starts each encoder at
+    max(a_k, the previous encoder's finish) in (a_k, k) order, Barrier starts
+    them back to back at A = max a in index order, and the post-join follows
+    the last encoder in both.  (Equal to the pre-arrival encoder work W_pre.)"""
+    K = len(a)
+    g = 0.0
+    for k in sorted(range(K), key=lambda k: (a[k], k)):
+        g = max(a[k], g) + c_enc[k]
+    t_r = g + c_post
+    t_b = max(a) + sum(c_enc) + c_post
+    return t_b - t_r
+
+
+def gain_validation(R, cfg, w, frames, flush, pairs=35, seed=7):
+    """Predicted vs measured gain on resident inputs (Sec. V-C, the 35 paired
+    resident-input runs; and the release fidelity of Sec. V-E).
+
+    Service times: each branch's span and the post-join span, from event
+    nodes in the graphs of a timeline context (medians over frames whose
+    arrivals are 2 ms apart, so branches run alone).  Then `pairs` seeded
+    traces with arrivals U[0, S], S = K x the median branch span (so the
+    pre-arrival overlap varies from trace to trace), each run in RTCC and in
+    Barrier mode on an uninstrumented context; measured gain = Barrier tail -
+    RTCC tail.  Lateness = host time a branch's graph was launched minus the
+    host time of its modelled release: the call that completed its payload
+    (RTCC), or the call that completed the last payload (Barrier).  The
+    controller's decision cost is the host time of one rtcc_ctrl_complete
+    through the binding (an upper bound: it includes the ctypes call)."""
+    import torch
+    K = cfg.n_agents
+    blob = synth.weight_blob(w)
+
+    def frame(c, mode, a, fid):
+        pts = frames[fid % len(frames)]
+        flush.zero_()
+        torch.cuda.synchronize()
+        for k in range(K):
+            assert R.rtcc_stage_resident(c, k, pts[k]) == R.OK
+        assert R.rtcc_set_mode(c, mode) == R.OK
+        assert R.rtcc_frame_begin(c, 50000 + fid, 0.0) == R.OK
+        t0 = R.rtcc_now_ms() + 0.5
+        t_call = [0.0] * K
+        for k in sorted(range(K), key=lambda k: (a[k], k)):
+            while R.rtcc_now_ms() < t0 + a[k]:
+                pass
+            t_call[k] = R.rtcc_now_ms()
+            assert R.rtcc_payload_resident(c, k, float(a[k])) == R.OK
+        s, _, _ = R.rtcc_wait_detection(c, 10000)
+        assert s == R.OK
+        info = R.rtcc_get_frame_info(c)
+        last = max(range(K), key=lambda k: (a[k], k))
+        late = [info.t_release_ms[k] - (t_call[k] if mode == R.MODE_RTCC else t_call[last])
+                for k in range(K)]
+        return (info.t_ready_ms - info.t_last_event_ms, [info.gpu_branch_ms[k] for k in range(K)],
+                info.gpu_post_ms, late)
+
+    tctx = R.rtcc_init(R.model_config(cfg, flags=R.FLAG_TIMELINE), blob)
+    spans, posts = [], []
+    for f in range(6):
+        _, br, po, _ = frame(tctx, R.MODE_RTCC, [2.0 * k for k in range(K)], f)
+        if f >= 2:
+            spans.append(br)
+            posts.append(po)
+    R.rtcc_destroy(tctx)
+    c_enc = [float(x) for x in np.median(np.array(spans), axis=0)]
+    c_post = float(np.median(posts))
+    spread = K * float(np.median(c_enc))
+
+    ctx = R.rtcc_init(R.model_config(cfg, flags=0), blob)
+    rng = np.random.default_rng(seed)
+    for f in range(3):                                   # warm-up
+        frame(ctx, R.MODE_RTCC, [0.0] * K, f)
+    pred, meas, late_r, late_b = [], [], [], []
+    for p in range(pairs):
+        a = [float(x) for x in rng.uniform(0.0, spread, size=K)]
+        modes = (R.MODE_RTCC, R.MODE_BARRIER) if p % 2 == 0 else (R.MODE_BARRIER, R.MODE_RTCC)
+        tail = {}
+        for m in modes:
+            tail[m], _, _, late = frame(ctx, m, a, p)
+            (late_r if m == R.MODE_RTCC else late_b).extend(late)
+        meas.append(tail[R.MODE_BARRIER] - tail[R.MODE_RTCC])
+        pred.append(predicted_gain(a, c_enc, c_post))
+    R.rtcc_destroy(ctx)
+
+    cc = R.rtcc_ctrl_create(6, 1000)
+    dec = []
+    for f in range(200):
+        R.rtcc_ctrl_begin(cc, f + 1, 0.0)
+        for k in range(6):
+            t = time.perf_counter()
+            R.rtcc_ctrl_complete(cc, k, True, 10, float(k))
+            dec.append((time.perf_counter() - t) * 1e6)
+        for k in range(6):
+            R.rtcc_ctrl_mark(cc, k, R.RUNNING)
+            R.rtcc_ctrl_mark(cc, k, R.FINISHED)
+        R.rtcc_ctrl_end(cc)
+    R.rtcc_ctrl_destroy(cc)
+
+    pred_a, meas_a = np.array(pred), np.array(meas)
+    r = float(np.corrcoef(pred_a, meas_a)[0, 1]) if pred_a.std() > 0 and meas_a.std() > 0 else None
+    return {"pairs": pairs, "arrivals": f"U[0, {spread:.3f}] ms (K x median branch span), seed {seed}",
+            "c_enc_ms": [round(x, 4) for x in c_enc], "c_post_ms": round(c_post, 4),
+            "r": r, "mae_ms": float(np.mean(np.abs(pred_a - meas_a))),
+            "mean_predicted_ms": float(pred_a.mean()), "mean_measured_ms": float(meas_a.mean()),
+            "measured_positive": int((meas_a > 0).sum()),
+            "lateness_us": {"rtcc_p50": pct(late_r, 50) * 1e3, "rtcc_p95": pct(late_r, 95) * 1e3,
+                            "barrier_p50": pct(late_b, 50) * 1e3,
+                            "barrier_p95": pct(late_b, 95) * 1e3},
+            "ctrl_decision_us_p50": pct(dec, 50)}
 
 
 def other_configs(R, frames=10, warm=3, gap_cap_ms=2.0):
