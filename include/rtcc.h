@@ -157,6 +157,10 @@ typedef struct {
   float gpu_post_ms;                /* whole post-join graph                  */
   int32_t dispatch_order[RTCC_MAX_AGENTS];  /* agents in launch order, -1 pad */
   int32_t n_dispatched;
+  float gpu_fusion_kernel_ms;       /* the fusion+head kernel's own span on the
+                                       GPU global timer (block 0 past its
+                                       dependency wait to the last block's
+                                       end); -1 without RTCC_FLAG_TIMELINE    */
 } rtcc_frame_info;
 
 /* ------------------------------------------------------------------------ */

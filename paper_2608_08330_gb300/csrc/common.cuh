@@ -198,6 +198,23 @@ __device__ __forceinline__ unsigned long long global_ns() {
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
   return t;
 }
+// Span of a multi-block kernel on the global timer, when `span` is not null:
+// span[0] = when block 0 passed its dependency wait, span[1] = when the last
+// block finished, span[2] = a finish counter that is 0 between launches.
+// span_begin after the wait; span_end by every block once all its threads
+// are done (after a block barrier).
+__device__ __forceinline__ void span_begin(unsigned long long* span) {
+  if (span && blockIdx.x == 0 && threadIdx.x == 0) span[0] = global_ns();
+}
+__device__ __forceinline__ void span_end(unsigned long long* span) {
+  if (span && threadIdx.x == 0) {
+    __threadfence();
+    if (atomicAdd(span + 2, 1ull) == (unsigned long long)(gridDim.x - 1)) {
+      span[1] = global_ns();
+      span[2] = 0ull;
+    }
+  }
+}
 // Make this thread's generic-proxy shared-memory writes visible to the async
 // proxy (TMA, tcgen05) before a barrier hands the buffer over.
 __device__ __forceinline__ void fence_async_smem() {

@@ -95,6 +95,7 @@ struct rtcc_ctx {
   int* dec_n = nullptr;               //         and their count
   uint32_t* nms_mask = nullptr;       //         suppression bitmask scratch
   unsigned* nms_ticket = nullptr;     //         last-block counter
+  unsigned long long* fuse_span = nullptr;   // RTCC_FLAG_TIMELINE: fusion kernel span stamps [3]
   uint8_t* det_host = nullptr;        // pinned; the decode (or NMS) kernel writes it directly
   size_t det_bytes = 0;
   volatile int* h_done = nullptr;     // pinned; the decode kernel sets it to 1 when det_host is complete
@@ -591,6 +592,7 @@ rtcc_status capture_post(rtcc_ctx* c) {
   fa.hist0 = c->hist0;
   fa.cls_thresh = c->cfg.cls_thresh;
   fa.anchors = c->cfg.anchors;
+  fa.span = c->fuse_span;
   // max fusion: tensor-core kernel (TMA-staged agent tiles, max in shared
   // memory, head as an N = 16 MMA); attention fusion: CUDA-core kernel
   const int bkc = fuse_tc_chunk(c->Cf, c->K);
@@ -616,6 +618,7 @@ rtcc_status capture_post(rtcc_ctx* c) {
     tp.cls_thresh = c->cfg.cls_thresh;
     tp.anchors = c->cfg.anchors;
     tp.err = c->d_err;
+    tp.span = c->fuse_span;
   }
   DecodeArgs da{};
   da.head = c->head_out;
@@ -701,6 +704,10 @@ rtcc_status init_impl(rtcc_ctx* c, const float* weights) {
   const rtcc_model_config& g = c->cfg;
   RS(upload_weights(c, weights));
   RS(dalloc(c, &c->d_err, 16));
+  if (g.flags & RTCC_FLAG_TIMELINE) {
+    RS(dalloc(c, &c->fuse_span, 3 * sizeof(unsigned long long)));
+    CK(cudaMemset(c->fuse_span, 0, 3 * sizeof(unsigned long long)));
+  }
   CK(cudaMemset(c->d_err, 0, 16));
   RS(dalloc(c, &c->d_present, RTCC_MAX_AGENTS * 4));
   CK(cudaMemset(c->d_present, 0, RTCC_MAX_AGENTS * 4));
@@ -917,6 +924,7 @@ rtcc_status rtcc_frame_begin(rtcc_ctx* c, uint64_t frame_id, double t0_ms) {
   }
   c->info.gpu_fusion_ms = -1.f;
   c->info.gpu_post_ms = -1.f;
+  c->info.gpu_fusion_kernel_ms = -1.f;
   return RTCC_OK;
 }
 
@@ -1022,6 +1030,10 @@ rtcc_status rtcc_wait_detection(rtcc_ctx* c, int32_t timeout_ms, rtcc_box* out, 
     float ms = -1.f;
     if (cudaEventElapsedTime(&ms, c->ev_fuse0, c->ev_fuse1) == cudaSuccess) c->info.gpu_fusion_ms = ms;
     if (cudaEventElapsedTime(&ms, c->ev_post0, c->ev_post1) == cudaSuccess) c->info.gpu_post_ms = ms;
+    unsigned long long sp[2] = {0ull, 0ull};
+    if (c->fuse_span && cudaMemcpy(sp, c->fuse_span, sizeof(sp), cudaMemcpyDeviceToHost) == cudaSuccess &&
+        sp[1] > sp[0])
+      c->info.gpu_fusion_kernel_ms = (float)((double)(sp[1] - sp[0]) * 1e-6);
     (void)cudaGetLastError();
   }
   c->ctrl.end();

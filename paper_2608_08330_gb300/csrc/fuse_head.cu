@@ -179,7 +179,7 @@ k_fuse_head(const void* const* __restrict__ feats, const int* present, int K,
             int cells, float inv_sqrt_c, const float* __restrict__ head_wp,
             const float* __restrict__ head_b, float* __restrict__ head_out, T* __restrict__ fused,
             uint32_t* __restrict__ keys, uint32_t* __restrict__ hist0, float cls_thresh,
-            int anchors) {
+            int anchors, unsigned long long* span) {
   constexpr int CPL = Lanes<C>::CPL;
   constexpr int NC = Group<C, ATTN>::NC;
   extern __shared__ float sw[];               // [16][CPL][32] permuted head weights
@@ -187,6 +187,7 @@ k_fuse_head(const void* const* __restrict__ feats, const int* present, int K,
   pdl_trigger();
   for (int i = threadIdx.x; i < kHeadOut * C; i += blockDim.x) sw[i] = head_wp[i];  // constant
   pdl_wait();
+  span_begin(span);
   if (threadIdx.x < RTCC_MAX_AGENTS)
     slot[threadIdx.x] = threadIdx.x < K ? static_cast<const T*>(feats[threadIdx.x]) : nullptr;
   __syncthreads();
@@ -262,6 +263,10 @@ k_fuse_head(const void* const* __restrict__ feats, const int* present, int K,
       if (keep && lane == __ffs(peers) - 1) atomicAdd(&hist0[bin], (uint32_t)__popc(peers));
     }
   }
+  if (span) {
+    __syncthreads();
+    span_end(span);
+  }
 }
 
 template <typename T, int C>
@@ -282,7 +287,7 @@ cudaError_t launch_c(const FuseArgs& a, cudaStream_t st) {
     cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   return launch_pdl(kern, dim3(blocks), dim3(kThreads), smem, st, a.feats, a.present, a.K,
                     a.cells, isc, a.head_wp, a.head_b, a.head_out, fused, a.keys, a.hist0,
-                    a.cls_thresh, a.anchors);
+                    a.cls_thresh, a.anchors, a.span);
 }
 
 template <typename T>

@@ -170,6 +170,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fuse_max_head(const __grid_cons
       tma_load_2d(wsm + j * kFuseHeadOut * bkc * 2, &P.wmap, wbar, j * bkc, 0);
   }
   pdl_wait();                                  // the slots are the branches' output
+  span_begin(P.span);
   if (threadIdx.x == 0) {
     int n = 0;
     for (int k = 0; k < P.K; ++k)
@@ -315,6 +316,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fuse_max_head(const __grid_cons
 
   tc_fence_before();
   __syncthreads();
+  span_end(P.span);
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem, 32);

@@ -182,6 +182,7 @@ struct FuseArgs {
   uint32_t* hist0;           // device [4096] histogram of the keys' top 12 bits
   float cls_thresh;
   int anchors;
+  unsigned long long* span;  // device [3] kernel span stamps (see span_begin), or null
 };
 cudaError_t launch_fuse_head(const FuseArgs& a, bool bf16, cudaStream_t st);
 
@@ -200,6 +201,7 @@ struct FuseTcParams {
   float cls_thresh;
   int anchors;
   int* err;                           // device error word
+  unsigned long long* span;           // device [3] kernel span stamps, or null
 };
 // Channel chunk (64 or 32) the kernel stages for C channels and K agent slots,
 // 0 if it cannot run that shape.

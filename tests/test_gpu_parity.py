@@ -136,6 +136,8 @@ def test_tiny_end_to_end(R):
     ctx, *_ = _end_to_end(R, cfg)
     info = R.rtcc_get_frame_info(ctx)
     assert info.n_dispatched == 2 and info.gpu_backbone_ms[0] > 0 and info.gpu_fusion_ms > 0
+    # the fusion kernel's own global-timer span sits inside its event-node span
+    assert 0 < info.gpu_fusion_kernel_ms <= info.gpu_fusion_ms + 1e-3
     R.rtcc_destroy(ctx)
 
 
