@@ -108,6 +108,16 @@ def fusion_bytes(cfg, k_present: int) -> float:
     return float(k_present * cells * cfg.feat_ch * 2 + cells * 16 * 4)
 
 
+def pfn_bytes(cfg, n_pillars: int, n_kept: int, n_raw: int) -> float:
+    """Bytes the PFN kernel itself moves for one branch: the kept points'
+    16-byte records (gathered), the raw point indices of the kept pillars'
+    lists, three per-pillar words (count, offset, cell), and per pillar its
+    C_p 16-bit channels into the pseudo-image plus two words (cell2pillar,
+    kept count).  The rest of the dense pseudo-image keeps its zeros: the
+    first pillar kernel clears only the previous pass's cells."""
+    return float(n_kept * 16 + n_raw * 4 + n_pillars * (12 + cfg.pfn_ch * 2 + 8))
+
+
 def _json_num(o):
     """numpy scalars in the JSON line become plain numbers."""
     return o.item() if hasattr(o, "item") else str(o)
@@ -326,6 +336,7 @@ def run_ours(args):
         return {"tail": info.t_ready_ms - info.t_last_event_ms,
                 "bb": [info.gpu_backbone_ms[k] for k in range(K)],
                 "fuse": info.gpu_fusion_ms, "fusek": info.gpu_fusion_kernel_ms,
+                "pfnk": [info.gpu_pfn_kernel_ms[k] for k in range(K)],
                 "post": info.gpu_post_ms,
                 "branch": [info.gpu_branch_ms[k] for k in range(K)], "n_boxes": len(boxes)}
 
@@ -335,7 +346,13 @@ def run_ours(args):
         for resident in (True, False):
             for mode in modes:
                 out.append((mode, resident, one_frame(step, mode, resident)))
-        out.append(("timeline", True, one_frame(step, R.MODE_RTCC, True, tctx)))
+        r = one_frame(step, R.MODE_RTCC, True, tctx)
+        r["pfn_bytes"] = []
+        for k in range(K):                        # read back after the frame (host sync)
+            gp = R.rtcc_get_pillars(tctx, k, cfg.grid_h, cfg.grid_w, cfg.max_pillars)
+            raw = gp["n_kept"] + gp["drop_ncap"]          # list entries the kernel reads
+            r["pfn_bytes"].append(pfn_bytes(cfg, gp["n_pillars"], gp["n_kept"], raw))
+        out.append(("timeline", True, r))
         return out
 
     for s in range(args.warmup):
@@ -369,6 +386,8 @@ def run_ours(args):
     bb = [x for (m, res, r) in rec if m == "timeline" for x in r["bb"] if x > 0]
     fu = [r["fuse"] for (m, res, r) in rec if m == "timeline" and r["fuse"] > 0]
     fk = [r["fusek"] for (m, res, r) in rec if m == "timeline" and r["fusek"] > 0]
+    pf = [(b, t) for (m, res, r) in rec if m == "timeline" for b, t in zip(r["pfn_bytes"], r["pfnk"])
+          if t > 0]
     value = pct(r_res, 50)
     if dist is not None:
         t = torch.tensor([value, wall_ms], device="cuda", dtype=torch.float64)
@@ -382,6 +401,9 @@ def run_ours(args):
     fu_ms = float(np.mean(fu)) if fu else None
     fu_ev_gbs = fusion_bytes(cfg, K) / (fu_ms * 1e-3) / 1e9 if fu_ms else None
     fk_ms = float(np.mean(fk)) if fk else None
+    pfn_ms = float(np.mean([t for _, t in pf])) if pf else None
+    pfn_mb = float(np.mean([b for b, _ in pf])) / 1e6 if pf else None
+    pfn_gbs = float(np.mean([b / (t * 1e-3) / 1e9 for b, t in pf])) if pf else None
     fu_gbs = fusion_bytes(cfg, K) / (fk_ms * 1e-3) / 1e9 if fk_ms else None
     n_launch = R.rtcc_kernels_per_frame(ctx, K) * 5 * args.steps
     h2d = sum(int(p.shape[0]) * 16 + 16 for p in frames[0])
@@ -411,6 +433,13 @@ def run_ours(args):
                              "dependency wait to the last block's end (the slots are read from "
                              "L2, written by the branches just before)",
                    "ms_event_nodes": fu_ms, "gbs_event_nodes": fu_ev_gbs},
+        "pfn": {"gbs": pfn_gbs, "frac_of_hbm": (pfn_gbs / hbm) if pfn_gbs else None, "ms": pfn_ms,
+                "mb_per_launch": pfn_mb,
+                "timing": "the PFN kernel's own span on the GPU global timer, per branch",
+                "bytes": "moved by the kernel: gathered kept points, the pillars' index lists "
+                         "and words, and the occupied cells of the pseudo-image (the dense "
+                         "image's zeros are not rewritten; the dense write would be "
+                         f"{2 * cfg.pfn_ch * cfg.grid_w * cfg.grid_h / 1e6:.2f} MB)"},
         "roofline": {"kernel": "k_backbone (persistent tcgen05 implicit-GEMM backbone of one "
                                "branch: 13 convs + 3 deconvs in one launch)",
                      "bound": "tensor", "achieved": enc_tflops, "peak": tflops_peak,

@@ -161,6 +161,8 @@ typedef struct {
                                        GPU global timer (block 0 past its
                                        dependency wait to the last block's
                                        end); -1 without RTCC_FLAG_TIMELINE    */
+  float gpu_pfn_kernel_ms[RTCC_MAX_AGENTS];  /* each branch's PFN kernel span, the
+                                                same way; -1 without the flag  */
 } rtcc_frame_info;
 
 /* ------------------------------------------------------------------------ */

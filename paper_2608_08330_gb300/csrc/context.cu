@@ -375,6 +375,10 @@ rtcc_status build_branch(rtcc_ctx* c, int k) {
   CK(cudaMemset(p.np_prev, 0, 4));
   p.clear_all = 0;                              // image and cell2pillar start cleared below
   p.present_flag = c->d_present + k;
+  if (g.flags & RTCC_FLAG_TIMELINE) {
+    RS(dalloc(c, &p.pfn_span, 3 * sizeof(unsigned long long)));
+    CK(cudaMemset(p.pfn_span, 0, 3 * sizeof(unsigned long long)));
+  }
   RS(dalloc(c, &p.pillar_cell, (size_t)c->P * 4));
   RS(dalloc(c, &p.pcount, (size_t)c->P * 4));
   // words cleared at the start of every branch graph (one memset): the pillar
@@ -925,6 +929,7 @@ rtcc_status rtcc_frame_begin(rtcc_ctx* c, uint64_t frame_id, double t0_ms) {
   c->info.gpu_fusion_ms = -1.f;
   c->info.gpu_post_ms = -1.f;
   c->info.gpu_fusion_kernel_ms = -1.f;
+  for (int k = 0; k < RTCC_MAX_AGENTS; ++k) c->info.gpu_pfn_kernel_ms[k] = -1.f;
   return RTCC_OK;
 }
 
@@ -1026,6 +1031,10 @@ rtcc_status rtcc_wait_detection(rtcc_ctx* c, int32_t timeout_ms, rtcc_box* out, 
       float ms = -1.f;
       if (cudaEventElapsedTime(&ms, b.ev_bb0, b.ev_bb1) == cudaSuccess) c->info.gpu_backbone_ms[k] = ms;
       if (cudaEventElapsedTime(&ms, b.ev_start, b.ev_end) == cudaSuccess) c->info.gpu_branch_ms[k] = ms;
+      unsigned long long ps[2] = {0ull, 0ull};
+      if (b.pb.pfn_span && cudaMemcpy(ps, b.pb.pfn_span, sizeof(ps), cudaMemcpyDeviceToHost) == cudaSuccess &&
+          ps[1] > ps[0])
+        c->info.gpu_pfn_kernel_ms[k] = (float)((double)(ps[1] - ps[0]) * 1e-6);
     }
     float ms = -1.f;
     if (cudaEventElapsedTime(&ms, c->ev_fuse0, c->ev_fuse1) == cudaSuccess) c->info.gpu_fusion_ms = ms;

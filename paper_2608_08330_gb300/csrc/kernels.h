@@ -63,6 +63,7 @@ struct PillarBufs {
   int* cell2pillar;      // [H*W]     -1 where no kept pillar
   void* image;           // [H][W][C] storage type, zeros where no kept pillar
   int* present_flag;     // optional: set to 1 by the pass (the agent's slot is filled)
+  unsigned long long* pfn_span;   // optional [3]: the PFN kernel's span stamps (span_begin)
   // optional zero-copy payload: the first kernel reads the header and points
   // from src_* (e.g. pinned host memory) and writes them to dst_* (= n_hdr,
   // pts) for the later kernels

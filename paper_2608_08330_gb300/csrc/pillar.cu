@@ -345,12 +345,13 @@ k_pfn(const float4* pts, const int* stats_in,
       const int* list, const int* pillar_cell,
       const float* __restrict__ w, const float* __restrict__ b, GridGeom g, int N,
       T* image, int* cell2pillar, int* np_prev,
-      int* pcount) {
+      int* pcount, unsigned long long* span) {
   __shared__ float sw[C * 9];
   __shared__ float sb[C];
   pdl_trigger();
   for (int j = threadIdx.x; j < C * 9; j += blockDim.x) sw[j] = w[j];   // weights: constant
   pdl_wait();
+  span_begin(span);
   for (int j = threadIdx.x; j < C; j += blockDim.x) sb[j] = b[j];
   __syncthreads();
   const int lane = threadIdx.x & 31;
@@ -437,6 +438,10 @@ k_pfn(const float4* pts, const int* stats_in,
       pcount[p] = m;
     }
   }
+  if (span) {
+    __syncthreads();
+    span_end(span);
+  }
 }
 
 template <typename T, int C>
@@ -463,7 +468,7 @@ cudaError_t launch_all(const PillarBufs& b, const GridGeom& g, const float* pfn_
   if (e != cudaSuccess) return e;
   e = launch_pdl(k_pfn<T, C>, dim3((b.P + 7) / 8), dim3(256), 0, st, b.pts, b.stats, b.pcnt_raw,
                  b.poff, b.list, b.pillar_cell, pfn_w, pfn_b, g, b.N, static_cast<T*>(b.image),
-                 b.cell2pillar, b.np_prev, b.pcount);
+                 b.cell2pillar, b.np_prev, b.pcount, b.pfn_span);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }

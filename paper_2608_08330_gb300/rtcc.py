@@ -60,7 +60,7 @@ class rtcc_frame_info(C.Structure):
         ("gpu_backbone_ms", C.c_float * MAX_AGENTS), ("gpu_branch_ms", C.c_float * MAX_AGENTS),
         ("gpu_fusion_ms", C.c_float), ("gpu_post_ms", C.c_float),
         ("dispatch_order", C.c_int32 * MAX_AGENTS), ("n_dispatched", C.c_int32),
-        ("gpu_fusion_kernel_ms", C.c_float),
+        ("gpu_fusion_kernel_ms", C.c_float), ("gpu_pfn_kernel_ms", C.c_float * MAX_AGENTS),
     ]
 
 

@@ -138,6 +138,7 @@ def test_tiny_end_to_end(R):
     assert info.n_dispatched == 2 and info.gpu_backbone_ms[0] > 0 and info.gpu_fusion_ms > 0
     # the fusion kernel's own global-timer span sits inside its event-node span
     assert 0 < info.gpu_fusion_kernel_ms <= info.gpu_fusion_ms + 1e-3
+    assert all(0 < info.gpu_pfn_kernel_ms[k] < info.gpu_branch_ms[k] for k in range(2))
     R.rtcc_destroy(ctx)
 
 
