@@ -166,18 +166,6 @@ __global__ void __launch_bounds__(kNmsThreads) k_nms(const rtcc_box* in, const i
   static_assert(32 * kNmsThreads <= kDecodeKeep * kNmsWords, "32 polygon slots per thread");
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   pdl_trigger();
-  {
-    // The blocks launch while the decode still runs: meanwhile, one pair
-    // test on two overlapping boxes built in registers (shared memory only,
-    // no global access) brings the clip path's instructions into this SM's
-    // instruction cache, off the critical path.
-    RRect a{0.0f, 0.0f, 1.0f, 0.0f, 2.0f, 1.0f}, b{0.5f, 0.25f, 0.8f, 0.6f, 2.0f, 1.0f};
-    if (warp == 0) {
-      const bool w = suppresses(a, 8.0f, b, 8.0f, thr, reinterpret_cast<float*>(sm) + tid);
-      asm volatile("" ::"r"((int)w));
-    }
-    __syncwarp();
-  }
   pdl_wait();                                   // the decoded boxes are the decode's output
   const int n = *n_in;
   const int W = (n + 31) >> 5;                  // row stride of the bitmask, in words
