@@ -6,8 +6,8 @@ The paper's DNN (Sec. III-B, Sec. V-A-1) is a PointPillars-based intermediate
 fusion detector: K independent per-agent encoder branches E_k, then a shared
 post-join subgraph (fusion and the classification/regression heads).  The paper
 states the structure but not the layer arithmetic, so each step below is the
-textbook definition of the named PointPillars operation, with the readings
-listed in the design doc where the paper is silent.
+textbook definition of the named PointPillars operation; where the paper is
+silent, each function's docstring states the reading it takes.
 
 All arithmetic is float64, except where a floating-point value decides an
 integer (the pillar index of a point), which is taken in float32 as the CUDA
