@@ -108,6 +108,22 @@ def fusion_bytes(cfg, k_present: int) -> float:
     return float(k_present * cells * cfg.feat_ch * 2 + cells * 16 * 4)
 
 
+def paired_gain(t_b, t_r, n_boot=2000, seed=0):
+    """Paired latency gain Barrier - RTCC over traces replayed in both modes
+    (index i of both lists is the same arrival trace), with a percentile
+    bootstrap 95% confidence interval of its mean (Sec. V-A-4's paired gain,
+    resampled pairs, seeded)."""
+    g = np.asarray(t_b, dtype=np.float64) - np.asarray(t_r, dtype=np.float64)
+    if g.size == 0:
+        return None
+    rng = np.random.default_rng(seed)
+    means = g[rng.integers(0, g.size, size=(n_boot, g.size))].mean(axis=1)
+    return {"pairs": int(g.size), "mean_ms": float(g.mean()), "median_ms": float(np.median(g)),
+            "ci95_ms": [float(np.percentile(means, 2.5)), float(np.percentile(means, 97.5))],
+            "positive": int((g > 0).sum()),
+            "rel_mean": float(np.mean(g / np.asarray(t_b, dtype=np.float64)))}
+
+
 def pfn_bytes(cfg, n_pillars: int, n_kept: int, n_raw: int) -> float:
     """Bytes the PFN kernel itself moves for one branch: the kept points'
     16-byte records (gathered), the raw point indices of the kept pillars'
@@ -423,7 +439,11 @@ def run_ours(args):
                        "barrier_p50": pct(b_res, 50), "barrier_p99": pct(b_res, 99),
                        "e2e_rtcc_p50": pct(r_e2e, 50), "e2e_rtcc_p99": pct(r_e2e, 99),
                        "e2e_barrier_p50": pct(b_e2e, 50), "e2e_barrier_p99": pct(b_e2e, 99),
-                       "frames_per_mode": len(r_res)},
+                       "frames_per_mode": len(r_res),
+                       # each step replays one trace in both modes: index i of the
+                       # RTCC and Barrier lists is the same trace
+                       "paired_gain": paired_gain(b_res, r_res),
+                       "paired_gain_e2e": paired_gain(b_e2e, r_e2e)},
         "encoder": {"tflops": enc_tflops, "frac_of_bf16_peak": (enc_tflops / tflops_peak)
                     if enc_tflops else None, "backbone_ms_per_branch": bb_ms,
                     "gflop_per_branch": flops / 1e9},

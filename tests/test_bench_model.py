@@ -34,3 +34,18 @@ def test_controller_decision_timing_runs_without_gpu():
             assert R.rtcc_ctrl_mark(cc, k, R.FINISHED) == R.OK
         assert R.rtcc_ctrl_end(cc) == R.OK
     R.rtcc_ctrl_destroy(cc)
+
+
+def test_paired_gain_bootstrap():
+    rng = np.random.default_rng(3)
+    t_r = rng.uniform(0.1, 0.2, 40)
+    t_b = t_r + 0.2 + rng.normal(0, 0.01, 40)
+    g = bench.paired_gain(t_b, t_r)
+    assert g["pairs"] == 40 and g["positive"] == 40
+    assert abs(g["mean_ms"] - float(np.mean(t_b - t_r))) < 1e-12
+    lo, hi = g["ci95_ms"]
+    assert lo < g["mean_ms"] < hi and hi - lo < 0.02
+    assert g == bench.paired_gain(t_b, t_r)                      # seeded
+    assert bench.paired_gain([], []) is None
+    one = bench.paired_gain([0.3], [0.1])
+    assert one["ci95_ms"][0] == one["ci95_ms"][1] == one["mean_ms"]
