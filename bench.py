@@ -108,6 +108,16 @@ def fusion_bytes(cfg, k_present: int) -> float:
     return float(k_present * cells * cfg.feat_ch * 2 + cells * 16 * 4)
 
 
+def max_over_ranks(vals, dist, device):
+    """Element-wise maximum of a few floats over all ranks: with one replica
+    per GPU, the job's latency is the worst replica's (and its wall time the
+    slowest rank's)."""
+    import torch
+    t = torch.tensor([float(v) for v in vals], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(x) for x in t]
+
+
 def paired_gain(t_b, t_r, n_boot=2000, seed=0):
     """Paired latency gain Barrier - RTCC over traces replayed in both modes
     (index i of both lists is the same arrival trace), with a percentile
@@ -406,9 +416,7 @@ def run_ours(args):
           if t > 0]
     value = pct(r_res, 50)
     if dist is not None:
-        t = torch.tensor([value, wall_ms], device="cuda", dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        value, wall_ms = float(t[0]), float(t[1])
+        value, wall_ms = max_over_ranks([value, wall_ms], dist, "cuda")
 
     hbm, tflops_peak, peak_kind = _peaks()
     flops = conv_flops(cfg)
