@@ -105,10 +105,11 @@ __device__ __forceinline__ void for_chunk(const uint32_t* keys, int lo, int chun
   }
 }
 
-// Coalesced pass over the (padded) key array: thread t takes the 16-byte
-// vectors t, t + kThreads, ...; f(key, index).
+// Coalesced pass over the (padded) key array, one 16-byte vector (4 keys) at
+// a time: thread t takes the vectors t, t + kThreads, ...; f(vector, index of
+// its first key).
 template <typename F>
-__device__ __forceinline__ void for_strided(const uint32_t* keys, int n4, F f) {
+__device__ __forceinline__ void for_strided4(const uint32_t* keys, int n4, F f) {
   const uint4* v = reinterpret_cast<const uint4*>(keys);
   constexpr int B = 8;                                   // loads in flight per thread
   for (int base = threadIdx.x; base < n4; base += B * kThreads) {
@@ -119,12 +120,7 @@ __device__ __forceinline__ void for_strided(const uint32_t* keys, int n4, F f) {
 #pragma unroll
     for (int j = 0; j < B; ++j) {
       const int q = base + j * kThreads;
-      if (q < n4) {
-        f(r[j].x, 4 * q);
-        f(r[j].y, 4 * q + 1);
-        f(r[j].z, 4 * q + 2);
-        f(r[j].w, 4 * q + 3);
-      }
+      if (q < n4) f(r[j], 4 * q);
     }
   }
 }
@@ -304,15 +300,21 @@ k_decode_select(const uint32_t* keys, uint32_t* hist0, const float* head, int ch
 
     if (nb0 <= kBndCap) {
       // ---- 2. one coalesced pass: lower bins -> sel, bin b0 -> bnd ----------
-      for_strided(keys, n4, [&](uint32_t k, int i) {
-        const uint32_t bin = k >> 20;                    // invalid keys: bin 4095 > b0
-        const bool cand = k != kInvalid && bin <= b0;
+      for_strided4(keys, n4, [&](const uint4& x, int i0) {
         // few keys are candidates (about K of tens of thousands): a warp
-        // skips the appends after one vote
-        if (__any_sync(__activemask(), cand)) {
-          const unsigned long long e = (static_cast<unsigned long long>(k) << 32) | static_cast<unsigned>(i);
-          warp_append(cand && bin < b0, e, &s_nsel, sel);
-          warp_append(cand && bin == b0, e, &s_nl, bnd);
+        // skips a round of 4 keys per lane after one vote on the smallest
+        // key of each lane's vector (invalid keys: bin 4095 > b0)
+        const uint32_t mn = min(min(x.x, x.y), min(x.z, x.w));
+        if (__any_sync(__activemask(), (mn >> 20) <= b0)) {
+          const uint32_t kk[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const uint32_t k = kk[e], bin = k >> 20;
+            const bool cand = k != kInvalid && bin <= b0;
+            const unsigned long long pr = (static_cast<unsigned long long>(k) << 32) | static_cast<unsigned>(i0 + e);
+            warp_append(cand && bin < b0, pr, &s_nsel, sel);
+            warp_append(cand && bin == b0, pr, &s_nl, bnd);
+          }
         }
       });
       __syncthreads();                                   // every thread has read nb0

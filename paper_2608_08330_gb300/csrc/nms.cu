@@ -239,6 +239,10 @@ __global__ void __launch_bounds__(kNmsThreads) k_nms(const rtcc_box* in, const i
       const uint32_t* rows = sm + (32 * c) * W;
       const uint32_t m = lane < left ? rows[lane * W + c] : 0u;
       uint32_t und = ~r, kept = 0u, sup = 0u;
+      if (__ballot_sync(0xFFFFFFFFu, m != 0u) == 0u) {
+        kept = und;                              // no row of the chunk suppresses another
+        und = 0u;
+      }
       for (int round = 0; round < 32 && und; ++round) {
         // rows still undecided may suppress later ones: those wait
         const uint32_t pot = __reduce_or_sync(0xFFFFFFFFu, ((und >> lane) & 1u) ? m : 0u);
