@@ -263,16 +263,20 @@ def encoder(points: np.ndarray, weights: Dict[str, np.ndarray], cfg,
             bb = store_round(weights[f"b{bi}.c{li}.b"], store)
             x = store_round(relu(conv3x3(x, w, bb, st if li == 0 else 1)), store)
         outs.append(x)
-    if cfg.up_strides:
-        ups = []
-        for bi, s in enumerate(cfg.up_strides):
-            w = store_round(weights[f"up{bi}.w"], store)
-            bb = store_round(weights[f"up{bi}.b"], store)
-            ups.append(store_round(relu(deconv(outs[bi], w, bb, s)), store))
-        feat = np.concatenate(ups, axis=0)
-    else:
-        feat = outs[-1]
+    feat = neck(outs, weights, cfg, store) if cfg.up_strides else outs[-1]
     return {"pillars": pill, "pfn": h, "image": image, "blocks": outs, "feat": feat}
+
+
+def neck(blocks: Sequence[np.ndarray], weights: Dict[str, np.ndarray], cfg,
+         store: Optional[str] = None) -> np.ndarray:
+    """Per block a deconv (kernel = stride = up_strides[b]) to up_ch channels
+    + ReLU, outputs rounded to the storage type, concatenated in block order."""
+    ups = []
+    for bi, s in enumerate(cfg.up_strides):
+        w = store_round(weights[f"up{bi}.w"], store)
+        bb = store_round(weights[f"up{bi}.b"], store)
+        ups.append(store_round(relu(deconv(blocks[bi], w, bb, s)), store))
+    return np.concatenate(ups, axis=0)
 
 
 # --------------------------------------------------------------------------
@@ -388,6 +392,28 @@ def detect(hd: np.ndarray, cfg) -> Dict[str, np.ndarray]:
 # --------------------------------------------------------------------------
 # whole frame
 # --------------------------------------------------------------------------
+
+
+def forward_multiscale(points: Sequence[Optional[np.ndarray]], weights: Dict[str, np.ndarray],
+                       cfg, store: Optional[str] = None) -> Dict[str, object]:
+    """The paper's placement of the fusion (Sec. IV-A; Sec. IV-D): every
+    present agent's encoder runs up to its backbone blocks; each block's
+    output is fused across the agents (the same per-cell max, or ego-query
+    attention at that block's channel count), rounded to the storage type;
+    the deconv neck and the concatenation then run once, after the join, on
+    the fused maps; then the head and the detections.  Parity unpinned
+    against the GPU (no kernel yet); pinned by the reductions in
+    tests/test_oracle_layers.py.
+    """
+    enc = [None if p is None else encoder(p, weights, cfg, store) for p in points]
+    fuse = fuse_max if cfg.fusion == "max" else fuse_attn
+    fused = [store_round(fuse([None if e is None else e["blocks"][bi] for e in enc]), store)
+             for bi in range(len(cfg.blocks))]
+    F = neck(fused, weights, cfg, store) if cfg.up_strides else fused[-1]
+    hw = store_round(weights["head.w"], store)
+    hb = store_round(weights["head.b"], store)
+    hd = head(F, hw, hb)
+    return {"enc": enc, "fused_blocks": fused, "fused": F, "head": hd, "det": detect(hd, cfg)}
 
 
 def forward(points: Sequence[Optional[np.ndarray]], weights: Dict[str, np.ndarray], cfg,

@@ -169,3 +169,67 @@ def test_forward_tiny_invariances():
     # storage-rounded and pure float64 forwards agree to the 16-bit rounding level
     pure = of.forward([p0, p1], w, cfg, store=None)
     assert np.max(np.abs(pure["head"] - out["head"])) < 2e-2 + 1e-2 * np.max(np.abs(pure["head"]))
+
+
+def _small_neck_cfg(fusion="max", n_agents=2):
+    import dataclasses
+    base = synth.get_config("pp3")
+    return dataclasses.replace(base, n_agents=n_agents, grid_w=32, grid_h=32, x_min=-6.4, x_max=6.4,
+                               y_min=-6.4, y_max=6.4, pts_x=(-7.0, 7.0), pts_y=(-7.0, 7.0),
+                               n_uniform=1500, n_clusters=2, cluster_pts=100, max_pillars=1024,
+                               fusion=fusion, anchors=2)
+
+
+@pytest.mark.parametrize("fusion", ["max", "attn"])
+def test_multiscale_fusion_of_one_agent_is_the_single_scale_path(fusion):
+    # one present agent: every per-scale fusion is the identity, so fusing
+    # before or after the neck gives the same head, exactly
+    cfg = _small_neck_cfg(fusion, n_agents=1)
+    w = synth.weights_for(cfg)
+    pts = [synth.points_for(cfg, 0, 0)]
+    a = of.forward(pts, w, cfg, store="fp16")
+    b = of.forward_multiscale(pts, w, cfg, store="fp16")
+    np.testing.assert_array_equal(a["head"], b["head"])
+    assert a["det"]["idx"].tolist() == b["det"]["idx"].tolist()
+
+
+def test_multiscale_attention_of_identical_agents_is_one_agent():
+    # identical agents have equal scores: uniform weights return the map
+    cfg = _small_neck_cfg("attn", n_agents=3)
+    w = synth.weights_for(cfg)
+    p = synth.points_for(cfg, 0, 0)
+    one = of.forward_multiscale([p], w, dataclasses_replace(cfg, n_agents=1))
+    three = of.forward_multiscale([p, p, p], w, cfg)
+    np.testing.assert_allclose(three["head"], one["head"], rtol=1e-12, atol=1e-12)
+
+
+def test_multiscale_max_is_agent_order_invariant_and_differs_from_late_fusion():
+    cfg = _small_neck_cfg("max", n_agents=3)
+    w = synth.weights_for(cfg)
+    pts = [synth.points_for(cfg, 0, k) for k in range(3)]
+    a = of.forward_multiscale(pts, w, cfg, store="fp16")
+    b = of.forward_multiscale(pts[::-1], w, cfg, store="fp16")
+    np.testing.assert_array_equal(a["head"], b["head"])
+    for bi, fb in enumerate(a["fused_blocks"]):             # each scale: max of the agents'
+        np.testing.assert_array_equal(fb, np.maximum.reduce([e["blocks"][bi] for e in a["enc"]]))
+    # the deconvs do not commute with the max: the placement changes the result
+    late = of.forward(pts, w, cfg, store="fp16")
+    assert not np.allclose(late["head"], a["head"])
+
+
+def dataclasses_replace(cfg, **kw):
+    import dataclasses
+    return dataclasses.replace(cfg, **kw)
+
+
+def test_multiscale_attention_is_a_convex_mix_per_scale():
+    # attention weights are a softmax: each fused cell lies between the
+    # agents' values, and (unlike max fusion) strictly inside somewhere
+    cfg = _small_neck_cfg("attn", n_agents=2)
+    w = synth.weights_for(cfg)
+    pts = [synth.points_for(cfg, 0, k) for k in range(2)]
+    r = of.forward_multiscale(pts, w, cfg)
+    for bi, fb in enumerate(r["fused_blocks"]):
+        xs = np.stack([e["blocks"][bi] for e in r["enc"]])
+        assert (fb >= xs.min(0) - 1e-12).all() and (fb <= xs.max(0) + 1e-12).all()
+        assert (fb < xs.max(0) - 1e-9).any()
