@@ -233,3 +233,44 @@ def test_multiscale_attention_is_a_convex_mix_per_scale():
         xs = np.stack([e["blocks"][bi] for e in r["enc"]])
         assert (fb >= xs.min(0) - 1e-12).all() and (fb <= xs.max(0) + 1e-12).all()
         assert (fb < xs.max(0) - 1e-9).any()
+
+
+def test_decode_regression_hand_worked():
+    # Two anchors with every regression term non-zero and distinct, so that
+    # each term is forced to its own channel and scale.  Expected values were
+    # worked out by hand from the anchor definition (tiny grid: 64 x 64 cells
+    # of 0.4 m from -12.8 m; car anchor l, w, h = 3.9, 1.6, 1.56 at z = -1,
+    # yaw a * pi / 2; d_a = sqrt(3.9^2 + 1.6^2) = sqrt(17.77) = 4.2154478).
+    #   anchor 0, cell (ix 10, iy 20): centre (-8.6, -4.6)
+    #     reg (0.5, -0.25, 0.2, 0.1, -0.2, 0.3, 0.1)
+    #     x = -8.6 + 0.5 d_a = -6.4922761    y = -4.6 - 0.25 d_a = -5.6538619
+    #     z = -1 + 0.2 * 1.56 = -0.688        l = 3.9 e^0.1 = 4.3101666
+    #     w = 1.6 e^-0.2 = 1.3099692          h = 1.56 e^0.3 = 2.1057797
+    #     yaw = 0 + 0.1
+    #   anchor 1, cell (ix 3, iy 5): centre (-11.4, -10.6)
+    #     reg (-0.1, 0.4, -0.5, -0.3, 0.25, -0.1, -0.2)
+    #     x = -11.4 - 0.1 d_a = -11.8215448   y = -10.6 + 0.4 d_a = -8.9138209
+    #     z = -1 - 0.5 * 1.56 = -1.78         l = 3.9 e^-0.3 = 2.8891911
+    #     w = 1.6 e^0.25 = 2.0544407          h = 1.56 e^-0.1 = 1.4115464
+    #     yaw = pi / 2 - 0.2 = 1.3707963
+    # A wrong diagonal (d_a = l_a), dz scaled by d_a, or a channel read one
+    # term off each move at least one of these numbers by more than 1e-3.
+    cfg = synth.get_config("tiny")
+    A, Hf, Wf = cfg.anchors, cfg.feat_h, cfg.feat_w
+    hd = np.zeros((8 * A, Hf, Wf))
+    hd[:A] = -5.0
+    hd[0, 20, 10] = 2.0
+    hd[1, 5, 3] = 1.0
+    hd[A + 0:A + 7, 20, 10] = (0.5, -0.25, 0.2, 0.1, -0.2, 0.3, 0.1)
+    hd[A + 7:A + 14, 5, 3] = (-0.1, 0.4, -0.5, -0.3, 0.25, -0.1, -0.2)
+    # decoy regression on the other anchor of each cell (must not be read)
+    hd[A + 7:A + 14, 20, 10] = 9.0
+    hd[A + 0:A + 7, 5, 3] = -9.0
+    det = of.decode(hd, cfg, cls_thresh=0.0, max_boxes=10)
+    assert det["idx"].tolist() == [(20 * Wf + 10) * A + 0, (5 * Wf + 3) * A + 1]
+    want = np.array([
+        [-6.4922761, -5.6538619, -0.688, 4.3101666, 1.3099692, 2.1057797, 0.1,
+         1.0 / (1.0 + math.exp(-2.0))],
+        [-11.8215448, -8.9138209, -1.78, 2.8891911, 2.0544407, 1.4115464, 1.3707963,
+         1.0 / (1.0 + math.exp(-1.0))]])
+    np.testing.assert_allclose(det["boxes"], want, rtol=0, atol=2e-7)

@@ -13,6 +13,7 @@ import os
 import numpy as np
 import pytest
 
+import synth
 from oracle import schedule as sch
 
 GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "schedule_example.json")
@@ -134,3 +135,34 @@ def test_uplink_multiple_rbs_and_weights():
     assert mw["alloc"][0] == [0, 0]                           # largest Q * R
     er = sch.uplink([10_000.0, 1_000.0, 3_000.0], [1, 1, 1], R, delta, "earliest")
     assert er["alloc"][0] == [1, 1]                           # smallest Q / (delta R)
+
+
+def test_rayleigh_rates_closed_forms():
+    # R = B log2(1 + snr |h|^2): snr 3 at |h|^2 = 1 gives log2(4) = 2 bit/s/Hz,
+    # snr 15 gives 4, snr 1 gives 1, and a faded-out slot (|h|^2 = 0) carries
+    # nothing.  A dB/linear mix-up or a natural log fails these.
+    B = 20e6
+    snr = np.array([3.0, 15.0, 1.0])
+    h2 = np.ones((2, 3, 4))
+    h2[1, :, 1] = 0.0
+    r = sch.rayleigh_rates(snr, h2, B)
+    assert r.shape == (2, 3, 4)
+    np.testing.assert_allclose(r[0, :, 0], [2 * B, 4 * B, B], rtol=1e-15)
+    assert np.all(r[1, :, 1] == 0.0)
+    # the rate doubles with |h|^2 = 5 at snr 3 (log2 16 = 4)
+    assert sch.rayleigh_rates(np.array([3.0]), np.full((1, 1, 1), 5.0), B)[0, 0, 0] == \
+        pytest.approx(4 * B, rel=1e-15)
+
+
+def test_channel_draws_snr_is_linear_from_db():
+    # Mean SNR is drawn uniform in dB over [0, 25] and returned linear: every
+    # value lies in [10^0, 10^2.5] and 10 log10 of the values is uniform (mean
+    # 12.5 dB); the fading power is Exp(1) (mean 1, variance 1).
+    d = synth.channel_draws(4000, 50, 8, frame=0, seed=11)
+    snr = d["snr"]
+    assert snr.min() >= 1.0 and snr.max() <= 10 ** 2.5
+    db = 10 * np.log10(snr)
+    assert abs(db.mean() - 12.5) < 0.4 and abs(db.std() - 25 / math.sqrt(12)) < 0.3
+    h2 = d["h2"]
+    assert h2.shape == (50, 4000, 8)
+    assert abs(h2.mean() - 1.0) < 0.01 and abs(h2.var() - 1.0) < 0.03
