@@ -393,3 +393,65 @@ def test_eight_agent_stress_full_size(R):
     cfg = synth.get_config("stress8")
     ctx, *_ = _end_to_end(R, cfg, frame=1, arrivals=[0.0] * cfg.n_agents)
     R.rtcc_destroy(ctx)
+
+
+def _production_frame(R, ctx, cfg, pts, a, mode, absent=()):
+    boxes = U.run_frame(ctx, cfg, pts, a, mode, absent=absent)
+    hd = R.rtcc_get_head(ctx, cfg.feat_h, cfg.feat_w).copy()
+    feats = b"".join(b"" if k in absent else R.rtcc_get_tensor(ctx, k, 8).tobytes()
+                     for k in range(cfg.n_agents))
+    dec = R.rtcc_get_decoded(ctx)
+    return hd, boxes, feats, dec
+
+
+@pytest.mark.parametrize("name,absent,spread", [("pp3", (), None), ("lr5", (2,), None),
+                                                ("stress8", (), "zero"),
+                                                ("stress8", (), "lognormal")])
+def test_production_context_full_size(R, name, absent, spread):
+    # The context the bench times: flags = 0, i.e. two ping-pong activation
+    # buffers per block (layer l + 1 overwrites what layer l - 1 wrote), the
+    # neck deconvs reading a block's last buffer while the next block runs,
+    # split-K through distributed shared memory, no per-layer buffers, no
+    # event nodes.  Checked end to end against the oracle (pillars bit-exact,
+    # pseudo-image, head, decode selection, NMS decisions), then the same
+    # frame in Barrier mode and again in RTCC mode must give byte-identical
+    # head, boxes and feature slots (Sec. III-C; Sec. V-F), and the debug
+    # context (per-layer buffers, checked layer by layer elsewhere) must give
+    # the same head byte for byte.
+    cfg = synth.get_config(name)
+    frame = 1
+    pts = [synth.points_for(cfg, frame, k) for k in range(cfg.n_agents)]
+    a = synth.arrivals_for(cfg, frame, spread)
+    ctx, w = U.make_ctx(cfg, flags=0)
+    try:
+        hd, boxes, feats, dec = _production_frame(R, ctx, cfg, pts, a, R.MODE_RTCC, absent)
+        for k in range(cfg.n_agents):
+            if k in absent:
+                continue
+            op = of.pillarise(pts[k], cfg)
+            gp = R.rtcc_get_pillars(ctx, k, cfg.grid_h, cfg.grid_w, cfg.max_pillars)
+            n = op["n_pillars"]
+            assert gp["n_pillars"] == n
+            np.testing.assert_array_equal(gp["cell2pillar"], op["cell2pillar"])
+            np.testing.assert_array_equal(gp["pillar_cell"][:n], op["pillar_cell"][:n])
+            np.testing.assert_array_equal(gp["count"][:n], op["count"][:n])
+            img_g = U.gpu_tensor(ctx, cfg, k, 0, (cfg.pfn_ch, cfg.grid_h, cfg.grid_w))
+            img_o = of.scatter(of.pfn(op, w["pfn.w"], w["pfn.b"], cfg, cfg.dtype), op, cfg)
+            U.assert_close(img_g, img_o, f"pseudo-image agent {k}")
+        hd_o = U.head_to_oracle_layout(hd)
+        full = of.forward([None if k in absent else pts[k] for k in range(cfg.n_agents)], w, cfg,
+                          store=cfg.dtype)
+        U.assert_close(hd_o, full["head"], "head (end to end, production context)")
+        _check_decode(cfg, hd_o, boxes, R, ctx)
+        ref = (hd.tobytes(), boxes.tobytes(), feats, dec.tobytes())
+        for mode in (R.MODE_BARRIER, R.MODE_RTCC):
+            h2, b2, f2, d2 = _production_frame(R, ctx, cfg, pts, a, mode, absent)
+            assert (h2.tobytes(), b2.tobytes(), f2, d2.tobytes()) == ref, f"mode {mode} differs"
+    finally:
+        R.rtcc_destroy(ctx)
+    dctx, _ = U.make_ctx(cfg)
+    try:
+        U.run_frame(dctx, cfg, pts, a, R.MODE_RTCC, absent=absent)
+        assert R.rtcc_get_head(dctx, cfg.feat_h, cfg.feat_w).tobytes() == ref[0]
+    finally:
+        R.rtcc_destroy(dctx)
