@@ -345,9 +345,12 @@ rtcc_status rtcc_get_tensor(struct rtcc_ctx* ctx, int32_t agent, int32_t which,
  * d_pillar_cell and d_count int32 [max_pillars] (entries >= n_pillars are left
  * untouched), d_stats int32 [8] = {n, n_in_range, n_pillars, n_kept, 0, 0,
  * dropped by the per-pillar cap, points of kept pillars before that cap},
- * d_image 16-bit [H][W][pfn_ch].  Work is enqueued on `stream` (a
- * cudaStream_t; NULL = the default stream) and the call returns without
- * waiting.
+ * d_image 16-bit [H][W][pfn_ch].  d_points and d_image must be 16-byte
+ * aligned and the other pointers 4-byte aligned, else RTCC_E_ARG.  Work is
+ * enqueued on `stream` (a cudaStream_t; NULL = the default stream) and the
+ * call returns without waiting.  RTCC_E_CUDA reports a failed launch of this
+ * call's own kernels; an error left by the caller's earlier work is neither
+ * reported nor cleared.
  *
  * The first call on a device looks up the array's device address; make that
  * first call outside any stream capture.  Every call shares the array and

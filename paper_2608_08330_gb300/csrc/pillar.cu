@@ -469,8 +469,7 @@ cudaError_t launch_all(const PillarBufs& b, const GridGeom& g, const float* pfn_
   e = launch_pdl(k_pfn<T, C>, dim3((b.P + 7) / 8), dim3(256), 0, st, b.pts, b.stats, b.pcnt_raw,
                  b.poff, b.list, b.pillar_cell, pfn_w, pfn_b, g, b.N, static_cast<T*>(b.image),
                  b.cell2pillar, b.np_prev, b.pcount, b.pfn_span);
-  if (e != cudaSuccess) return e;
-  return cudaGetLastError();
+  return e;                                       // each launch reported its own status
 }
 
 }  // namespace

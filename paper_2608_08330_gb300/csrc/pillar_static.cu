@@ -102,6 +102,14 @@ extern "C" rtcc_status rtcc_pillarise_noalloc(const rtcc_model_config* cfg, cons
   if (cfg->pfn_ch != 32 && cfg->pfn_ch != kMaxCh) return RTCC_E_ARG;
   if (cfg->dtype != RTCC_FP16 && cfg->dtype != RTCC_BF16) return RTCC_E_ARG;
   if (!(cfg->pillar > 0.f)) return RTCC_E_ARG;
+  // The kernels read the points as float4 and clear the image with 16-byte
+  // stores; a sub-view that is not so aligned is refused here instead of
+  // faulting on the device.
+  auto misaligned = [](const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) != 0; };
+  if ((n_points > 0 && misaligned(d_points, 16)) || misaligned(d_image, 16) || misaligned(d_pfn_w, 4) ||
+      misaligned(d_pfn_b, 4) || misaligned(d_cell2pillar, 4) || misaligned(d_pillar_cell, 4) ||
+      misaligned(d_count, 4) || misaligned(d_stats, 4))
+    return RTCC_E_ARG;
   unsigned char* base = nullptr;
   rtcc_status s = scratch_address(&base);
   if (s != RTCC_OK) return s;
@@ -134,10 +142,15 @@ extern "C" rtcc_status rtcc_pillarise_noalloc(const rtcc_model_config* cfg, cons
 
   int blocks = (int)((cells + 255) / 256);
   if (blocks < 1) blocks = 1;
-  k_static_reset<<<blocks, 256, 0, st>>>(n_points, (int)cells,
-                                         reinterpret_cast<int*>(base + kOffN), b.cnt_cell,
-                                         b.first_cell, d_stats);
-  if (cudaGetLastError() != cudaSuccess) return RTCC_E_CUDA;
+  // cudaLaunchKernelEx reports this launch's own error; an error state the
+  // caller's earlier work left on the thread is neither returned nor cleared
+  cudaLaunchConfig_t lc = {};
+  lc.gridDim = dim3(blocks);
+  lc.blockDim = dim3(256);
+  lc.stream = st;
+  if (cudaLaunchKernelEx(&lc, k_static_reset, n_points, (int)cells, reinterpret_cast<int*>(base + kOffN),
+                         b.cnt_cell, b.first_cell, d_stats) != cudaSuccess)
+    return RTCC_E_CUDA;
   GridGeom g{cfg->x_min, cfg->y_min, cfg->z_min, cfg->z_max, cfg->pillar, cfg->grid_w,
              cfg->grid_h};
   if (launch_pillarise(b, g, d_pfn_w, d_pfn_b, cfg->dtype == RTCC_BF16, nullptr, st) !=
