@@ -97,6 +97,18 @@ typedef enum {
                                     clusters: split-K slices then reduce
                                     through global memory instead of
                                     distributed shared memory (same results)  */
+#define RTCC_FLAG_SHORT_WAITS 32 /* bounded device waits give up after about
+                                    10 ms instead of about 1 s, and
+                                    rtcc_test_unreachable_wait is enabled
+                                    (tests of the wait limit)                  */
+#define RTCC_FLAG_NO_BATCH    64 /* every branch runs its own backbone launch,
+                                    also when branches are released together
+                                    (same results; for comparisons)           */
+#define RTCC_FLAG_H2D_COPY   128 /* host payloads reach the device slot by a
+                                    copy-engine transfer on a transfer stream
+                                    whose event gates the branch stream, instead
+                                    of the branch's first kernel reading the
+                                    pinned staging buffer (same results)       */
 
 /*
  * Network and workload description.  Supported: 1 <= n_agents <= 8;
@@ -163,6 +175,13 @@ typedef struct {
                                        end); -1 without RTCC_FLAG_TIMELINE    */
   float gpu_pfn_kernel_ms[RTCC_MAX_AGENTS];  /* each branch's PFN kernel span, the
                                                 same way; -1 without the flag  */
+  int32_t n_backbone_launches;      /* backbone launches of the frame: agents
+                                       released together share one            */
+  int32_t backbone_batch[RTCC_MAX_AGENTS];  /* agents in each launch, in launch
+                                               order; 0 pad                    */
+  float gpu_launch_ms[RTCC_MAX_AGENTS];     /* each launch's backbone span (CUDA
+                                               events); -1 without
+                                               RTCC_FLAG_TIMELINE              */
 } rtcc_frame_info;
 
 /* ------------------------------------------------------------------------ */
@@ -176,8 +195,10 @@ typedef struct {
  * b; head W [8A][C_feat], b.  The library rounds each tensor once to the
  * storage dtype and repacks it for its kernels; the caller's blob is not kept.
  * Allocates all device memory, pinned staging buffers, streams, events and
- * the K branch graphs plus the post-join graph.  RTCC_E_ARG for an
- * unsupported config or a blob of the wrong length.
+ * the K branch graphs plus the post-join graph, and (unless
+ * RTCC_FLAG_NO_BATCH) starts one host thread, the dispatcher of batched
+ * backbone launches (see rtcc_payload_complete), which rtcc_destroy joins.
+ * RTCC_E_ARG for an unsupported config or a blob of the wrong length.
  */
 rtcc_status rtcc_init(const rtcc_model_config* cfg, const float* weights,
                       size_t n_floats, struct rtcc_ctx** out);
@@ -222,6 +243,16 @@ rtcc_status rtcc_frame_begin(struct rtcc_ctx* ctx, uint64_t frame_id, double t0_
  * Barrier mode it is held until every branch is resolved.  host_points must
  * stay unchanged until rtcc_wait_detection returns for this frame; when it is
  * the staging buffer no host copy is made.
+ *
+ * Launches (Sec. III-B's single encoder stream, kept busy): a branch released
+ * while no backbone runs starts at once, pillar chain and backbone.  One
+ * released while another branch's backbone still runs starts its pillar chain
+ * at once; its backbone is held and, when the running backbone ends, the
+ * dispatcher thread launches one backbone over every branch held meanwhile.
+ * Branches released by one event (Barrier at A) share one launch, and the
+ * event that resolves the last branch launches whatever is held at once.
+ * Every branch writes its own slot and its result does not depend on the
+ * launch that ran it, so RTCC and Barrier outputs stay byte-identical.
  */
 rtcc_status rtcc_payload_complete(struct rtcc_ctx* ctx, int32_t agent,
                                   const float* host_points, int32_t n_points,
@@ -405,9 +436,22 @@ rtcc_status rtcc_ctrl_end(rtcc_controller* c);
 const char* rtcc_status_str(rtcc_status s);
 /* Library steady clock in milliseconds. */
 double rtcc_now_ms(void);
-/* Number of kernel launches one frame makes (branches + post-join), for the
- * given number of present agents. */
+/* Number of kernel launches of the most recent frame (pillar chains, backbone
+ * launches, post-join) for the given number of present agents; before any
+ * frame, with one backbone launch per branch. */
 int32_t rtcc_kernels_per_frame(struct rtcc_ctx* ctx, int32_t n_present);
+
+/*
+ * Test hook for the device-side wait limit (no counterpart in the paper): each
+ * backbone launch of the next frame waits, in its first layer that depends on
+ * another, for one more finished work item than that layer has.  The wait runs
+ * out after the context's limit (use RTCC_FLAG_SHORT_WAITS: about 10 ms), the
+ * kernel sets its error word and winds down without trapping, and
+ * rtcc_wait_detection returns RTCC_E_DEVICE; it then clears the error state so
+ * the next frame runs normally.  Only between frames; RTCC_E_STATE on a
+ * context without RTCC_FLAG_SHORT_WAITS.
+ */
+rtcc_status rtcc_test_unreachable_wait(struct rtcc_ctx* ctx);
 
 /*
  * Rotated BEV NMS of n <= 512 boxes already in rank order (the frame's own

@@ -13,9 +13,11 @@
 #include <atomic>
 #include <chrono>
 #include <cmath>
+#include <condition_variable>
 #include <cstring>
 #include <mutex>
 #include <new>
+#include <thread>
 #include <vector>
 
 #include <cuda_bf16.h>
@@ -40,24 +42,25 @@ struct Branch {
   float* staging = nullptr;        // pinned [kHdrBytes][cap][4]
   uint8_t* in_dev = nullptr;       // device [kHdrBytes][cap][4]
   PillarBufs pb{};
-  void* block_buf[RTCC_MAX_BLOCKS][2] = {};
-  std::vector<void*> layer_out;    // every conv layer's output (RTCC_FLAG_KEEP_LAYERS)
-  std::vector<size_t> layer_elems;
-  void* block_out[RTCC_MAX_BLOCKS] = {};
-  int block_w[RTCC_MAX_BLOCKS] = {}, block_h[RTCC_MAX_BLOCKS] = {};
-  void* feat = nullptr;            // agent-indexed feature slot [H'][W'][C_feat]
-  std::vector<ConvLayer> layers;
-  float* splitk_ws = nullptr;      // split-K partials, shared by the branch's layers
+  void* feat = nullptr;            // agent-indexed feature slot [H'][W'][C_feat] (a view
+                                   // into the context's feature slots)
+  float* splitk_ws = nullptr;      // split-K partials of this branch's own launches
   int* splitk_cnt = nullptr;       // split-K per-tile arrival counters
-  unsigned* grid_bar = nullptr;      // inside frame_zero
-  void* frame_zero = nullptr;         // [kFrameZeroBytes] cleared at the start of every branch graph    // backbone per-layer arrival counters
+  unsigned* grid_bar = nullptr;      // inside frame_zero: per-layer counters + exit count
+  void* frame_zero = nullptr;         // [kFrameZeroBytes] cleared at the start of every branch graph
   unsigned long long* stamps = nullptr;   // RTCC_FLAG_LAYER_TIMES: layer starts, then ends
-  BackboneParams* bb = nullptr;    // backbone kernel parameters (host copy)
+  BackboneParams* bb = nullptr;    // backbone kernel parameters of this agent alone
   cudaStream_t st = nullptr;
-  cudaGraphExec_t exec = nullptr;       // payload already in the device slot
-  cudaGraphExec_t exec_host = nullptr;  // payload in the pinned staging buffer (zero-copy)
-  cudaEvent_t h2d_done = nullptr, done = nullptr;
+  cudaGraphExec_t exec = nullptr;       // pillar chain + backbone, payload in the device slot
+  cudaGraphExec_t exec_host = nullptr;  // the same, payload in the pinned staging buffer (zero-copy)
+  cudaGraphExec_t pill = nullptr;       // pillar chain alone (the backbone runs in a batch)
+  cudaGraphExec_t pill_host = nullptr;
+  cudaEvent_t h2d_done = nullptr, done = nullptr, pill_done = nullptr;
   cudaEvent_t ev_start = nullptr, ev_bb0 = nullptr, ev_bb1 = nullptr, ev_end = nullptr;
+  cudaEvent_t feat_ev = nullptr;   // this frame: the event after which the slot is written
+  int stamp_src = -1;              // this frame: whose stamps buffer its launch wrote
+  int launch_idx = -1;             // this frame: index of the backbone launch that ran it
+  bool full_graph = false;         // this frame: ran as its own branch graph (event nodes)
   const float* pend_ptr = nullptr;
   int pend_n = 0;
   bool pend_resident = false;
@@ -83,6 +86,42 @@ struct rtcc_ctx {
   float* head_b = nullptr;
   void* head_w16 = nullptr;   // head weights [16][C] in the storage type (tensor-core head)
   Branch br[RTCC_MAX_AGENTS];
+  void* image_all = nullptr;          // pseudo-images [K][H][W][C_p]
+  // Backbone tensors of all agents, agent-major with a fixed stride (one
+  // tensor map covers every agent; a launch runs any subset)
+  void* feat_all = nullptr;           // [K][H'][W'][C_feat]
+  void* block_all[RTCC_MAX_BLOCKS][2] = {};   // ping-pong activations [K][H_b][W_b][C_b]
+  std::vector<void*> layer_all;       // RTCC_FLAG_KEEP_LAYERS: every conv's output [K][...]
+  std::vector<size_t> layer_elems;    // elements per agent
+  void* block_out[RTCC_MAX_BLOCKS] = {};
+  int block_w[RTCC_MAX_BLOCKS] = {}, block_h[RTCC_MAX_BLOCKS] = {};
+  size_t img_elems = 0, feat_elems = 0;
+  std::vector<ConvLayer> layers;      // the layer list (N tiles of a one-agent launch)
+  BackboneParams* bbt[RTCC_MAX_AGENTS + 1] = {};  // launch parameters per batch size
+  long long wait_budget = 0;
+  // batched backbone launches (agents released together)
+  cudaStream_t bbst = nullptr;
+  float* batch_ws = nullptr;
+  int* batch_cnt = nullptr;
+  unsigned* batch_bar = nullptr;      // [kMaxLayers + 1], zero between launches
+  cudaEvent_t batch_ev[RTCC_MAX_AGENTS] = {}, batch_t0[RTCC_MAX_AGENTS] = {},
+              batch_t1[RTCC_MAX_AGENTS] = {};
+  BackboneParams* launch_p = nullptr; // scratch for one launch's parameters
+  volatile int* done_words = nullptr; // pinned [2 * RTCC_MAX_AGENTS]: written 1 by the last
+                                      // CTA of branch k's own backbone launch (k) or of
+                                      // batched launch j (RTCC_MAX_AGENTS + j)
+  int inflight = -1;                  // done word of the last backbone launched, -1 none
+  int n_launches = 0;                 // backbone launches this frame
+  int launch_size[RTCC_MAX_AGENTS] = {};
+  int launch_word[RTCC_MAX_AGENTS] = {};
+  std::vector<int> pending;           // released agents whose backbone waits for a batch
+  std::thread disp;                   // dispatcher of deferred batches
+  std::condition_variable cv;
+  bool stop = false;
+  int dev = 0;
+  volatile int* stall = nullptr;      // pinned test hook word (RTCC_FLAG_SHORT_WAITS)
+  bool disp_err = false;              // the dispatcher failed to launch a batch
+  size_t splitk_cnt_bytes = 0;        // split-K tile counters of one branch (batch: K x)
   cudaStream_t xfer = nullptr, post = nullptr;
   cudaGraphExec_t post_exec = nullptr;
   int* d_present = nullptr;           // [K] set by a branch's first kernel, cleared by the decode
@@ -339,16 +378,212 @@ void pick_tile(int m_tiles, int co, int total_kb, int grid, int* bn_out, int* sp
   *sp_out = bs;
 }
 
-constexpr size_t kFrameZeroBytes = 8 * sizeof(int) + kMaxLayers * sizeof(unsigned);
+constexpr size_t kFrameZeroBytes = 8 * sizeof(int) + (kMaxLayers + 1) * sizeof(unsigned);
 
-rtcc_status build_branch(rtcc_ctx* c, int k) {
-  Branch& b = c->br[k];
+// N tile of a conv layer in a launch over `batch` agents, with its K slices
+// fixed (they decide the fp32 summation order, so they are the same for every
+// batch size and a branch's result does not depend on the launch that ran
+// it; the N tile only decides which channels an item computes).  Cost model
+// of pick_tile: rounds of items over the grid times k-blocks per item; ties go
+// to the wider tile (fewer, longer items per FLOP).
+int pick_bn_batch(int m_tiles, int co, int total_kb, int sp, int grid, int batch, bool need64) {
+  double best = 1e30;
+  int bb = std::min(co, 64);
+  for (int bn : {128, 64, 32}) {
+    if (bn > co || co % bn) continue;
+    if (need64 && bn != 64) continue;
+    const int items = batch * m_tiles * (co / bn) * sp;
+    const int rounds = (items + grid - 1) / grid;
+    const double cost = rounds * (double)((total_kb + sp - 1) / sp);
+    if (cost < best - 1e-9) {
+      best = cost;
+      bb = bn;
+    }
+  }
+  return bb;
+}
+
+// The backbone's layer list over the agent-major tensors of all K agents, and
+// the launch parameters for every batch size.
+rtcc_status build_backbone(rtcc_ctx* c) {
   const rtcc_model_config& g = c->cfg;
-  // CTAs of a backbone launch in clusters (split-K slices share a cluster)
+  const int K = c->K;
+  // the tile choice uses the clustered grid with or without clusters, so the
+  // K slices (and the results) do not depend on RTCC_FLAG_NO_CLUSTERS
   int grid = backbone_grid(kMaxSplits);
   if (grid < 1) grid = backbone_grid(1);
   if (grid < 1) return RTCC_E_CUDA;
   const size_t es = 2;   // 16-bit storage
+  c->img_elems = (size_t)c->W * c->H * c->Cp;
+  c->feat_elems = (size_t)c->Wf * c->Hf * c->Cf;
+  RS(dalloc(c, &c->feat_all, (size_t)K * c->feat_elems * es));
+  CK(cudaMemset(c->feat_all, 0, (size_t)K * c->feat_elems * es));
+  const bool neck = g.up_stride[0] != 0;
+  const bool keep = (g.flags & RTCC_FLAG_KEEP_LAYERS) != 0;
+  int block_last[RTCC_MAX_BLOCKS] = {};
+  const void* in = c->image_all;                  // the agents' pseudo-images, agent-major
+  long long in_as = (long long)c->img_elems;
+  int cin = c->Cp, w = c->W, h = c->H;
+  int wi = 0;
+  for (int bi = 0; bi < g.n_blocks; ++bi) {
+    const int st = g.block_stride[bi];
+    const int ow = w / st, oh = h / st;
+    const int co = g.block_ch[bi];
+    const size_t per = (size_t)ow * oh * co;
+    if (!keep) {
+      RS(dalloc(c, &c->block_all[bi][0], (size_t)K * per * es));
+      RS(dalloc(c, &c->block_all[bi][1], (size_t)K * per * es));
+    }
+    for (int li = 0; li < g.block_layers[bi]; ++li) {
+      ConvLayer L{};
+      L.kind = (li == 0 && st == 2) ? CONV3_S2 : CONV3_S1;
+      L.n_agents = K;
+      L.cin = cin;
+      L.cout = co;
+      L.s = 1;
+      L.in_w = (li == 0) ? w : ow;
+      L.in_h = (li == 0) ? h : oh;
+      L.out_w = ow;
+      L.out_h = oh;
+      L.gw = ow;
+      L.gh = oh;
+      L.ldc = co;
+      L.choff = 0;
+      const int m_tiles = ((ow + conv_tile_w() - 1) / conv_tile_w()) *
+                          ((oh + conv_tile_h() - 1) / conv_tile_h());
+      L.bk = (cin >= 64) ? 64 : 32;
+      pick_tile(m_tiles, co, 9 * (cin / L.bk), grid, &L.bn, &L.splits);
+      L.n_tiles_n = co / L.bn;
+      L.in = in;
+      L.in_astride = in_as;
+      const bool last = (bi == g.n_blocks - 1) && (li == g.block_layers[bi] - 1);
+      void* dst = nullptr;
+      long long out_as = (long long)per;
+      if (!neck && last) {
+        dst = c->feat_all;
+        out_as = (long long)c->feat_elems;
+      } else if (keep) {
+        RS(dalloc(c, &dst, (size_t)K * per * es));
+      } else {
+        dst = c->block_all[bi][li & 1];
+      }
+      L.out = dst;
+      L.out_astride = out_as;
+      c->layer_all.push_back(dst);
+      c->layer_elems.push_back(per);
+      L.wpacked = c->wbufs[wi];
+      L.bias = c->bbufs[wi];
+      L.wait_layers = (int)c->layers.size();          // reads the previous conv's output
+      ++wi;
+      c->layers.push_back(L);
+      in = L.out;
+      in_as = out_as;
+      cin = co;
+    }
+    c->block_out[bi] = const_cast<void*>(in);
+    block_last[bi] = (int)c->layers.size();          // layers [0, block_last) done
+    c->block_w[bi] = ow;
+    c->block_h[bi] = oh;
+    w = ow;
+    h = oh;
+  }
+  if (neck) {
+    for (int bi = 0; bi < g.n_blocks; ++bi) {
+      ConvLayer L{};
+      L.kind = DECONV;
+      L.n_agents = K;
+      L.s = g.up_stride[bi];
+      L.cin = g.block_ch[bi];
+      L.cout = g.up_ch;
+      L.in_w = c->block_w[bi];
+      L.in_h = c->block_h[bi];
+      L.out_w = c->Wf;
+      L.out_h = c->Hf;
+      L.gw = L.in_w;
+      L.gh = L.in_h;
+      L.ldc = c->Cf;
+      L.choff = bi * g.up_ch;
+      L.bn = g.up_ch;
+      L.bk = (L.cin >= 64) ? 64 : 32;
+      L.n_tiles_n = L.s * L.s;
+      L.in = c->block_out[bi];
+      L.in_astride = (long long)c->block_w[bi] * c->block_h[bi] * g.block_ch[bi];
+      L.out = c->feat_all;
+      L.out_astride = (long long)c->feat_elems;
+      L.wpacked = c->wbufs[wi];
+      L.bias = c->bbufs[wi];
+      L.wait_layers = block_last[bi];                 // only its block's output
+      ++wi;
+      c->layers.push_back(L);
+    }
+  }
+  // fp32 workspace of the global-memory split-K reduction (used when a split
+  // layer cannot reduce through DSMEM): one per branch for its own launches,
+  // and one for the batched launches; deconvs never split
+  size_t ws_floats = 0, max_tiles = 0;
+  for (ConvLayer& L : c->layers) {
+    const int m_tiles = ((L.gw + conv_tile_w() - 1) / conv_tile_w()) *
+                        ((L.gh + conv_tile_h() - 1) / conv_tile_h());
+    if (L.kind == DECONV || L.splits < 1) L.splits = 1;
+    if (L.splits > 1) {
+      // the widest tile any batch size may pick: co / 32 tiles of 32 ... 128 columns
+      ws_floats = std::max(ws_floats, (size_t)L.splits * m_tiles * L.cout * conv_tile_m());
+      max_tiles = std::max(max_tiles, (size_t)m_tiles * (L.cout / 32));
+    }
+  }
+  c->splitk_cnt_bytes = max_tiles * sizeof(int);
+  for (int k = 0; k < K; ++k) {
+    Branch& b = c->br[k];
+    if (ws_floats) {
+      RS(dalloc(c, &b.splitk_ws, ws_floats * sizeof(float)));
+      RS(dalloc(c, &b.splitk_cnt, max_tiles * sizeof(int)));
+      CK(cudaMemset(b.splitk_cnt, 0, max_tiles * sizeof(int)));
+    }
+  }
+  if (ws_floats) {
+    RS(dalloc(c, &c->batch_ws, (size_t)K * ws_floats * sizeof(float)));
+    RS(dalloc(c, &c->batch_cnt, (size_t)K * max_tiles * sizeof(int)));
+    CK(cudaMemset(c->batch_cnt, 0, (size_t)K * max_tiles * sizeof(int)));
+  }
+  RS(dalloc(c, &c->batch_bar, (kMaxLayers + 1) * sizeof(unsigned)));
+  CK(cudaMemset(c->batch_bar, 0, (kMaxLayers + 1) * sizeof(unsigned)));
+  c->wait_budget = (g.flags & RTCC_FLAG_SHORT_WAITS) ? 20000000LL : 2000000000LL;
+  // launch parameters per batch size: the same K slices, the N tile chosen
+  // for the batch
+  for (int nb = 1; nb <= K; ++nb) {
+    std::vector<ConvLayer> Lb = c->layers;
+    for (ConvLayer& L : Lb) {
+      if (nb > 1 && L.kind != DECONV) {
+        const int m_tiles = ((L.gw + conv_tile_w() - 1) / conv_tile_w()) *
+                            ((L.gh + conv_tile_h() - 1) / conv_tile_h());
+        const int total_kb = 9 * (L.cin / L.bk);
+        // a split layer whose items fit the clustered grid keeps the DSMEM
+        // exchange (64-wide tiles); otherwise it reduces through global memory
+        const bool dsm_fit = L.splits > 1 && nb * m_tiles * (L.cout / 64) * L.splits <= grid;
+        L.bn = pick_bn_batch(m_tiles, L.cout, total_kb, L.splits, grid, nb, dsm_fit);
+        L.n_tiles_n = L.cout / L.bn;
+      }
+      L.ws = c->batch_ws;
+      L.counters = c->batch_cnt;
+      if (conv_make_maps(L, c->bf16) != cudaSuccess) return RTCC_E_CUDA;
+    }
+    if (nb == 1) c->layers = Lb;                      // the maps of the one-agent tiles
+    c->bbt[nb] = new (std::nothrow) BackboneParams;
+    if (!c->bbt[nb]) return RTCC_E_NOMEM;
+    if (backbone_fill(Lb, nb, c->batch_bar, c->d_err, nullptr, (g.flags & RTCC_FLAG_NO_CLUSTERS) == 0,
+                      c->wait_budget, c->bbt[nb]) != cudaSuccess)
+      return RTCC_E_ARG;
+  }
+  c->launch_p = new (std::nothrow) BackboneParams;
+  if (!c->launch_p) return RTCC_E_NOMEM;
+  return RTCC_OK;
+}
+
+// Per-agent state of branch k: payload slot, pillar scratch, its own launch
+// parameters (the one-agent template pointed at this agent and its counters).
+rtcc_status build_branch(rtcc_ctx* c, int k) {
+  Branch& b = c->br[k];
+  const rtcc_model_config& g = c->cfg;
   const int cells = c->W * c->H;
   RS(halloc(c, &b.staging, kHdrBytes + (size_t)c->cap * 16));
   std::memset(b.staging, 0, kHdrBytes);
@@ -382,152 +617,48 @@ rtcc_status build_branch(rtcc_ctx* c, int k) {
   RS(dalloc(c, &p.pillar_cell, (size_t)c->P * 4));
   RS(dalloc(c, &p.pcount, (size_t)c->P * 4));
   // words cleared at the start of every branch graph (one memset): the pillar
-  // stats [8] and the backbone's per-layer arrival counters [kMaxLayers]
+  // stats [8] and the backbone's per-layer arrival counters and exit count
   RS(dalloc(c, &b.frame_zero, kFrameZeroBytes));
   CK(cudaMemset(b.frame_zero, 0, kFrameZeroBytes));
   p.stats = reinterpret_cast<int*>(b.frame_zero);
   RS(dalloc(c, &p.cell2pillar, (size_t)cells * 4));
-  RS(dalloc(c, &p.image, (size_t)cells * c->Cp * es));
   CK(cudaMemset(p.cnt_cell, 0, (size_t)cells * 4));
   CK(cudaMemset(p.first_cell, 0x7F, (size_t)cells * 4));
-  CK(cudaMemset(p.image, 0, (size_t)cells * c->Cp * es));
   CK(cudaMemset(p.cell2pillar, 0xFF, (size_t)cells * 4));
-  RS(dalloc(c, &b.feat, (size_t)c->Wf * c->Hf * c->Cf * es));
-  CK(cudaMemset(b.feat, 0, (size_t)c->Wf * c->Hf * c->Cf * es));
-
-  // backbone layers
-  const bool neck = g.up_stride[0] != 0;
-  int block_last[RTCC_MAX_BLOCKS] = {};
-  const void* in = p.image;
-  int cin = c->Cp, w = c->W, h = c->H;
-  int wi = 0;
-  for (int bi = 0; bi < g.n_blocks; ++bi) {
-    const int st = g.block_stride[bi];
-    const int ow = w / st, oh = h / st;
-    const int co = g.block_ch[bi];
-    const bool keep = (g.flags & RTCC_FLAG_KEEP_LAYERS) != 0;
-    if (!keep) {
-      RS(dalloc(c, &b.block_buf[bi][0], (size_t)ow * oh * co * es));
-      RS(dalloc(c, &b.block_buf[bi][1], (size_t)ow * oh * co * es));
-    }
-    for (int li = 0; li < g.block_layers[bi]; ++li) {
-      ConvLayer L{};
-      L.kind = (li == 0 && st == 2) ? CONV3_S2 : CONV3_S1;
-      L.cin = cin;
-      L.cout = co;
-      L.s = 1;
-      L.in_w = (li == 0) ? w : ow;
-      L.in_h = (li == 0) ? h : oh;
-      L.out_w = ow;
-      L.out_h = oh;
-      L.gw = ow;
-      L.gh = oh;
-      L.ldc = co;
-      L.choff = 0;
-      const int m_tiles = ((ow + conv_tile_w() - 1) / conv_tile_w()) *
-                          ((oh + conv_tile_h() - 1) / conv_tile_h());
-      L.bk = (cin >= 64) ? 64 : 32;
-      pick_tile(m_tiles, co, 9 * (cin / L.bk), grid, &L.bn, &L.splits);
-      L.n_tiles_n = co / L.bn;
-      L.in = in;
-      const bool last = (bi == g.n_blocks - 1) && (li == g.block_layers[bi] - 1);
-      void* dst = nullptr;
-      if (!neck && last) {
-        dst = b.feat;
-      } else if (keep) {
-        RS(dalloc(c, &dst, (size_t)ow * oh * co * es));
-      } else {
-        dst = b.block_buf[bi][li & 1];
-      }
-      L.out = dst;
-      b.layer_out.push_back(dst);
-      b.layer_elems.push_back((size_t)ow * oh * co);
-      L.wpacked = c->wbufs[wi];
-      L.bias = c->bbufs[wi];
-      L.wait_layers = (int)b.layers.size();          // reads the previous conv's output
-      ++wi;
-      if (conv_make_maps(L, c->bf16) != cudaSuccess) return RTCC_E_CUDA;
-      b.layers.push_back(L);
-      in = L.out;
-      cin = co;
-    }
-    b.block_out[bi] = const_cast<void*>(in);
-    block_last[bi] = (int)b.layers.size();          // layers [0, block_last) done
-
-    b.block_w[bi] = ow;
-    b.block_h[bi] = oh;
-    w = ow;
-    h = oh;
-  }
-  if (neck) {
-    for (int bi = 0; bi < g.n_blocks; ++bi) {
-      ConvLayer L{};
-      L.kind = DECONV;
-      L.s = g.up_stride[bi];
-      L.cin = g.block_ch[bi];
-      L.cout = g.up_ch;
-      L.in_w = b.block_w[bi];
-      L.in_h = b.block_h[bi];
-      L.out_w = c->Wf;
-      L.out_h = c->Hf;
-      L.gw = L.in_w;
-      L.gh = L.in_h;
-      L.ldc = c->Cf;
-      L.choff = bi * g.up_ch;
-      L.bn = g.up_ch;
-      L.bk = (L.cin >= 64) ? 64 : 32;
-      L.n_tiles_n = L.s * L.s;
-      L.in = b.block_out[bi];
-      L.out = b.feat;
-      L.wpacked = c->wbufs[wi];
-      L.bias = c->bbufs[wi];
-      L.wait_layers = block_last[bi];                 // only its block's output
-      ++wi;
-      if (conv_make_maps(L, c->bf16) != cudaSuccess) return RTCC_E_CUDA;
-      b.layers.push_back(L);
-    }
-  }
-  // fp32 workspace of the global-memory split-K reduction (used when a split
-  // layer cannot reduce through DSMEM); deconvs do not wait on their
-  // predecessor, so they may not share it: they never split
-  size_t ws_floats = 0, max_tiles = 0;
-  for (ConvLayer& L : b.layers) {
-    const int m_tiles = ((L.gw + conv_tile_w() - 1) / conv_tile_w()) *
-                        ((L.gh + conv_tile_h() - 1) / conv_tile_h());
-    const int base = m_tiles * L.n_tiles_n;
-    if (L.kind == DECONV || L.splits < 1) L.splits = 1;
-    const int sp = L.splits;
-    if (sp > 1) {
-      ws_floats = std::max(ws_floats, (size_t)sp * base * conv_tile_m() * L.bn);
-      max_tiles = std::max(max_tiles, (size_t)base);
-    }
-  }
-  if (ws_floats) {
-    RS(dalloc(c, &b.splitk_ws, ws_floats * sizeof(float)));
-    RS(dalloc(c, &b.splitk_cnt, max_tiles * sizeof(int)));
-    CK(cudaMemset(b.splitk_cnt, 0, max_tiles * sizeof(int)));
-  }
-  for (ConvLayer& L : b.layers) {
-    L.ws = b.splitk_ws;
-    L.counters = b.splitk_cnt;
-  }
+  // the pseudo-image is agent k's part of the agent-major image tensor
+  p.image = static_cast<uint8_t*>(c->image_all) + (size_t)k * c->img_elems * 2;
   b.grid_bar = reinterpret_cast<unsigned*>(static_cast<uint8_t*>(b.frame_zero) + 8 * sizeof(int));
-  if (g.flags & RTCC_FLAG_LAYER_TIMES) {
-    RS(dalloc(c, &b.stamps, 2 * b.layers.size() * sizeof(unsigned long long)));
-    CK(cudaMemset(b.stamps, 0, 2 * b.layers.size() * sizeof(unsigned long long)));
-  }
-  b.bb = new (std::nothrow) BackboneParams;
-  if (!b.bb) return RTCC_E_NOMEM;
-  if (backbone_fill(b.layers, b.grid_bar, c->d_err, b.stamps,
-                    (g.flags & RTCC_FLAG_NO_CLUSTERS) == 0, b.bb) != cudaSuccess)
-    return RTCC_E_ARG;
   CK(cudaStreamCreateWithFlags(&b.st, cudaStreamNonBlocking));
   CK(cudaEventCreateWithFlags(&b.h2d_done, cudaEventDisableTiming));
   CK(cudaEventCreateWithFlags(&b.done, cudaEventDisableTiming));
+  CK(cudaEventCreateWithFlags(&b.pill_done, cudaEventDisableTiming));
   CK(cudaEventCreate(&b.ev_start));
   CK(cudaEventCreate(&b.ev_bb0));
   CK(cudaEventCreate(&b.ev_bb1));
   CK(cudaEventCreate(&b.ev_end));
+  return RTCC_OK;
+}
+
+// Branch k's own launch parameters (after build_backbone).
+rtcc_status build_branch_params(rtcc_ctx* c, int k) {
+  Branch& b = c->br[k];
+  b.feat = static_cast<uint8_t*>(c->feat_all) + (size_t)k * c->feat_elems * 2;
+  if (c->cfg.flags & RTCC_FLAG_LAYER_TIMES) {
+    RS(dalloc(c, &b.stamps, 2 * c->layers.size() * sizeof(unsigned long long)));
+    CK(cudaMemset(b.stamps, 0, 2 * c->layers.size() * sizeof(unsigned long long)));
+  }
+  b.bb = new (std::nothrow) BackboneParams;
+  if (!b.bb) return RTCC_E_NOMEM;
+  *b.bb = *c->bbt[1];
+  b.bb->agents[0] = k;
+  b.bb->grid_bar = b.grid_bar;
+  b.bb->stamps = b.stamps;
+  b.bb->done_word = c->done_words + k;
+  b.bb->stall = c->stall;
+  for (int l = 0; l < b.bb->n_layers; ++l) {
+    b.bb->L[l].ws = b.splitk_ws;
+    b.bb->L[l].counters = b.splitk_cnt;
+  }
   return RTCC_OK;
 }
 
@@ -537,9 +668,12 @@ cudaError_t record_node(cudaEvent_t ev, cudaStream_t st) {
   return cudaEventRecordWithFlags(ev, st, cudaEventRecordExternal);
 }
 
-rtcc_status capture_branch_graph(rtcc_ctx* c, int k, const PillarBufs& pb, cudaGraphExec_t* out) {
+// Branch k's graph: the per-frame words, the pillar chain, and (with_bb) the
+// backbone of this agent alone as a programmatic dependent of the PFN.
+rtcc_status capture_branch_graph(rtcc_ctx* c, int k, const PillarBufs& pb, bool with_bb,
+                                 cudaGraphExec_t* out) {
   Branch& b = c->br[k];
-  const bool tl = (c->cfg.flags & RTCC_FLAG_TIMELINE) != 0;
+  const bool tl = with_bb && (c->cfg.flags & RTCC_FLAG_TIMELINE) != 0;
   (void)cudaGetLastError();   // no stale error may leak into the launch checks
   GridGeom gg{c->cfg.x_min, c->cfg.y_min, c->cfg.z_min, c->cfg.z_max, c->cfg.pillar, c->W, c->H};
   CK(cudaStreamBeginCapture(b.st, cudaStreamCaptureModeRelaxed));
@@ -550,7 +684,7 @@ rtcc_status capture_branch_graph(rtcc_ctx* c, int k, const PillarBufs& pb, cudaG
   if (e == cudaSuccess) e = cudaMemsetAsync(b.frame_zero, 0, kFrameZeroBytes, b.st);
   if (e == cudaSuccess) e = launch_pillarise(pb, gg, c->pfn_w, c->pfn_b, c->bf16, c->d_err, b.st);
   if (e == cudaSuccess && tl) e = record_node(b.ev_bb0, b.st);
-  if (e == cudaSuccess) e = launch_backbone(*b.bb, c->bf16, b.st);
+  if (e == cudaSuccess && with_bb) e = launch_backbone(*b.bb, c->bf16, b.st);
   if (e == cudaSuccess && tl) e = record_node(b.ev_bb1, b.st);
   if (e == cudaSuccess && tl) e = record_node(b.ev_end, b.st);
   cudaGraph_t graph = nullptr;
@@ -564,19 +698,23 @@ rtcc_status capture_branch_graph(rtcc_ctx* c, int k, const PillarBufs& pb, cudaG
   return e == cudaSuccess ? RTCC_OK : RTCC_E_CUDA;
 }
 
-// Two graphs per branch: one for payloads already in the device slot, and
-// one whose first kernel reads the payload from the pinned staging buffer
-// (over the host link) and copies it into the device slot as it goes, so a
-// host payload needs no copy-engine transfer and no cross-stream event.
+// Four graphs per branch: with and without the backbone (a branch released
+// alone runs its own; branches released together share one batched launch),
+// each for a payload already in the device slot and for one whose first
+// kernel reads the payload from the pinned staging buffer (over the host
+// link) and copies it into the device slot as it goes, so a host payload
+// needs no copy-engine transfer and no cross-stream event.
 rtcc_status capture_branch(rtcc_ctx* c, int k) {
   Branch& b = c->br[k];
-  RS(capture_branch_graph(c, k, b.pb, &b.exec));
   PillarBufs ph = b.pb;
   ph.src_hdr = reinterpret_cast<const int*>(b.staging);
   ph.src_pts = reinterpret_cast<const float4*>(reinterpret_cast<const uint8_t*>(b.staging) + kHdrBytes);
   ph.dst_hdr = reinterpret_cast<int*>(b.in_dev);
   ph.dst_pts = reinterpret_cast<float4*>(b.in_dev + kHdrBytes);
-  return capture_branch_graph(c, k, ph, &b.exec_host);
+  RS(capture_branch_graph(c, k, b.pb, true, &b.exec));
+  RS(capture_branch_graph(c, k, ph, true, &b.exec_host));
+  RS(capture_branch_graph(c, k, b.pb, false, &b.pill));
+  return capture_branch_graph(c, k, ph, false, &b.pill_host);
 }
 
 rtcc_status capture_post(rtcc_ctx* c) {
@@ -680,22 +818,41 @@ rtcc_status capture_post(rtcc_ctx* c) {
 }
 
 void free_all(rtcc_ctx* c) {
+  if (c->disp.joinable()) {
+    {
+      std::lock_guard<std::mutex> lk(c->mu);
+      c->stop = true;
+    }
+    c->cv.notify_all();
+    c->disp.join();
+  }
   for (int k = 0; k < RTCC_MAX_AGENTS; ++k) {
     Branch& b = c->br[k];
     if (b.st) cudaStreamSynchronize(b.st);
-    if (b.exec) cudaGraphExecDestroy(b.exec);
-    if (b.exec_host) cudaGraphExecDestroy(b.exec_host);
-    for (cudaEvent_t ev : {b.h2d_done, b.done, b.ev_start, b.ev_bb0, b.ev_bb1, b.ev_end})
+    for (cudaGraphExec_t g : {b.exec, b.exec_host, b.pill, b.pill_host})
+      if (g) cudaGraphExecDestroy(g);
+    for (cudaEvent_t ev : {b.h2d_done, b.done, b.pill_done, b.ev_start, b.ev_bb0, b.ev_bb1, b.ev_end})
       if (ev) cudaEventDestroy(ev);
     delete b.bb;
     b.bb = nullptr;
     if (b.st) cudaStreamDestroy(b.st);
   }
+  if (c->bbst) cudaStreamSynchronize(c->bbst);
   if (c->post) cudaStreamSynchronize(c->post);
   if (c->xfer) cudaStreamSynchronize(c->xfer);
   if (c->post_exec) cudaGraphExecDestroy(c->post_exec);
   for (cudaEvent_t ev : {c->det_ready, c->ev_post0, c->ev_fuse0, c->ev_fuse1, c->ev_post1})
     if (ev) cudaEventDestroy(ev);
+  for (int j = 0; j < RTCC_MAX_AGENTS; ++j)
+    for (cudaEvent_t ev : {c->batch_ev[j], c->batch_t0[j], c->batch_t1[j]})
+      if (ev) cudaEventDestroy(ev);
+  for (int n = 0; n <= RTCC_MAX_AGENTS; ++n) {
+    delete c->bbt[n];
+    c->bbt[n] = nullptr;
+  }
+  delete c->launch_p;
+  c->launch_p = nullptr;
+  if (c->bbst) cudaStreamDestroy(c->bbst);
   if (c->post) cudaStreamDestroy(c->post);
   if (c->xfer) cudaStreamDestroy(c->xfer);
   for (void* p : c->allocs) cudaFree(p);
@@ -703,6 +860,8 @@ void free_all(rtcc_ctx* c) {
   c->allocs.clear();
   c->host_allocs.clear();
 }
+
+void dispatcher_main(rtcc_ctx* c);
 
 rtcc_status init_impl(rtcc_ctx* c, const float* weights) {
   const rtcc_model_config& g = c->cfg;
@@ -715,7 +874,25 @@ rtcc_status init_impl(rtcc_ctx* c, const float* weights) {
   CK(cudaMemset(c->d_err, 0, 16));
   RS(dalloc(c, &c->d_present, RTCC_MAX_AGENTS * 4));
   CK(cudaMemset(c->d_present, 0, RTCC_MAX_AGENTS * 4));
+  {
+    int* d = nullptr;
+    RS(halloc(c, &d, 2 * RTCC_MAX_AGENTS * sizeof(int)));
+    for (int i = 0; i < 2 * RTCC_MAX_AGENTS; ++i) d[i] = 1;
+    c->done_words = d;
+    if (g.flags & RTCC_FLAG_SHORT_WAITS) {
+      int* s = nullptr;
+      RS(halloc(c, &s, sizeof(int)));
+      *s = 0;
+      c->stall = s;
+    }
+  }
+  const size_t img = (size_t)c->W * c->H * c->Cp;
+  RS(dalloc(c, &c->image_all, (size_t)c->K * img * 2));
+  CK(cudaMemset(c->image_all, 0, (size_t)c->K * img * 2));
+  c->img_elems = img;
   for (int k = 0; k < c->K; ++k) RS(build_branch(c, k));
+  RS(build_backbone(c));
+  for (int k = 0; k < c->K; ++k) RS(build_branch_params(c, k));
   const int cells_f = c->Wf * c->Hf;
   RS(dalloc(c, &c->d_feat_ptrs, RTCC_MAX_AGENTS * sizeof(void*)));
   void* fp[RTCC_MAX_AGENTS] = {};
@@ -750,55 +927,169 @@ rtcc_status init_impl(rtcc_ctx* c, const float* weights) {
   }
   CK(cudaStreamCreateWithFlags(&c->xfer, cudaStreamNonBlocking));
   CK(cudaStreamCreateWithFlags(&c->post, cudaStreamNonBlocking));
+  CK(cudaStreamCreateWithFlags(&c->bbst, cudaStreamNonBlocking));
   CK(cudaEventCreateWithFlags(&c->det_ready, cudaEventDisableTiming));
   CK(cudaEventCreate(&c->ev_post0));
   CK(cudaEventCreate(&c->ev_fuse0));
   CK(cudaEventCreate(&c->ev_fuse1));
   CK(cudaEventCreate(&c->ev_post1));
+  for (int j = 0; j < RTCC_MAX_AGENTS; ++j) {
+    CK(cudaEventCreateWithFlags(&c->batch_ev[j], cudaEventDisableTiming));
+    CK(cudaEventCreate(&c->batch_t0[j]));
+    CK(cudaEventCreate(&c->batch_t1[j]));
+  }
   for (int k = 0; k < c->K; ++k) RS(capture_branch(c, k));
   RS(capture_post(c));
-  // warm-up: every graph once on empty payloads (pays first-launch costs)
+  // warm-up: every graph once on empty payloads (pays first-launch costs),
+  // and one batched launch of every batch size
   for (int k = 0; k < c->K; ++k) CK(cudaGraphLaunch(c->br[k].exec, c->br[k].st));
   for (int k = 0; k < c->K; ++k) CK(cudaGraphLaunch(c->br[k].exec_host, c->br[k].st));
+  for (int k = 0; k < c->K; ++k) CK(cudaGraphLaunch(c->br[k].pill, c->br[k].st));
   for (int k = 0; k < c->K; ++k) CK(cudaStreamSynchronize(c->br[k].st));
+  for (int n = 2; n <= c->K; ++n) {
+    *c->launch_p = *c->bbt[n];
+    c->launch_p->stall = nullptr;
+    CK(launch_backbone(*c->launch_p, c->bf16, c->bbst));
+  }
+  CK(cudaStreamSynchronize(c->bbst));
   CK(cudaGraphLaunch(c->post_exec, c->post));
   CK(cudaStreamSynchronize(c->post));
   int herr = 0;
   CK(cudaMemcpy(&herr, c->d_err, 4, cudaMemcpyDeviceToHost));
-  return herr ? RTCC_E_DEVICE : RTCC_OK;
+  if (herr) return RTCC_E_DEVICE;
+  if (!(g.flags & RTCC_FLAG_NO_BATCH)) {
+    c->disp = std::thread(dispatcher_main, c);
+  }
+  return RTCC_OK;
 }
 
-// Launch branch k: H2D of its payload on the transfer stream (unless the input
-// is resident), an event gating the branch stream, the branch graph, and the
-// branch's completion event.  Called with the context mutex held.
-rtcc_status launch_branch(rtcc_ctx* c, int k) {
+// Make agent k's payload available to its first kernel.  Returns whether the
+// branch graphs that read the pinned staging buffer (zero-copy) are to be
+// used; with RTCC_FLAG_H2D_COPY the payload is instead copied to the device
+// slot by the copy engine on the transfer stream, and the branch stream waits
+// for that copy's event (the release path of Sec. IV-F as written).
+rtcc_status stage_payload(rtcc_ctx* c, int k, bool* host_variant) {
   Branch& b = c->br[k];
-  if (!b.pend_resident) {
-    // the branch's first kernel reads the payload from the pinned staging
-    // buffer and copies it to the device slot (no copy engine, no event)
-    const int n = b.pend_n;
-    float* pts = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(b.staging) + kHdrBytes);
-    if (n > 0 && b.pend_ptr != pts) std::memcpy(pts, b.pend_ptr, (size_t)n * 16);
-    *reinterpret_cast<volatile int*>(b.staging) = n;
-    std::atomic_thread_fence(std::memory_order_seq_cst);
-    CK(cudaGraphLaunch(b.exec_host, b.st));
-  } else {
-    CK(cudaGraphLaunch(b.exec, b.st));
+  *host_variant = false;
+  if (b.pend_resident) return RTCC_OK;
+  const int n = b.pend_n;
+  float* pts = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(b.staging) + kHdrBytes);
+  if (n > 0 && b.pend_ptr != pts) std::memcpy(pts, b.pend_ptr, (size_t)n * 16);
+  *reinterpret_cast<volatile int*>(b.staging) = n;
+  std::atomic_thread_fence(std::memory_order_seq_cst);
+  if (c->cfg.flags & RTCC_FLAG_H2D_COPY) {
+    CK(cudaMemcpyAsync(b.in_dev, b.staging, kHdrBytes + (size_t)n * 16, cudaMemcpyHostToDevice, c->xfer));
+    CK(cudaEventRecord(b.h2d_done, c->xfer));
+    CK(cudaStreamWaitEvent(b.st, b.h2d_done, 0));
+    return RTCC_OK;
   }
-  CK(cudaEventRecord(b.done, b.st));
+  *host_variant = true;
+  return RTCC_OK;
+}
+
+void note_dispatch(rtcc_ctx* c, int k) {
+  Branch& b = c->br[k];
   b.launched = true;
   c->ctrl.mark(k, RTCC_RUNNING);
   c->present_dirty = true;
   c->info.t_release_ms[k] = now_ms();
   if (c->info.n_dispatched < RTCC_MAX_AGENTS) c->info.dispatch_order[c->info.n_dispatched++] = k;
+}
+
+void note_launch(rtcc_ctx* c, int word, int size) {
+  if (c->n_launches < RTCC_MAX_AGENTS) {
+    c->launch_size[c->n_launches] = size;
+    c->launch_word[c->n_launches] = word;
+  }
+  ++c->n_launches;
+  c->inflight = word;
+}
+
+// Branch k released alone: pillar chain and its own backbone (one graph).
+// Called with the context mutex held, as are the launches below.
+rtcc_status launch_full(rtcc_ctx* c, int k) {
+  Branch& b = c->br[k];
+  bool hv = false;
+  RS(stage_payload(c, k, &hv));
+  c->done_words[k] = 0;
+  CK(cudaGraphLaunch(hv ? b.exec_host : b.exec, b.st));
+  CK(cudaEventRecord(b.done, b.st));
+  b.feat_ev = b.done;
+  b.stamp_src = k;
+  b.launch_idx = c->n_launches;
+  b.full_graph = true;
+  note_launch(c, k, 1);
+  note_dispatch(c, k);
   return RTCC_OK;
 }
+
+// Branch k's pillar chain alone; its backbone joins a batch.
+rtcc_status launch_pill(rtcc_ctx* c, int k) {
+  Branch& b = c->br[k];
+  bool hv = false;
+  RS(stage_payload(c, k, &hv));
+  CK(cudaGraphLaunch(hv ? b.pill_host : b.pill, b.st));
+  CK(cudaEventRecord(b.pill_done, b.st));
+  c->pending.push_back(k);
+  note_dispatch(c, k);
+  return RTCC_OK;
+}
+
+// One backbone launch for every pending agent (their pillar chains are
+// already enqueued).  One agent: its own launch parameters, on its own stream
+// behind its pillar chain.  Several: the batch template for that count, on
+// the batch stream after every chain's event; each agent still writes its
+// own slot, and its result does not depend on the batch (see pick_bn_batch).
+rtcc_status launch_batch(rtcc_ctx* c) {
+  std::vector<int> ag = c->pending;
+  c->pending.clear();
+  if (ag.empty()) return RTCC_OK;
+  std::sort(ag.begin(), ag.end());
+  const bool tl = (c->cfg.flags & RTCC_FLAG_TIMELINE) != 0;
+  const int n = (int)ag.size();
+  if (n == 1) {
+    Branch& b = c->br[ag[0]];
+    c->done_words[ag[0]] = 0;
+    if (tl) CK(cudaEventRecord(b.ev_bb0, b.st));
+    CK(launch_backbone(*b.bb, c->bf16, b.st));
+    if (tl) CK(cudaEventRecord(b.ev_bb1, b.st));
+    CK(cudaEventRecord(b.done, b.st));
+    b.feat_ev = b.done;
+    b.stamp_src = ag[0];
+    b.launch_idx = c->n_launches;
+    note_launch(c, ag[0], 1);
+    return RTCC_OK;
+  }
+  const int j = std::min(c->n_launches, RTCC_MAX_AGENTS - 1);
+  const int word = RTCC_MAX_AGENTS + j;
+  BackboneParams& P = *c->launch_p;
+  P = *c->bbt[n];
+  for (int i = 0; i < n; ++i) P.agents[i] = ag[i];
+  P.stamps = c->br[ag[0]].stamps;
+  P.done_word = c->done_words + word;
+  P.stall = c->stall;
+  for (int k : ag) CK(cudaStreamWaitEvent(c->bbst, c->br[k].pill_done, 0));
+  c->done_words[word] = 0;
+  if (tl) CK(cudaEventRecord(c->batch_t0[j], c->bbst));
+  CK(launch_backbone(P, c->bf16, c->bbst));
+  if (tl) CK(cudaEventRecord(c->batch_t1[j], c->bbst));
+  CK(cudaEventRecord(c->batch_ev[j], c->bbst));
+  for (int k : ag) {
+    c->br[k].feat_ev = c->batch_ev[j];
+    c->br[k].stamp_src = ag[0];
+    c->br[k].launch_idx = c->n_launches;
+  }
+  note_launch(c, word, n);
+  return RTCC_OK;
+}
+
+bool backbone_busy(const rtcc_ctx* c) { return c->inflight >= 0 && c->done_words[c->inflight] == 0; }
 
 rtcc_status launch_post(rtcc_ctx* c) {
   // the presence flags are set on the device by the branches that ran (their
   // first kernel) and cleared by the decode kernel
   for (int k = 0; k < c->K; ++k)
-    if (c->ctrl.present(k)) CK(cudaStreamWaitEvent(c->post, c->br[k].done, 0));
+    if (c->ctrl.present(k)) CK(cudaStreamWaitEvent(c->post, c->br[k].feat_ev, 0));
   *c->h_done = 0;                                 // the decode kernel sets it when the boxes are written
   std::atomic_thread_fence(std::memory_order_seq_cst);
   CK(cudaGraphLaunch(c->post_exec, c->post));
@@ -809,13 +1100,57 @@ rtcc_status launch_post(rtcc_ctx* c) {
 
 // Dispatch what an event made ready; launch the post-join once every branch
 // is resolved.  `t_entry` is the host time the event call began.
+//
+// Batching (unless RTCC_FLAG_NO_BATCH): a branch released while the GPU is
+// free starts at once with its own backbone; one released while a backbone
+// is still running enqueues only its pillar chain and waits in `pending`.
+// When the running backbone ends, the dispatcher thread launches one backbone
+// over every pending agent.  Agents released by one event (Barrier's release
+// of all branches at A) form one batch.  Once the last branch is resolved no
+// later release can join a batch, so whatever is pending is launched at once,
+// queued behind the running backbone, followed by the post-join.
 rtcc_status after_event(rtcc_ctx* c, const std::vector<int>& released, double t_entry) {
-  for (int k : released) RS(launch_branch(c, k));
-  if (c->ctrl.join_ready() && !c->post_launched) {
+  const bool batching = (c->cfg.flags & RTCC_FLAG_NO_BATCH) == 0;
+  const bool last = c->ctrl.join_ready();
+  if (!batching) {
+    for (int k : released) RS(launch_full(c, k));
+  } else if (released.size() == 1 && c->pending.empty() && !backbone_busy(c)) {
+    RS(launch_full(c, released[0]));
+  } else if (!released.empty()) {
+    for (int k : released) RS(launch_pill(c, k));
+    if (released.size() > 1 || last || !backbone_busy(c)) RS(launch_batch(c));
+    else c->cv.notify_all();
+  }
+  if (last && !c->post_launched) {
+    if (!c->pending.empty()) RS(launch_batch(c));
     c->t_last_event = t_entry;
     RS(launch_post(c));
   }
   return RTCC_OK;
+}
+
+// Launches the pending batch once the backbone in flight has ended (see
+// after_event).  Waits for the end on the launch's done word in pinned host
+// memory, without the context mutex.
+void dispatcher_main(rtcc_ctx* c) {
+  cudaSetDevice(c->dev);
+  std::unique_lock<std::mutex> lk(c->mu);
+  while (true) {
+    c->cv.wait(lk, [c] { return c->stop || !c->pending.empty(); });
+    if (c->stop) break;
+    const int w = c->inflight;
+    lk.unlock();
+    const double t0 = now_ms();
+    for (uint32_t it = 1; w >= 0 && c->done_words[w] == 0; ++it) {
+      // a launch that never reports its end (it failed) stops holding the batch back
+      if ((it & 1023u) == 0 && now_ms() - t0 > 2000.0) break;
+    }
+    lk.lock();
+    if (c->stop) break;
+    if (!c->pending.empty() && c->inflight == w) {
+      if (launch_batch(c) != RTCC_OK) c->disp_err = true;
+    }
+  }
 }
 
 }  // namespace
@@ -840,6 +1175,7 @@ rtcc_status rtcc_init(const rtcc_model_config* cfg, const float* weights, size_t
                                             cfg->fusion == RTCC_FUSE_ATTN);
   if (!c) return RTCC_E_NOMEM;
   c->cfg = *cfg;
+  c->dev = dev;
   c->bf16 = cfg->dtype == RTCC_BF16;
   c->K = cfg->n_agents;
   c->W = cfg->grid_w;
@@ -913,10 +1249,13 @@ rtcc_status rtcc_frame_begin(rtcc_ctx* c, uint64_t frame_id, double t0_ms) {
     // a previous frame launched branches but ran no post-join to clear their
     // presence flags
     for (int k = 0; k < c->K; ++k) CK(cudaStreamSynchronize(c->br[k].st));
+    CK(cudaStreamSynchronize(c->bbst));
     CK(cudaMemset(c->d_present, 0, RTCC_MAX_AGENTS * 4));
     c->present_dirty = false;
   }
   c->post_launched = false;
+  c->n_launches = 0;
+  c->pending.clear();
   c->t_last_event = 0.0;
   std::memset(&c->info, 0, sizeof(c->info));
   for (int k = 0; k < RTCC_MAX_AGENTS; ++k) {
@@ -925,6 +1264,10 @@ rtcc_status rtcc_frame_begin(rtcc_ctx* c, uint64_t frame_id, double t0_ms) {
     c->info.gpu_branch_ms[k] = -1.f;
     c->info.t_release_ms[k] = NAN;
     c->br[k].launched = false;
+    c->br[k].feat_ev = nullptr;
+    c->br[k].stamp_src = -1;
+    c->br[k].launch_idx = -1;
+    c->br[k].full_graph = false;
   }
   c->info.gpu_fusion_ms = -1.f;
   c->info.gpu_post_ms = -1.f;
@@ -983,8 +1326,13 @@ rtcc_status rtcc_wait_detection(rtcc_ctx* c, int32_t timeout_ms, rtcc_box* out, 
     std::lock_guard<std::mutex> lk(c->mu);
     if (!c->ctrl.frame_open()) return RTCC_E_STATE;
     if (c->ctrl.aborted()) {
+      // branches already released finish; a batch still held back is
+      // launched now so that its pillar chains' work is not left half done
+      const rtcc_status ls = launch_batch(c);
       for (int k = 0; k < c->K; ++k)
         if (c->br[k].launched) cudaStreamSynchronize(c->br[k].st);
+      cudaStreamSynchronize(c->bbst);
+      if (ls != RTCC_OK) return ls;
       // no decode ran to clear the presence flags of the branches that did
       if (cudaMemset(c->d_present, 0, RTCC_MAX_AGENTS * 4) != cudaSuccess) return RTCC_E_CUDA;
       c->present_dirty = false;
@@ -1024,13 +1372,31 @@ rtcc_status rtcc_wait_detection(rtcc_ctx* c, int32_t timeout_ms, rtcc_box* out, 
   if (t_ready_ms) *t_ready_ms = t_ready;
   c->info.t_ready_ms = t_ready;
   c->info.t_last_event_ms = c->t_last_event;
+  c->info.n_backbone_launches = c->n_launches;
+  for (int j = 0; j < RTCC_MAX_AGENTS; ++j) {
+    c->info.backbone_batch[j] = j < c->n_launches ? c->launch_size[j] : 0;
+    c->info.gpu_launch_ms[j] = -1.f;
+  }
   if (c->cfg.flags & RTCC_FLAG_TIMELINE) {
+    for (int j = 0; j < c->n_launches && j < RTCC_MAX_AGENTS; ++j) {
+      float ms = -1.f;
+      const int w = c->launch_word[j];
+      if (w >= RTCC_MAX_AGENTS) {
+        if (cudaEventElapsedTime(&ms, c->batch_t0[w - RTCC_MAX_AGENTS], c->batch_t1[w - RTCC_MAX_AGENTS]) ==
+            cudaSuccess)
+          c->info.gpu_launch_ms[j] = ms;
+      } else if (cudaEventElapsedTime(&ms, c->br[w].ev_bb0, c->br[w].ev_bb1) == cudaSuccess) {
+        c->info.gpu_launch_ms[j] = ms;
+      }
+    }
     for (int k = 0; k < c->K; ++k) {
       Branch& b = c->br[k];
       if (!b.launched) continue;
       float ms = -1.f;
-      if (cudaEventElapsedTime(&ms, b.ev_bb0, b.ev_bb1) == cudaSuccess) c->info.gpu_backbone_ms[k] = ms;
-      if (cudaEventElapsedTime(&ms, b.ev_start, b.ev_end) == cudaSuccess) c->info.gpu_branch_ms[k] = ms;
+      if (b.launch_idx >= 0 && b.launch_idx < RTCC_MAX_AGENTS)
+        c->info.gpu_backbone_ms[k] = c->info.gpu_launch_ms[b.launch_idx];
+      if (b.full_graph && cudaEventElapsedTime(&ms, b.ev_start, b.ev_end) == cudaSuccess)
+        c->info.gpu_branch_ms[k] = ms;
       unsigned long long ps[2] = {0ull, 0ull};
       if (b.pb.pfn_span && cudaMemcpy(ps, b.pb.pfn_span, sizeof(ps), cudaMemcpyDeviceToHost) == cudaSuccess &&
           ps[1] > ps[0])
@@ -1046,7 +1412,27 @@ rtcc_status rtcc_wait_detection(rtcc_ctx* c, int32_t timeout_ms, rtcc_box* out, 
     (void)cudaGetLastError();
   }
   c->ctrl.end();
-  return hdr->err ? RTCC_E_DEVICE : RTCC_OK;
+  if (c->stall) *c->stall = 0;                 // the test hook lasts one frame
+  if (c->disp_err) {
+    c->disp_err = false;
+    return RTCC_E_CUDA;
+  }
+  if (hdr->err) {
+    // A bounded device wait ran out.  The frame's kernels have all ended (the
+    // post-join waited for them); clear the error word and the split-K tile
+    // counters a kernel that wound down may have left, so the next frame
+    // starts clean.
+    for (int k = 0; k < c->K; ++k) cudaStreamSynchronize(c->br[k].st);
+    cudaStreamSynchronize(c->bbst);
+    cudaStreamSynchronize(c->post);
+    CK(cudaMemset(c->d_err, 0, 16));
+    for (int k = 0; k < c->K; ++k)
+      if (c->br[k].splitk_cnt) CK(cudaMemset(c->br[k].splitk_cnt, 0, c->splitk_cnt_bytes));
+    if (c->batch_cnt) CK(cudaMemset(c->batch_cnt, 0, (size_t)c->K * c->splitk_cnt_bytes));
+    CK(cudaMemset(c->batch_bar, 0, (kMaxLayers + 1) * sizeof(unsigned)));
+    return RTCC_E_DEVICE;
+  }
+  return RTCC_OK;
 }
 
 rtcc_status rtcc_get_frame_info(rtcc_ctx* c, rtcc_frame_info* info) {
@@ -1061,12 +1447,14 @@ rtcc_status rtcc_get_layer_spans(rtcc_ctx* c, int32_t agent, float* start_ms, fl
   if (!c) return RTCC_E_ARG;
   std::lock_guard<std::mutex> lk(c->mu);
   if (agent < 0 || agent >= c->K) return RTCC_E_AGENT;
-  Branch& b = c->br[agent];
-  if (!b.stamps) return RTCC_E_STATE;
-  const int n = (int)b.layers.size();
+  if (!c->br[agent].stamps) return RTCC_E_STATE;
+  const int n = (int)c->layers.size();
   if (n_out) *n_out = n;
   if (!start_ms && !end_ms) return RTCC_OK;
+  // the stamps of the launch that ran this agent (alone or in a batch)
+  Branch& b = c->br[c->br[agent].stamp_src >= 0 ? c->br[agent].stamp_src : agent];
   CK(cudaStreamSynchronize(b.st));
+  CK(cudaStreamSynchronize(c->bbst));
   std::vector<unsigned long long> t(2 * n);
   CK(cudaMemcpy(t.data(), b.stamps, 2 * n * sizeof(unsigned long long), cudaMemcpyDeviceToHost));
   unsigned long long t0 = 0;
@@ -1099,8 +1487,8 @@ rtcc_status rtcc_get_branch_state(rtcc_ctx* c, int32_t agent, int32_t* state, do
     // observe FINISHED lazily through the branch's completion event
     int st = 0;
     c->ctrl.state(agent, &st, nullptr);
-    if (st == RTCC_RUNNING && cudaEventQuery(c->br[agent].done) == cudaSuccess)
-      c->ctrl.mark(agent, RTCC_FINISHED);
+    const cudaEvent_t fe = c->br[agent].feat_ev;
+    if (st == RTCC_RUNNING && fe && cudaEventQuery(fe) == cudaSuccess) c->ctrl.mark(agent, RTCC_FINISHED);
   }
   int32_t st = 0;
   rtcc_status s = c->ctrl.state(agent, &st, release_ms);
@@ -1189,19 +1577,20 @@ rtcc_status rtcc_get_tensor(rtcc_ctx* c, int32_t agent, int32_t which, uint16_t*
     if (agent < 0 || agent >= c->K) return RTCC_E_AGENT;
     Branch& b = c->br[agent];
     CK(cudaStreamSynchronize(b.st));
+    CK(cudaStreamSynchronize(c->bbst));
     if (which == 0) {
       src = b.pb.image;
       n = (size_t)c->W * c->H * c->Cp;
     } else if (which >= 1 && which <= c->cfg.n_blocks) {
-      src = b.block_out[which - 1];
-      n = (size_t)b.block_w[which - 1] * b.block_h[which - 1] * c->cfg.block_ch[which - 1];
+      n = (size_t)c->block_w[which - 1] * c->block_h[which - 1] * c->cfg.block_ch[which - 1];
+      src = static_cast<const uint8_t*>(c->block_out[which - 1]) + (size_t)agent * n * 2;
     } else if (which == 8) {
       src = b.feat;
       n = (size_t)c->Wf * c->Hf * c->Cf;
-    } else if (which >= 16 && which - 16 < (int)b.layer_out.size() &&
+    } else if (which >= 16 && which - 16 < (int)c->layer_all.size() &&
                (c->cfg.flags & RTCC_FLAG_KEEP_LAYERS)) {
-      src = b.layer_out[which - 16];
-      n = b.layer_elems[which - 16];
+      n = c->layer_elems[which - 16];
+      src = static_cast<const uint8_t*>(c->layer_all[which - 16]) + (size_t)agent * n * 2;
     } else {
       return RTCC_E_ARG;
     }
@@ -1235,8 +1624,20 @@ double rtcc_now_ms(void) { return now_ms(); }
 
 int32_t rtcc_kernels_per_frame(rtcc_ctx* c, int32_t n_present) {
   if (!c) return 0;
-  // pillar chain + backbone per branch; fusion, decode (and NMS)
-  return n_present * (5 + 1) + 2 + (c->dec_boxes ? 1 : 0);
+  std::lock_guard<std::mutex> lk(c->mu);
+  // pillar chain per branch; the backbone launches of the last frame (one per
+  // branch when none was batched); fusion, decode (and NMS)
+  const int bb = c->n_launches > 0 ? c->n_launches : n_present;
+  return n_present * 5 + bb + 2 + (c->dec_boxes ? 1 : 0);
+}
+
+rtcc_status rtcc_test_unreachable_wait(rtcc_ctx* c) {
+  if (!c) return RTCC_E_ARG;
+  std::lock_guard<std::mutex> lk(c->mu);
+  if (!c->stall) return RTCC_E_STATE;
+  if (c->ctrl.frame_open()) return RTCC_E_STATE;
+  *c->stall = 1;
+  return RTCC_OK;
 }
 
 rtcc_status rtcc_nms(const rtcc_box* host_in, int32_t n, float iou, rtcc_box* host_out,

@@ -121,7 +121,7 @@ __device__ __forceinline__ unsigned atom_add_release_gpu(unsigned* ctr, unsigned
 }
 
 // Wait until the grid-wide arrival counter reaches `target` (bounded).
-__device__ __forceinline__ bool grid_wait(const unsigned* ctr, unsigned target) {
+__device__ __forceinline__ bool grid_wait(const unsigned* ctr, unsigned target, long long budget) {
   unsigned v;
   asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
   if (v >= target) return true;
@@ -130,7 +130,7 @@ __device__ __forceinline__ bool grid_wait(const unsigned* ctr, unsigned target) 
     __nanosleep(64);
     asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
     if (v >= target) return true;
-    if (clock64() - t0 > kWaitBudgetCycles) return false;
+    if (clock64() - t0 > budget) return false;
   }
 }
 
@@ -154,10 +154,14 @@ struct LayerScalars {
                            // kBBytes / (bn * 128) taps into one stage, others 1 (A + B)
   int spc;                 // halo layers: stages per 64-channel chunk (a stage never spans
                            // two chunks)
-  void* out;               // output [.][ow][ldc], 16-bit
+  void* out;               // output [agent][.][ow][ldc], 16-bit
+  long long out_astride;   // elements between agents in out
   int ow, ldc, gw, gh;     // output row length (pixels), pixel stride (channels), tile grid extent
+  int ipa;                 // items per agent
+  int deconv_idx;
+  int n_batch;
 };
-__device__ __forceinline__ LayerScalars layer_scalars(const LayerDesc& D) {
+__device__ __forceinline__ LayerScalars layer_scalars(const LayerDesc& D, int n_batch) {
   LayerScalars S;
   S.bias = D.bias;
   S.ws = D.ws;
@@ -180,13 +184,17 @@ __device__ __forceinline__ LayerScalars layer_scalars(const LayerDesc& D) {
   S.wait_items = D.wait_items;
   S.halo = D.halo;
   S.out = D.out;
+  S.out_astride = D.out_astride;
+  S.ipa = D.ipa;
+  S.deconv_idx = D.deconv_idx;
+  S.n_batch = n_batch;
   S.ow = D.ow;
   S.ldc = D.ldc;
   S.gw = D.gw;
   S.gh = D.gh;
   S.kpb = S.halo ? kBBytes / (S.bn * 128) : 1;
   S.spc = (9 + S.kpb - 1) / S.kpb;
-  S.n_items = S.m_tiles * S.n_tiles * S.splits;
+  S.n_items = n_batch * S.ipa;
   S.ncb_log2 = __ffs(S.cin / S.bk) - 1;            // cin / bk is a power of two
   S.total_kb = (S.kind == DECONV ? 1 : 9) << S.ncb_log2;
   return S;
@@ -200,15 +208,20 @@ __device__ __forceinline__ int first_item(const LayerScalars& S) {
   return b - S.cta_lo < S.n_items ? b - S.cta_lo : -1;
 }
 
-// Work item t of a layer -> (tile = (m tile, n tile), K slice z), its tile
-// origin and its k-block range [kb0, kb1).  The slice index runs fastest, so
-// the slices of a tile are consecutive items: with one item per CTA and a
-// grid of clusters of kMaxSplits CTAs they share a cluster, slice z on rank z.
+// Work item t of a layer -> (batch slot j, tile = (m tile, n tile), K slice
+// z), its agent, its tile origin and its k-block range [kb0, kb1).  Items
+// run agent-major, and within an agent the slice index runs fastest, so the
+// slices of a tile are consecutive items: with one item per CTA and a grid of
+// clusters of kMaxSplits CTAs they share a cluster, slice z on rank z (an
+// agent's item count is a multiple of the slice count).
 struct Item {
-  int x0, y0, n0, z, tile, kb0, kb1;
+  int x0, y0, n0, z, tile, kb0, kb1, slot, agent;
 };
-__device__ __forceinline__ Item item_of(const LayerScalars& S, int t) {
+__device__ __forceinline__ Item item_of(const LayerScalars& S, int t, const int* agents) {
   Item it;
+  it.slot = t / S.ipa;
+  it.agent = agents[it.slot];
+  t -= it.slot * S.ipa;
   it.z = t % S.splits;
   it.tile = t / S.splits;
   const int mt = it.tile % S.m_tiles;
@@ -245,7 +258,7 @@ __device__ __forceinline__ void load_a(const LayerScalars& S, const CUtensorMap*
   const int cb = kb - (tap << S.ncb_log2);
   if (S.kind == CONV3_S1) {
     const int dy = tap / 3, dx = tap - 3 * (tap / 3);
-    tma_load_4d(dA, map, bar, cb * S.bk, I.x0 + dx - 1, I.y0 + dy - 1, 0);
+    tma_load_4d(dA, map, bar, cb * S.bk, I.x0 + dx - 1, I.y0 + dy - 1, I.agent);
   } else if (S.kind == CONV3_S2) {
     // input x = 2*ox + dx - 1 = 2*j + p; input y = 2*oy + dy - 1 = 2*i + q
     const int dy = tap / 3, dx = tap - 3 * (tap / 3);
@@ -253,9 +266,9 @@ __device__ __forceinline__ void load_a(const LayerScalars& S, const CUtensorMap*
     const int p = (dx == 1) ? 0 : 1;
     const int i = I.y0 + (dy == 0 ? -1 : 0);
     const int q = (dy == 1) ? 0 : 1;
-    tma_load_5d(dA, map, bar, p * S.cin + cb * S.bk, j, q, i, 0);
+    tma_load_5d(dA, map, bar, p * S.cin + cb * S.bk, j, q, i, I.agent);
   } else {
-    tma_load_4d(dA, map, bar, cb * S.bk, I.x0, I.y0, 0);
+    tma_load_4d(dA, map, bar, cb * S.bk, I.x0, I.y0, I.agent);
   }
 }
 
@@ -280,7 +293,7 @@ __device__ __forceinline__ void load_b(const LayerScalars& S, const CUtensorMap*
 // memory address, so a start at any 128-byte row matches the TMA placement.
 __device__ __forceinline__ void load_halo(const CUtensorMap* map, uint8_t* dH, uint64_t* bar,
                                           const Item& I, int cb) {
-  tma_load_4d(dH, map, bar, cb * 64, I.x0 - 1, I.y0 - 1, 0);
+  tma_load_4d(dH, map, bar, cb * 64, I.x0 - 1, I.y0 - 1, I.agent);
 }
 
 // One k-block of MMAs (BK = 64 or 32 -> 4 or 2 MMAs of K = 16).  The
@@ -340,6 +353,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(hempty + kHalo);
   __shared__ int s_last;
   __shared__ float s_bias[2][128];             // bias of the tile in each accumulator
+  __shared__ int s_agents[RTCC_MAX_AGENTS];    // the launch's agents (batch slot -> agent)
+  const long long budget = P.wait_budget;
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -350,6 +365,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
   const uint32_t ncl = cluster_nctarank();
   const bool clustered = ncl == (uint32_t)kMaxSplits;
 
+  if (threadIdx.x < RTCC_MAX_AGENTS) s_agents[threadIdx.x] = P.agents[threadIdx.x];
   if (warp == 0 && lane == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&full[s], 1);
@@ -387,9 +403,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
       uint32_t it = 0, hc = 0;                   // stages (B ring) and halo tiles issued
       int a_mode = 0;                            // last user of the A area: 1 tap boxes, 2 halo tiles
       bool alive = true, waited_pdl = false;
+      // test hook: one wait for an item that never comes (read once)
+      unsigned stall = (P.stall && *P.stall != 0) ? 1u : 0u;
       for (int l = 0; l < P.n_layers && alive; ++l) {
         const LayerDesc& D = P.L[l];
-        const LayerScalars S = layer_scalars(D);
+        const LayerScalars S = layer_scalars(D, P.n_batch);
         const CUtensorMap* mapA = &D.mapA;
         const CUtensorMap* mapB = &D.mapB;
         tma_prefetch_desc(mapA);
@@ -407,13 +425,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
         int npre = 0;
         Item I0{};
         {
-          I0 = item_of(S, t0);
+          I0 = item_of(S, t0, s_agents);
           npre = item_stages(S, I0);
           if (npre > kStages) npre = kStages;
           for (int j = 0; j < npre; ++j) {
             const uint32_t u = it + j;
             const int s = u % kStages;
-            if (!mbar_wait(&empty[s], ((u / kStages) & 1) ^ 1)) {
+            if (!mbar_wait(&empty[s], ((u / kStages) & 1) ^ 1, budget)) {
               atomicOr(P.err, ERR_WAIT_PRODUCER);
               alive = false;
               break;
@@ -432,11 +450,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
         }
         if (S.wait_layers > 0) {
           // every item of the layer this one reads has been stored
-          if (!grid_wait(&P.grid_bar[S.wait_layers - 1], (unsigned)S.wait_items)) {
+          if (!grid_wait(&P.grid_bar[S.wait_layers - 1], (unsigned)S.wait_items + stall, budget)) {
             atomicOr(P.err, ERR_WAIT_PRODUCER);
             alive = false;
             break;
           }
+          stall = 0;
           fence_async_global();
         }
         // Tap boxes and halo tiles share the A area: before it changes use,
@@ -446,7 +465,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
         // when the phase has long completed, so one wait, not one per slot).
         const int mode = S.halo ? 2 : 1;
         if (a_mode != 0 && a_mode != mode && it > 0) {
-          if (!mbar_wait(&empty[(it - 1) % kStages], ((it - 1) / kStages) & 1)) {
+          if (!mbar_wait(&empty[(it - 1) % kStages], ((it - 1) / kStages) & 1, budget)) {
             atomicOr(P.err, ERR_WAIT_PRODUCER);
             break;
           }
@@ -455,7 +474,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
         if (P.stamps && t0 == 0) P.stamps[l] = global_ns();
         if (S.halo) {
           for (int t = t0; t < S.n_items && alive; t += tstep) {
-            const Item I = (t == t0) ? I0 : item_of(S, t);
+            const Item I = (t == t0) ? I0 : item_of(S, t, s_agents);
             // The item's chunks: the first kHalo halo tiles go out at once;
             // from then on, reaching chunk c issues chunk c + 1's halo tile
             // into the slot of chunk c + 1 - kHalo (released when its MMAs are
@@ -465,7 +484,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
             for (int c = 0; c < nch && alive; ++c) {
               while (issued < nch && (issued < kHalo ? c == 0 : issued == c + kHalo - 2)) {
                 const int h = hc % kHalo;
-                if (!mbar_wait(&hempty[h], ((hc / kHalo) & 1) ^ 1)) {
+                if (!mbar_wait(&hempty[h], ((hc / kHalo) & 1) ^ 1, budget)) {
                   atomicOr(P.err, ERR_WAIT_PRODUCER);
                   alive = false;
                   break;
@@ -481,7 +500,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
                 int k0, n;
                 stage_kbs(S, I, j, &k0, &n);
                 const int s = it % kStages;
-                if (!mbar_wait(&empty[s], ((it / kStages) & 1) ^ 1)) {
+                if (!mbar_wait(&empty[s], ((it / kStages) & 1) ^ 1, budget)) {
                   atomicOr(P.err, ERR_WAIT_PRODUCER);
                   alive = false;
                   break;
@@ -494,7 +513,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
           }
         } else {
           for (int t = t0; t < S.n_items && alive; t += tstep) {
-            const Item I = (t == t0) ? I0 : item_of(S, t);
+            const Item I = (t == t0) ? I0 : item_of(S, t, s_agents);
             for (int kb = I.kb0; kb < I.kb1; ++kb, ++it) {
               const int s = it % kStages;
               uint8_t* dA = smem + s * kABytes;
@@ -502,7 +521,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
                 load_a(S, mapA, dA, &full[s], I, kb);         // B already in flight
                 continue;
               }
-              if (!mbar_wait(&empty[s], ((it / kStages) & 1) ^ 1)) {
+              if (!mbar_wait(&empty[s], ((it / kStages) & 1) ^ 1, budget)) {
                 atomicOr(P.err, ERR_WAIT_PRODUCER);
                 alive = false;
                 break;
@@ -522,7 +541,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
       bool alive = true;
       const uint32_t smem0 = smem_u32(smem);
       for (int l = 0; l < P.n_layers && alive; ++l) {
-        const LayerScalars S = layer_scalars(P.L[l]);
+        const LayerScalars S = layer_scalars(P.L[l], P.n_batch);
         const uint32_t idesc = idesc_f16(BM, S.bn, std::is_same<T, __nv_bfloat16>::value);
         const bool bk64 = S.bk == 64;
         const uint32_t swz = bk64 ? 2u : 4u;            // 128B : 64B swizzle
@@ -535,9 +554,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
         const uint32_t a_hi_halo = (uint32_t)(smem_desc(smem0, kHaloW * 128, 2u) >> 32);
         const int t0 = first_item(S), tstep = S.cta_hi - S.cta_lo;
         for (int t = t0; t >= 0 && t < S.n_items && alive; t += tstep, ++tc) {
-          const Item I = item_of(S, t);
+          const Item I = item_of(S, t, s_agents);
           const int acc = tc & 1;
-          if (!mbar_wait(&accempty[acc], ((tc >> 1) & 1) ^ 1)) {
+          if (!mbar_wait(&accempty[acc], ((tc >> 1) & 1) ^ 1, budget)) {
             atomicOr(P.err, ERR_WAIT_MMA);
             alive = false;
             break;
@@ -554,7 +573,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
             const uint32_t bstep = (uint32_t)(S.bn * 8);        // one weight box, 16-byte units
             for (int c = 0; c < nch && alive; ++c) {
               const int h = hc % kHalo;
-              if (!mbar_wait(&hfull[h], (hc / kHalo) & 1)) {
+              if (!mbar_wait(&hfull[h], (hc / kHalo) & 1, budget)) {
                 atomicOr(P.err, ERR_WAIT_MMA);
                 alive = false;
                 break;
@@ -567,7 +586,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
               for (int tap = 0; tap < 9; ++tap) {
                 if ((tap & km) == 0) {
                   s = it % kStages;
-                  if (!mbar_wait(&full[s], (it / kStages) & 1)) {
+                  if (!mbar_wait(&full[s], (it / kStages) & 1, budget)) {
                     atomicOr(P.err, ERR_WAIT_MMA);
                     alive = false;
                     break;
@@ -588,7 +607,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
           } else {
             for (int kb = I.kb0; kb < I.kb1; ++kb, ++it) {
               const int s = it % kStages;
-              if (!mbar_wait(&full[s], (it / kStages) & 1)) {
+              if (!mbar_wait(&full[s], (it / kStages) & 1, budget)) {
                 atomicOr(P.err, ERR_WAIT_MMA);
                 alive = false;
                 break;
@@ -614,18 +633,17 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
     uint32_t tc = 0, dsm_phase = 0;
     bool alive = true;
     for (int l = 0; l < P.n_layers; ++l) {
-      const LayerDesc& D = P.L[l];
-      const LayerScalars S = layer_scalars(D);
+      const LayerScalars S = layer_scalars(P.L[l], P.n_batch);
       const int t0 = first_item(S), tstep = S.cta_hi - S.cta_lo;
       if (t0 < 0) continue;                    // no items here: no count
       int mine = 0;
       for (int t = t0; t < S.n_items; t += tstep, ++tc, ++mine) {
-        const Item I = item_of(S, t);
+        const Item I = item_of(S, t, s_agents);
         const int acc = tc & 1;
         // bias of this tile, read while the MMAs run (the slot was last read
         // two tiles ago, before the barriers in between)
         if (row < S.bn) s_bias[acc][row] = S.bias[(S.kind == DECONV ? 0 : I.n0) + row];
-        if (alive && !mbar_wait(&accfull[acc], (tc >> 1) & 1)) {
+        if (alive && !mbar_wait(&accfull[acc], (tc >> 1) & 1, budget)) {
           if (lane == 0) atomicOr(P.err, ERR_WAIT_EPILOGUE);
           alive = false;
         }
@@ -651,7 +669,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
               pix = (size_t)py * S.ow + px;
               c0 = S.choff + I.n0;
             }
-            orow = static_cast<T*>(S.out) + pix * S.ldc + c0;
+            orow = static_cast<T*>(S.out) + (size_t)I.agent * S.out_astride + pix * S.ldc + c0;
           }
         }
         // the previous item's bulk copies (DSMEM exchange) or tile stores
@@ -727,7 +745,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
             }
             bulk_commit();
           }
-          if (alive && !mbar_wait(recvbar, dsm_phase)) {
+          if (alive && !mbar_wait(recvbar, dsm_phase, budget)) {
             if (lane == 0) atomicOr(P.err, ERR_WAIT_EPILOGUE);
             alive = false;
           }
@@ -754,9 +772,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
         } else {
           // publish this slice's fp32 partial ([bn/4][BM][4] per (slice, tile),
           // so a warp's float4 stores cover 512 contiguous bytes), then the
-          // last slice of the tile sums the slices in slice order
-          const int tiles = S.m_tiles * S.n_tiles;
-          const int tile_id = I.tile;
+          // last slice of the tile sums the slices in slice order (tiles of
+          // the batch's agents numbered slot-major)
+          const int tiles = S.n_batch * S.m_tiles * S.n_tiles;
+          const int tile_id = I.slot * S.m_tiles * S.n_tiles + I.tile;
           float4* mine =
               reinterpret_cast<float4*>(S.ws + (size_t)(I.z * tiles + tile_id) * BM * S.bn) + row;
           for (int c0 = 0; c0 < S.bn; c0 += 16) {
@@ -826,8 +845,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
           if (row == 0) {
             const int sub = I.n0 / S.cout;
             const int sy = sub / S.s, sx = sub - sy * S.s;
+            const CUtensorMap* mapC = &P.mapC[S.deconv_idx][I.agent];
             for (int g = 0; g < S.bn / 64; ++g)
-              tma_store_5d(&D.mapC, stage + g * BM * 128, S.choff + g * 64, sx, I.x0, sy, I.y0);
+              tma_store_5d(mapC, stage + g * BM * 128, S.choff + g * 64, sx, I.x0, sy, I.y0);
             bulk_commit();
           }
         }
@@ -861,6 +881,21 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
+  }
+  // The last CTA to leave zeroes the counters for the next launch that uses
+  // them (every other CTA is past its last wait and count) and reports the
+  // launch's end to the host.
+  if (threadIdx.x == 0) {
+    __threadfence();
+    const unsigned old = atomicAdd(&P.grid_bar[kMaxLayers], 1u);
+    if (old == gridDim.x - 1) {
+      for (int l = 0; l < P.n_layers; ++l) P.grid_bar[l] = 0u;
+      P.grid_bar[kMaxLayers] = 0u;
+      if (P.done_word) {
+        __threadfence_system();
+        *P.done_word = 1;
+      }
+    }
   }
 }
 
@@ -920,19 +955,25 @@ cudaError_t conv_make_maps(ConvLayer& L, bool bf16) {
   const CUtensorMapSwizzle sw =
       (L.bk == 64) ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
   const cuuint64_t C = (cuuint64_t)L.cin, W = (cuuint64_t)L.in_w, H = (cuuint64_t)L.in_h;
+  // the agents' inputs are one tensor, agent outermost
+  const cuuint64_t NA = (cuuint64_t)(L.n_agents > 0 ? L.n_agents : 1);
+  const cuuint64_t AS = (cuuint64_t)L.in_astride * 2;
+  if (L.n_agents < 1 || L.n_agents > RTCC_MAX_AGENTS || L.in_astride < (long long)(C * W * H) ||
+      (L.kind == DECONV && L.out_astride < (long long)L.out_w * L.out_h * L.ldc))
+    return cudaErrorInvalidValue;
   CUresult r;
   if (L.kind == CONV3_S2) {
     if ((L.in_w & 1) || (L.in_h & 1)) return cudaErrorInvalidValue;
-    cuuint64_t dims[5] = {2 * C, W / 2, 2, H / 2, 1};
-    cuuint64_t strides[4] = {2 * C * 2, W * C * 2, 2 * W * C * 2, H * W * C * 2};
+    cuuint64_t dims[5] = {2 * C, W / 2, 2, H / 2, NA};
+    cuuint64_t strides[4] = {2 * C * 2, W * C * 2, 2 * W * C * 2, AS};
     cuuint32_t box[5] = {(cuuint32_t)L.bk, (cuuint32_t)TW, 1, (cuuint32_t)TH, 1};
     cuuint32_t es[5] = {1, 1, 1, 1, 1};
     r = enc(&L.mapA, dt, 5, const_cast<void*>(L.in), dims, strides, box, es,
             CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   } else {
-    cuuint64_t dims[4] = {C, W, H, 1};
-    cuuint64_t strides[3] = {C * 2, W * C * 2, H * W * C * 2};
+    cuuint64_t dims[4] = {C, W, H, NA};
+    cuuint64_t strides[3] = {C * 2, W * C * 2, AS};
     const bool halo = conv_uses_halo(L);
     cuuint32_t box[4] = {(cuuint32_t)L.bk, (cuuint32_t)(halo ? kHaloW : TW),
                          (cuuint32_t)(halo ? kHaloH : TH), 1};
@@ -953,8 +994,10 @@ cudaError_t conv_make_maps(ConvLayer& L, bool bf16) {
           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
   if (L.kind == DECONV) {
-    // output store map: [in_h][s][in_w][s][ldc] view of the output, so one
-    // sub-pixel position of a tile is one box of 64 channels
+    // output store map of each agent: [in_h][s][in_w][s][ldc] view of its
+    // output, so one sub-pixel position of a tile is one box of 64 channels
+    // (a ragged tile's rows past in_h are clipped by the map, which an agent
+    // dimension folded into in_h would not do)
     if (L.bn % 64) return cudaErrorInvalidValue;
     const cuuint64_t LD = (cuuint64_t)L.ldc, S = (cuuint64_t)L.s;
     const cuuint64_t IW = (cuuint64_t)L.in_w, IH = (cuuint64_t)L.in_h, OW = (cuuint64_t)L.out_w;
@@ -962,25 +1005,38 @@ cudaError_t conv_make_maps(ConvLayer& L, bool bf16) {
     cuuint64_t strides[4] = {LD * 2, S * LD * 2, OW * LD * 2, S * OW * LD * 2};
     cuuint32_t box[5] = {64, 1, (cuuint32_t)TW, 1, (cuuint32_t)TH};
     cuuint32_t es[5] = {1, 1, 1, 1, 1};
-    r = enc(&L.mapC, dt, 5, L.out, dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
-            CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    for (int k = 0; k < L.n_agents; ++k) {
+      void* base = static_cast<uint8_t*>(L.out) + (size_t)k * (size_t)L.out_astride * 2;
+      r = enc(&L.mapC[k], dt, 5, base, dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+              CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+      if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+    }
   }
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, unsigned* grid_bar, int* err,
-                          unsigned long long* stamps, bool allow_clusters, BackboneParams* P) {
+cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, int n_batch, unsigned* grid_bar,
+                          int* err, unsigned long long* stamps, bool allow_clusters,
+                          long long wait_budget, BackboneParams* P) {
   if (layers.empty() || layers.size() > (size_t)kMaxLayers) return cudaErrorInvalidValue;
+  if (n_batch < 1 || n_batch > RTCC_MAX_AGENTS || n_batch > layers[0].n_agents || wait_budget < 1)
+    return cudaErrorInvalidValue;
   std::memset(P, 0, sizeof(*P));
   P->n_layers = (int)layers.size();
+  P->n_batch = n_batch;
+  for (int j = 0; j < n_batch; ++j) P->agents[j] = j;
   P->grid_bar = grid_bar;
   P->err = err;
   P->stamps = stamps;
+  P->wait_budget = wait_budget;
   const int grid_sm = backbone_grid(1), grid_cl = allow_clusters ? backbone_grid(kMaxSplits) : 0;
   if (grid_sm < 1) return cudaErrorInvalidValue;
   bool any_dsm = false;
+  int n_deconv = 0;
   for (size_t i = 0; i < layers.size(); ++i) {
     const ConvLayer& L = layers[i];
+    if (L.n_agents != layers[0].n_agents) return cudaErrorInvalidValue;
     const int ncb = L.bk > 0 ? L.cin / L.bk : 0;
     if (L.bk < 1 || L.cin % L.bk || ncb < 1 || (ncb & (ncb - 1)) ||   // a power of two
         (L.kind != DECONV && L.cout % L.bn) || (L.kind == DECONV && L.bn != L.cout) ||
@@ -992,6 +1048,13 @@ cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, unsigned* grid_b
     LayerDesc& D = P->L[i];
     D.mapA = L.mapA;
     D.mapB = L.mapB;
+    D.deconv_idx = -1;
+    if (L.kind == DECONV) {
+      if (n_deconv >= kMaxDeconv) return cudaErrorInvalidValue;
+      D.deconv_idx = n_deconv;
+      for (int k = 0; k < L.n_agents; ++k) P->mapC[n_deconv][k] = L.mapC[k];
+      ++n_deconv;
+    }
     D.bias = L.bias;
     D.ws = L.ws;
     D.counters = L.counters;
@@ -1007,8 +1070,9 @@ cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, unsigned* grid_b
     D.n_tiles = L.n_tiles_n;
     D.choff = L.choff;
     D.wait_layers = L.wait_layers;
-    D.mapC = L.mapC;
     D.out = L.out;
+    D.out_astride = L.out_astride;
+    D.ipa = D.m_tiles * D.n_tiles * L.splits;
     D.ow = L.out_w;
     D.ldc = L.ldc;
     D.gw = L.gw;
@@ -1018,7 +1082,7 @@ cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, unsigned* grid_b
     // CTA, reduces its slices through distributed shared memory within a
     // cluster of kMaxSplits CTAs
     D.dsm = (L.kind != DECONV && (L.splits == 2 || L.splits == kMaxSplits) && L.bn == 64 && grid_cl > 0 &&
-             D.m_tiles * D.n_tiles * L.splits <= grid_cl)
+             n_batch * D.ipa <= grid_cl)
                 ? 1
                 : 0;
     any_dsm = any_dsm || D.dsm;
@@ -1035,7 +1099,7 @@ cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, unsigned* grid_b
   for (int i = 0; i < P->n_layers; ++i) {
     const LayerDesc& D = P->L[i];
     if (D.kind != DECONV) {
-      main_max = std::max(main_max, D.m_tiles * D.n_tiles * D.splits);
+      main_max = std::max(main_max, n_batch * D.ipa);
       last_conv = i;
     }
   }
@@ -1049,7 +1113,7 @@ cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, unsigned* grid_b
     D.wait_items = 0;
     if (D.wait_layers > 0) {
       const LayerDesc& W = P->L[D.wait_layers - 1];
-      D.wait_items = W.m_tiles * W.n_tiles * W.splits;
+      D.wait_items = n_batch * W.ipa;
     }
   }
   return cudaSuccess;

@@ -94,6 +94,12 @@ enum ConvKind { CONV3_S1 = 0, CONV3_S2 = 1, DECONV = 2 };
 
 struct ConvLayer {
   ConvKind kind;
+  // Every agent's tensors of a layer live in one allocation, agent-major with
+  // a fixed stride, so one tensor map covers all agents (the agent index is
+  // the map's outermost coordinate) and a launch may run any set of agents.
+  int n_agents;          // agents the buffers hold
+  long long in_astride;  // elements between agents in `in`
+  long long out_astride; // elements between agents in `out`
   int cin, cout;         // conv: Cout; deconv: Cout per sub-position
   int s;                 // deconv stride (= kernel); 1 for convs
   int in_w, in_h;        // input map
@@ -104,14 +110,15 @@ struct ConvLayer {
   int n_tiles_n;         // N tiles
   int splits;            // split-K factor; 1 = none
   int wait_layers;       // this layer reads outputs of layers [0, wait_layers)
-  float* ws;             // split-K partials [splits][m_tiles * n_tiles][128][bn] fp32
-  int* counters;         // split-K arrivals per tile [m_tiles * n_tiles], zero-initialised
-  const void* in;        // device [in_h][in_w][cin]
-  void* out;             // device [out_h][out_w][ldc]
+  float* ws;             // split-K partials [batch][splits][m_tiles * n_tiles][128][bn] fp32
+  int* counters;         // split-K arrivals per tile [batch][m_tiles * n_tiles], zero-initialised
+  const void* in;        // device [agent][in_h][in_w][cin]
+  void* out;             // device [agent][out_h][out_w][ldc]
   const void* wpacked;   // device, K-major: conv [Cout][9][Cin]; deconv [s*s*Cout][Cin]
   const float* bias;     // device [Cout]
-  CUtensorMap mapA, mapB;         // input (tap boxes or halo tiles), packed weights
-  CUtensorMap mapC;               // deconvs: output store map
+  CUtensorMap mapA, mapB;         // input (tap boxes or halo tiles; outermost
+                                  // coordinate = agent), packed weights
+  CUtensorMap mapC[RTCC_MAX_AGENTS];  // deconvs: output store map of each agent
 };
 
 // Encode the layer's tensor maps (input activations, packed weights).
@@ -128,10 +135,10 @@ int conv_tile_m();
 
 // One layer of the persistent backbone kernel (kernel-parameter layout).
 constexpr int kMaxLayers = 20;
+constexpr int kMaxDeconv = 3;     // neck deconvs (one per block)
 constexpr int kMaxSplits = 4;     // split-K slices per tile (the reducing slice keeps one load per slice in flight)
 struct alignas(128) LayerDesc {   // CUtensorMap is 128-byte aligned
   CUtensorMap mapA, mapB;
-  CUtensorMap mapC;              // deconvs: output store map (convs store from registers)
   const float* bias;
   float* ws;
   int* counters;
@@ -142,24 +149,40 @@ struct alignas(128) LayerDesc {   // CUtensorMap is 128-byte aligned
   int cta_lo, cta_hi;            // the CTAs this layer's items are dealt to (round-robin)
   int wait_items;                // items of layer wait_layers - 1 (its counter's target)
   int halo;                      // 3x3 stride-1 with 64-channel k-blocks: A from halo tiles
-  void* out;                     // output [out_h][ow][ldc], channels from choff
+  void* out;                     // output [agent][out_h][ow][ldc], channels from choff
+  long long out_astride;         // elements between agents in `out`
   int ow, ldc, gw, gh;           // output row length, pixel stride, tile grid extent
+  int ipa;                       // items per agent (m_tiles * n_tiles * splits)
+  int deconv_idx;                // deconvs: index into BackboneParams::mapC
 };
 struct BackboneParams {
   LayerDesc L[kMaxLayers];
+  CUtensorMap mapC[kMaxDeconv][RTCC_MAX_AGENTS];   // deconv output store maps per agent
   int n_layers;
-  unsigned* grid_bar;            // [kMaxLayers] per-layer counts of finished items, zero before each launch
+  int n_batch;                   // agents this launch runs
+  int agents[RTCC_MAX_AGENTS];   // their indices, ascending (the agent coordinate of the maps)
+  unsigned* grid_bar;            // [kMaxLayers + 1] per-layer counts of finished items, then
+                                 // the CTA exit count; zero before a launch (the last CTA to
+                                 // leave zeroes them again)
   int* err;
   unsigned long long* stamps;    // optional [2 * n_layers] global-timer ns: layer starts
                                  // (first item's wait passed), then layer ends (last item counted)
+  volatile int* done_word;       // optional (pinned host): the last CTA to leave writes 1
+  const volatile int* stall;     // optional test hook: when *stall != 0 the first layer that
+                                 // waits for another waits for one item too many (the wait
+                                 // runs out, the error word is set, the kernel winds down)
+  long long wait_budget;         // cycles after which a wait gives up
   int cluster;                   // 1, or kMaxSplits when some layer reduces through DSMEM
   int grid;                      // CTAs of the launch
 };
 
-// Fill the kernel parameters of a branch's backbone from its layer list;
-// grid_bar holds kMaxLayers counters.
-cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, unsigned* grid_bar, int* err,
-                          unsigned long long* stamps, bool allow_clusters, BackboneParams* P);
+// Fill the kernel parameters of a backbone launch over `n_batch` agents from
+// the layer list (whose bn fields are the N tiles for that batch size);
+// grid_bar holds kMaxLayers + 1 counters.  The agent list is set by the
+// caller (agents[0 .. n_batch)).
+cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, int n_batch, unsigned* grid_bar,
+                          int* err, unsigned long long* stamps, bool allow_clusters,
+                          long long wait_budget, BackboneParams* P);
 // One cooperative launch (one CTA per SM) running every layer.
 cudaError_t launch_backbone(const BackboneParams& P, bool bf16, cudaStream_t st);
 // CTAs of a backbone launch: every SM (cluster = 1), or as many CTAs as can be

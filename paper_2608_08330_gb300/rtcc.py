@@ -28,7 +28,7 @@ FUSE_MAX, FUSE_ATTN = 0, 1
 FP16, BF16 = 0, 1
 WAITING, RELEASED, RUNNING, FINISHED, ABSENT = range(5)
 FLAG_TIMELINE, FLAG_KEEP_FUSED, FLAG_KEEP_LAYERS, FLAG_LAYER_TIMES = 1, 2, 4, 8
-FLAG_NO_CLUSTERS = 16
+FLAG_NO_CLUSTERS, FLAG_SHORT_WAITS, FLAG_NO_BATCH, FLAG_H2D_COPY = 16, 32, 64, 128
 TENSOR_IMAGE, TENSOR_FEAT, TENSOR_FUSED, TENSOR_LAYER0 = 0, 8, 9, 16
 
 
@@ -61,6 +61,8 @@ class rtcc_frame_info(C.Structure):
         ("gpu_fusion_ms", C.c_float), ("gpu_post_ms", C.c_float),
         ("dispatch_order", C.c_int32 * MAX_AGENTS), ("n_dispatched", C.c_int32),
         ("gpu_fusion_kernel_ms", C.c_float), ("gpu_pfn_kernel_ms", C.c_float * MAX_AGENTS),
+        ("n_backbone_launches", C.c_int32), ("backbone_batch", C.c_int32 * MAX_AGENTS),
+        ("gpu_launch_ms", C.c_float * MAX_AGENTS),
     ]
 
 
@@ -134,6 +136,7 @@ def load(path: Optional[str] = None) -> C.CDLL:
         "rtcc_status_str": (C.c_char_p, [C.c_int]),
         "rtcc_now_ms": (C.c_double, []),
         "rtcc_kernels_per_frame": (C.c_int32, [_ctx_p, C.c_int32]),
+        "rtcc_test_unreachable_wait": (S, [_ctx_p]),
         "rtcc_pillarise_noalloc": (S, [C.POINTER(rtcc_model_config), C.c_void_p, C.c_int32,
                                        C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
                                        C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]),
@@ -349,6 +352,11 @@ def rtcc_now_ms() -> float:
 
 def rtcc_kernels_per_frame(ctx, n_present: int) -> int:
     return load().rtcc_kernels_per_frame(ctx, n_present)
+
+
+def rtcc_test_unreachable_wait(ctx) -> int:
+    """Arm the wait-limit test hook for the next frame (see rtcc.h)."""
+    return load().rtcc_test_unreachable_wait(ctx)
 
 
 def rtcc_pillarise_noalloc(cfg: rtcc_model_config, d_points: int, n_points: int, d_pfn_w: int,
