@@ -430,6 +430,38 @@ rtcc_status rtcc_ctrl_state(const rtcc_controller* c, int32_t agent,
 rtcc_status rtcc_ctrl_end(rtcc_controller* c);
 
 /* ------------------------------------------------------------------------ */
+/* Slot-level uplink (host only; the source of completion events)           */
+/* ------------------------------------------------------------------------ */
+
+typedef enum {
+  RTCC_SCHED_MAXRATE = 0,     /* RB to the eligible agent of highest rate      */
+  RTCC_SCHED_ROUNDROBIN = 1,  /* RB to the first eligible agent after the one
+                                 served last, in cyclic index order           */
+  RTCC_SCHED_MAXWEIGHT = 2,   /* highest queue x rate                          */
+  RTCC_SCHED_EARLIEST = 3,    /* least time to empty the queue at this rate    */
+  RTCC_SCHED_WEIGHTED = 4     /* highest weight_k x rate (DAG rank, task weight) */
+} rtcc_sched;
+
+/*
+ * Completion slots of one frame's uploads over a slot-level OFDMA uplink
+ * (Sec. III-A, Eqs. 1-5).  Each slot t = 1..t_max: agents with bits left and
+ * t >= first_slot[k] are eligible; each of the n_rb resource blocks goes to
+ * one eligible agent by `policy` (ties to the smaller index); agent k then
+ * sends slot_s x rate bits on each of its RBs; completion_slot[k] is the slot
+ * in which its queue reached zero (0 if not within t_max).  Inputs (host,
+ * caller-owned): payload_bits[n_agents], first_slot[n_agents] (1-based),
+ * rates float64 [t_max][n_agents][n_rb] in bit/s, weight[n_agents] for
+ * RTCC_SCHED_WEIGHTED (else unused, may be NULL).  *n_slots_used (optional)
+ * receives the last slot simulated.  RTCC_E_ARG for bad sizes or pointers.
+ * Deterministic: the same rates give the same slots.
+ */
+rtcc_status rtcc_uplink_simulate(int32_t n_agents, int32_t n_rb, int32_t t_max,
+                                 const double* payload_bits, const int32_t* first_slot,
+                                 const double* rates, double slot_s, int32_t policy,
+                                 const double* weight, int32_t* completion_slot,
+                                 int32_t* n_slots_used);
+
+/* ------------------------------------------------------------------------ */
 /* Misc                                                                     */
 /* ------------------------------------------------------------------------ */
 

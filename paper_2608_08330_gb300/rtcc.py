@@ -137,6 +137,9 @@ def load(path: Optional[str] = None) -> C.CDLL:
         "rtcc_now_ms": (C.c_double, []),
         "rtcc_kernels_per_frame": (C.c_int32, [_ctx_p, C.c_int32]),
         "rtcc_test_unreachable_wait": (S, [_ctx_p]),
+        "rtcc_uplink_simulate": (S, [C.c_int32, C.c_int32, C.c_int32, C.c_void_p, C.c_void_p,
+                                     C.c_void_p, C.c_double, C.c_int32, C.c_void_p, C.c_void_p,
+                                     C.POINTER(C.c_int32)]),
         "rtcc_pillarise_noalloc": (S, [C.POINTER(rtcc_model_config), C.c_void_p, C.c_int32,
                                        C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
                                        C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]),
@@ -352,6 +355,26 @@ def rtcc_now_ms() -> float:
 
 def rtcc_kernels_per_frame(ctx, n_present: int) -> int:
     return load().rtcc_kernels_per_frame(ctx, n_present)
+
+
+SCHED_MAXRATE, SCHED_ROUNDROBIN, SCHED_MAXWEIGHT, SCHED_EARLIEST, SCHED_WEIGHTED = range(5)
+
+
+def rtcc_uplink_simulate(payload_bits, first_slot, rates: np.ndarray, slot_s: float, policy: int,
+                         weight=None):
+    """Completion slots of one frame's uploads (see rtcc.h); rates [T][K][F]
+    bit/s.  Returns (completion slots int32 [K], 0 = not within T; slots used)."""
+    r = np.ascontiguousarray(rates, dtype=np.float64)
+    T, K, F = r.shape
+    b = np.ascontiguousarray(payload_bits, dtype=np.float64)
+    l = np.ascontiguousarray(first_slot, dtype=np.int32)
+    wt = None if weight is None else np.ascontiguousarray(weight, dtype=np.float64)
+    out = np.zeros(K, dtype=np.int32)
+    used = C.c_int32(0)
+    _chk(load().rtcc_uplink_simulate(K, F, T, _ptr(b), _ptr(l), _ptr(r), float(slot_s), int(policy),
+                                     None if wt is None else _ptr(wt), _ptr(out), C.byref(used)),
+         "rtcc_uplink_simulate")
+    return out, used.value
 
 
 def rtcc_test_unreachable_wait(ctx) -> int:
