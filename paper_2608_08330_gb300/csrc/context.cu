@@ -275,12 +275,13 @@ rtcc_status upload_f32(rtcc_ctx* c, const float* src, size_t n, float** dst) {
 }
 
 // W [Co][Ci][3][3] -> [Co][tap][Ci] in the storage type
+// W [Co][Ci][3][3] -> tap-major [tap][Co][Ci] (one TMA box carries several taps)
 rtcc_status upload_conv(rtcc_ctx* c, const float* w, int co, int ci) {
   std::vector<uint16_t> p((size_t)co * 9 * ci);
   for (int o = 0; o < co; ++o)
     for (int i = 0; i < ci; ++i)
       for (int t = 0; t < 9; ++t)
-        p[((size_t)o * 9 + t) * ci + i] = bits_store(w[((size_t)o * ci + i) * 9 + t], c->bf16);
+        p[((size_t)t * co + o) * ci + i] = bits_store(w[((size_t)o * ci + i) * 9 + t], c->bf16);
   void* d = nullptr;
   RS(dalloc(c, &d, p.size() * 2));
   CK(cudaMemcpy(d, p.data(), p.size() * 2, cudaMemcpyHostToDevice));
@@ -380,27 +381,46 @@ void pick_tile(int m_tiles, int co, int total_kb, int grid, int* bn_out, int* sp
 
 constexpr size_t kFrameZeroBytes = 8 * sizeof(int) + (kMaxLayers + 1) * sizeof(unsigned);
 
-// N tile of a conv layer in a launch over `batch` agents, with its K slices
+// Tile of a conv layer in a launch over `batch` agents, with its K slices
 // fixed (they decide the fp32 summation order, so they are the same for every
 // batch size and a branch's result does not depend on the launch that ran
-// it; the N tile only decides which channels an item computes).  Cost model
-// of pick_tile: rounds of items over the grid times k-blocks per item; ties go
-// to the wider tile (fewer, longer items per FLOP).
-int pick_bn_batch(int m_tiles, int co, int total_kb, int sp, int grid, int batch, bool need64) {
+// it; the N tile only decides which channels an item computes, and the tile
+// height which pixels).  Cost model: rounds of items over the grid times
+// k-blocks per item times a k-block's MMA time at that N tile (measured:
+// 45, 48 and 64 clocks per K = 16 MMA at N = 32, 64, 128); a tall tile
+// (halo layers without split-K: two 128-row MMAs on every weight box) costs
+// kTallCost short k-blocks per k-block -- more than one because it does
+// twice the MMAs, less than two because it halves the weight boxes per FLOP,
+// which bound a short k-block once every CTA has several items.  Ties go to
+// the narrower tile, then to the short one (more, shorter items).
+constexpr double kTallCost = 1.6;
+double kblock_cost(int bn) { return bn >= 128 ? 1.0 : bn >= 64 ? 0.75 : 0.70; }
+void pick_tile_batch(const ConvLayer& L0, int sp, int grid, int batch, bool need64, int* bn_out,
+                     int* tall_out) {
   double best = 1e30;
-  int bb = std::min(co, 64);
-  for (int bn : {128, 64, 32}) {
-    if (bn > co || co % bn) continue;
-    if (need64 && bn != 64) continue;
-    const int items = batch * m_tiles * (co / bn) * sp;
-    const int rounds = (items + grid - 1) / grid;
-    const double cost = rounds * (double)((total_kb + sp - 1) / sp);
-    if (cost < best - 1e-9) {
-      best = cost;
-      bb = bn;
+  *bn_out = std::min(L0.cout, 64);
+  *tall_out = 0;
+  const int total_kb = 9 * (L0.cin / L0.bk);
+  for (int tall = 0; tall <= 1; ++tall) {
+    ConvLayer L = L0;
+    L.tall = tall;
+    L.splits = sp;
+    if (tall && (sp != 1 || !conv_uses_halo(L))) continue;
+    const int m_tiles = conv_m_tiles(L);
+    for (int bn : {32, 64, 128}) {
+      if (bn > L.cout || L.cout % bn) continue;
+      if (need64 && bn != 64) continue;
+      const int items = batch * m_tiles * (L.cout / bn) * sp;
+      const int rounds = (items + grid - 1) / grid;
+      const double cost =
+          rounds * (double)((total_kb + sp - 1) / sp) * kblock_cost(bn) * (tall ? kTallCost : 1.0);
+      if (cost < best - 1e-9) {
+        best = cost;
+        *bn_out = bn;
+        *tall_out = tall;
+      }
     }
   }
-  return bb;
 }
 
 // The backbone's layer list over the agent-major tensors of all K agents, and
@@ -548,19 +568,17 @@ rtcc_status build_backbone(rtcc_ctx* c) {
   RS(dalloc(c, &c->batch_bar, (kMaxLayers + 1) * sizeof(unsigned)));
   CK(cudaMemset(c->batch_bar, 0, (kMaxLayers + 1) * sizeof(unsigned)));
   c->wait_budget = (g.flags & RTCC_FLAG_SHORT_WAITS) ? 20000000LL : 2000000000LL;
-  // launch parameters per batch size: the same K slices, the N tile chosen
-  // for the batch
+  // launch parameters per batch size: the same K slices, the N tile and tile
+  // height chosen for the batch
   for (int nb = 1; nb <= K; ++nb) {
     std::vector<ConvLayer> Lb = c->layers;
     for (ConvLayer& L : Lb) {
-      if (nb > 1 && L.kind != DECONV) {
-        const int m_tiles = ((L.gw + conv_tile_w() - 1) / conv_tile_w()) *
-                            ((L.gh + conv_tile_h() - 1) / conv_tile_h());
-        const int total_kb = 9 * (L.cin / L.bk);
+      if (L.kind != DECONV) {
+        const int m_tiles = conv_m_tiles(L);           // short tiles (the one-agent K slices)
         // a split layer whose items fit the clustered grid keeps the DSMEM
         // exchange (64-wide tiles); otherwise it reduces through global memory
         const bool dsm_fit = L.splits > 1 && nb * m_tiles * (L.cout / 64) * L.splits <= grid;
-        L.bn = pick_bn_batch(m_tiles, L.cout, total_kb, L.splits, grid, nb, dsm_fit);
+        pick_tile_batch(L, L.splits, grid, nb, dsm_fit, &L.bn, &L.tall);
         L.n_tiles_n = L.cout / L.bn;
       }
       L.ws = c->batch_ws;
@@ -1039,7 +1057,7 @@ rtcc_status launch_pill(rtcc_ctx* c, int k) {
 // already enqueued).  One agent: its own launch parameters, on its own stream
 // behind its pillar chain.  Several: the batch template for that count, on
 // the batch stream after every chain's event; each agent still writes its
-// own slot, and its result does not depend on the batch (see pick_bn_batch).
+// own slot, and its result does not depend on the batch (see pick_tile_batch).
 rtcc_status launch_batch(rtcc_ctx* c) {
   std::vector<int> ag = c->pending;
   c->pending.clear();

@@ -51,26 +51,39 @@ namespace {
 
 constexpr int TW = 8;                        // tile width in pixels: one 8-row MMA atom per image row
 constexpr int TH = 16;                       // tile height
+constexpr int kTallTH = 2 * TH;              // height of a tall tile: two MMA row blocks
 constexpr int BM = TW * TH;                  // 128 = MMA M
-constexpr int kThreads = 192;
+// warps: 0 TMA producer, 1 MMA issuer, 2..5 epilogue, 6..7 more TMA producers
+constexpr int kThreads = 256;
+constexpr int kProducers = 3;
+constexpr int kFirstExtraProducer = 6;
 constexpr int kStages = 5;
 constexpr int kABytes = BM * 64 * 2;         // A slot (BK <= 64)
 constexpr int kBBytes = 128 * 64 * 2;        // B slot (BN <= 128, BK <= 64)
-constexpr int kBOff = kStages * kABytes;     // the A slots, then the B slots
+// taps of 64 channels one B slot holds at N tile bn (a halo layer's stage)
+__host__ __device__ constexpr int kStageTaps(int bn) { return kBBytes / (bn * 128); }
 // Halo tiles (3x3 stride-1 convs with 64-channel k-blocks): the (TW+2) x
-// (TH+2) input pixels of a tile for one 64-channel chunk, 128 bytes each in
-// the 128-byte swizzle; kHalo slots reuse the A area.
-constexpr int kHaloW = TW + 2, kHaloH = TH + 2;
+// (th+2) input pixels of a tile for one 64-channel chunk, 128 bytes each in
+// the 128-byte swizzle; kHalo slots (sized for a tall tile) reuse the A area.
+constexpr int kHaloW = TW + 2, kHaloH = TH + 2, kHaloHTall = kTallTH + 2;
 constexpr int kHaloBytes = kHaloW * kHaloH * 128;
-constexpr int kHaloSlot = 24 * 1024;
-constexpr int kHalo = 3;
-static_assert(kHaloBytes <= kHaloSlot && kHalo * kHaloSlot <= kBOff, "halo slots must fit the A area");
-constexpr int kStagingBytes = 64 * 1024;     // DSMEM split-K exchange: the outgoing slots
+constexpr int kHaloBytesTall = kHaloW * kHaloHTall * 128;
+constexpr int kHaloSlot = 44 * 1024;         // 1024-byte aligned (128-byte swizzle atoms)
+constexpr int kHalo = 2;
+// the lower row block of a tall tile starts TH halo rows further in (16-byte units)
+constexpr uint32_t kTallHalfDesc = (uint32_t)(TH * kHaloW * 128 / 16);
+constexpr int kAArea = 88 * 1024;            // A area: kStages tap-box slots or kHalo halo slots
+constexpr int kBOff = kAArea;                // the A area, then the B slots
+static_assert(kStages * kABytes <= kAArea, "tap-box slots must fit the A area");
+static_assert(kHaloBytesTall <= kHaloSlot && kHalo * kHaloSlot <= kAArea, "halo slots must fit the A area");
+constexpr int kStagingBytes = 56 * 1024;     // DSMEM split-K exchange: the outgoing slots
                                              // (4 x 128 x 16 fp32) and the receive slots
                                              // (3 x 128 x 16 fp32); deconvs: the output
                                              // tile (128 x 128 channels, 16-bit)
-constexpr int kSmem = kStages * (kABytes + kBBytes) + kStagingBytes + 1024 + 256;
-constexpr uint32_t kTmemCols = 256;          // two 128-column accumulators
+constexpr int kSmem = kAArea + kStages * kBBytes + kStagingBytes + 1024 + 256;
+// two accumulators of 256 columns: a tall tile's row blocks at +0 and +128
+constexpr uint32_t kAccStride = 256;
+constexpr uint32_t kTmemCols = 2 * kAccStride;
 
 // bias + ReLU of 16 fp32 values, packed to 16 bits and written as two
 // 16-byte stores to dst (16-byte aligned: the channel offset is a multiple of
@@ -104,6 +117,10 @@ __device__ __forceinline__ void stage16(uint8_t* stage, int row, int c0, const f
   *reinterpret_cast<uint4*>(base + ((j0 ^ x) << 4)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
   *reinterpret_cast<uint4*>(base + (((j0 + 1) ^ x) << 4)) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
 }
+
+// The epilogue threads that issue a deconv item's TMA box stores: the first
+// thread of each of the bn / 64 first epilogue warps (one 64-channel box each).
+__device__ __forceinline__ bool deconv_storer(int row, int bn) { return (row & 31) == 0 && row < bn / 2; }
 
 // barrier among the 4 epilogue warps only (named barrier 1, 128 threads)
 __device__ __forceinline__ void epilogue_sync() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
@@ -150,6 +167,8 @@ struct LayerScalars {
   int cta_lo, cta_hi;      // CTAs the items are dealt to
   int wait_items;          // target of the awaited layer's counter
   int halo;                // A from halo tiles; k-blocks chunk-major (kb = 9 chunk + tap)
+  int tall;                // halo layers: tiles of TW x kTallTH pixels (two MMA row blocks
+                           // sharing every weight box) instead of TW x TH
   int kpb;                 // k-blocks per pipeline stage: halo layers put the weight boxes of
                            // kBBytes / (bn * 128) taps into one stage, others 1 (A + B)
   int spc;                 // halo layers: stages per 64-channel chunk (a stage never spans
@@ -183,6 +202,7 @@ __device__ __forceinline__ LayerScalars layer_scalars(const LayerDesc& D, int n_
   S.cta_hi = D.cta_hi;
   S.wait_items = D.wait_items;
   S.halo = D.halo;
+  S.tall = D.tall;
   S.out = D.out;
   S.out_astride = D.out_astride;
   S.ipa = D.ipa;
@@ -192,7 +212,7 @@ __device__ __forceinline__ LayerScalars layer_scalars(const LayerDesc& D, int n_
   S.ldc = D.ldc;
   S.gw = D.gw;
   S.gh = D.gh;
-  S.kpb = S.halo ? kBBytes / (S.bn * 128) : 1;
+  S.kpb = S.halo ? kStageTaps(S.bn) : 1;
   S.spc = (9 + S.kpb - 1) / S.kpb;
   S.n_items = n_batch * S.ipa;
   S.ncb_log2 = __ffs(S.cin / S.bk) - 1;            // cin / bk is a power of two
@@ -227,7 +247,7 @@ __device__ __forceinline__ Item item_of(const LayerScalars& S, int t, const int*
   const int mt = it.tile % S.m_tiles;
   const int nt = it.tile / S.m_tiles;
   it.x0 = (mt % S.tiles_x) * TW;
-  it.y0 = (mt / S.tiles_x) * TH;
+  it.y0 = (mt / S.tiles_x) * (S.tall ? kTallTH : TH);
   it.n0 = nt * S.bn;
   it.kb0 = (it.z * S.total_kb) / S.splits;
   it.kb1 = ((it.z + 1) * S.total_kb) / S.splits;
@@ -272,17 +292,24 @@ __device__ __forceinline__ void load_a(const LayerScalars& S, const CUtensorMap*
   }
 }
 
-// TMA load of the weight (B) box of k-block kb of item I.  The packed
-// weights are [Cout][tap][Cin]: K index = tap * cin + cb * bk, which is kb * bk
-// for tap-major k-blocks.
+// TMA load of the weight (B) box starting at k-block kb of item I.  Conv
+// weights are packed tap-major, [tap][Cout][Cin], and mapped as a 3-D tensor
+// (Cin, Cout, tap): the box (bk channels, bn rows, taps) at (cb * bk, n0, tap)
+// lands as one bn x bk operand per tap, bn * bk * 2 bytes apart (a halo
+// layer's stage loads its kpb consecutive taps of one chunk in one box; map
+// decides the tap count).  Deconv weights stay [(sub-position, Cout)][Cin].
 __device__ __forceinline__ void load_b(const LayerScalars& S, const CUtensorMap* map, uint8_t* dB,
                                        uint64_t* bar, const Item& I, int kb) {
-  int k = kb * S.bk;
-  if (S.halo) {
+  if (S.kind == DECONV) {
+    tma_load_2d(dB, map, bar, kb * S.bk, I.n0);
+  } else if (S.halo) {
     const int cb = kb / 9, tap = kb - 9 * cb;
-    k = tap * S.cin + cb * 64;
+    tma_load_3d(dB, map, bar, cb * 64, I.n0, tap);
+  } else {
+    const int tap = kb >> S.ncb_log2;
+    const int cb = kb - (tap << S.ncb_log2);
+    tma_load_3d(dB, map, bar, cb * S.bk, I.n0, tap);
   }
-  tma_load_2d(dB, map, bar, k, I.n0);
 }
 
 // TMA load of the halo tile of 64-channel chunk cb of item I: input pixels
@@ -337,12 +364,46 @@ __device__ __forceinline__ void mma_kblock(uint32_t d_tmem, uint32_t a_lo, uint3
   }
 }
 
+// The MMAs of one 64-channel chunk of a halo layer's item: the 9 taps fully
+// unrolled, so every descriptor offset is an immediate and the MMAs issue
+// back to back; a stage of kpb taps (km = kpb - 1) starts with a wait on its
+// weight box and ends with a commit that frees it.  TALL: the tile's lower
+// row block (accumulator columns +128) takes the same weight box with the A
+// rows TH halo rows further down.  False if a wait runs out.
+template <bool TALL>
+__device__ __forceinline__ bool halo_chunk_mma(uint32_t d_tmem, uint32_t a_lo, uint32_t a_hi, uint32_t b_lo0,
+                                               uint32_t b_hi, uint32_t idesc, int km, uint32_t bstep,
+                                               bool accumulate, uint64_t* full, uint64_t* empty, uint32_t& it,
+                                               long long budget) {
+  uint32_t b_lo = 0;
+  int s = 0;
+#pragma unroll
+  for (int tap = 0; tap < 9; ++tap) {
+    if ((tap & km) == 0) {
+      s = it % kStages;
+      if (!mbar_wait(&full[s], (it / kStages) & 1, budget)) return false;
+      tc_fence_after();
+      b_lo = b_lo0 + (uint32_t)(s * (kBBytes >> 4));
+    }
+    const uint32_t a_tap = a_lo + (uint32_t)(((tap / 3) * kHaloW + tap % 3) * 8);
+    const uint32_t b_tap = b_lo + (uint32_t)(tap & km) * bstep;
+    const uint32_t accum = (accumulate || tap > 0) ? 1u : 0u;
+    mma_kblock(d_tmem, a_tap, a_hi, b_tap, b_hi, idesc, accum, true);
+    if (TALL) mma_kblock(d_tmem + 128, a_tap + kTallHalfDesc, a_hi, b_tap, b_hi, idesc, accum, true);
+    if (((tap + 1) & km) == 0 || tap == 8) {
+      umma_commit(&empty[s]);
+      ++it;
+    }
+  }
+  return true;
+}
+
 template <typename T>
 __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant__ BackboneParams P) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint8_t* stage = smem + kStages * (kABytes + kBBytes);
+  uint8_t* stage = smem + kAArea + kStages * kBBytes;
   uint64_t* full = reinterpret_cast<uint64_t*>(stage + kStagingBytes);
   uint64_t* empty = full + kStages;
   uint64_t* accfull = empty + kStages;         // [2]
@@ -393,14 +454,24 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   pdl_trigger();
-  // the pseudo-image is the previous kernel's output; the producer waits for it
-  // only after it has issued layer 0's weight boxes
-  if (warp != 0) pdl_wait();
+  // the pseudo-image is the previous kernel's output; the producers wait for
+  // it only after they have issued layer 0's weight boxes
+  const bool producer_warp = warp == 0 || warp >= kFirstExtraProducer;
+  if (!producer_warp) pdl_wait();
 
-  if (warp == 0) {
+  if (producer_warp) {
     if (lane == 0) {
-      // ---------------- TMA producer (one thread) ----------------
-      uint32_t it = 0, hc = 0;                   // stages (B ring) and halo tiles issued
+      // ---------------- TMA producers (one thread in each of kProducers warps) ----------------
+      // One thread's TMA boxes complete one after another, each in about the
+      // same time whatever its size (measured on GB300: ~600 clocks), so a
+      // single issuing thread cannot keep the tensor pipe fed.  The boxes are
+      // dealt over kProducers threads: pipeline stage u (its A and B boxes,
+      // or a halo layer's one weight box of kpb taps) to thread
+      // u % kProducers, and a chunk's halo tile to the thread of the chunk's
+      // first stage, issued just before that stage.  Every thread walks the
+      // same sequence of layers, items and stages and issues only its own.
+      const uint32_t pid = (warp == 0) ? 0u : (uint32_t)(warp - kFirstExtraProducer + 1);
+      uint32_t it = 0, hc = 0;                   // stages (B ring) and halo tiles so far
       int a_mode = 0;                            // last user of the A area: 1 tap boxes, 2 halo tiles
       bool alive = true, waited_pdl = false;
       // test hook: one wait for an item that never comes (read once)
@@ -410,40 +481,38 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
         const LayerScalars S = layer_scalars(D, P.n_batch);
         const CUtensorMap* mapA = &D.mapA;
         const CUtensorMap* mapB = &D.mapB;
+        const CUtensorMap* mapB1 = &D.mapB1;
         tma_prefetch_desc(mapA);
         tma_prefetch_desc(mapB);
+        if (S.halo) tma_prefetch_desc(mapB1);
         // bytes landing on a stage's barrier: the tap box and the weight box,
         // or for a layer that reads halo tiles (they have their own barriers)
-        // the weight boxes of the stage's kpb k-blocks
-        const uint32_t bbox = (uint32_t)S.bn * S.bk * 2;
-        const uint32_t bytes = S.halo ? bbox * S.kpb : (uint32_t)(BM * S.bk * 2) + bbox;
+        // the weight box of the stage's taps
+        const uint32_t bbox = (uint32_t)S.bn * S.bk * 2;       // one tap's weight rows
+        const uint32_t bytes = (uint32_t)(BM * S.bk * 2) + bbox;
         // The weights do not depend on the previous layer: load the B boxes
-        // of the first k-blocks of this CTA's first item before waiting for
+        // of the first stages of this CTA's first item before waiting for
         // the layer's input, so only the A boxes remain after the wait.
         const int t0 = first_item(S), tstep = S.cta_hi - S.cta_lo;
         if (t0 < 0) continue;                    // no items here: no wait, no count
-        int npre = 0;
-        Item I0{};
-        {
-          I0 = item_of(S, t0, s_agents);
-          npre = item_stages(S, I0);
-          if (npre > kStages) npre = kStages;
-          for (int j = 0; j < npre; ++j) {
-            const uint32_t u = it + j;
-            const int s = u % kStages;
-            if (!mbar_wait(&empty[s], ((u / kStages) & 1) ^ 1, budget)) {
-              atomicOr(P.err, ERR_WAIT_PRODUCER);
-              alive = false;
-              break;
-            }
-            int k0, n;
-            stage_kbs(S, I0, j, &k0, &n);
-            mbar_arrive_expect_tx(&full[s], S.halo ? bbox * n : bytes);
-            for (int i = 0; i < n; ++i)
-              load_b(S, mapB, smem + kBOff + s * kBBytes + i * bbox, &full[s], I0, k0 + i);
+        const Item I0 = item_of(S, t0, s_agents);
+        int npre = item_stages(S, I0);
+        if (npre > kStages) npre = kStages;
+        for (int j = 0; j < npre; ++j) {
+          const uint32_t u = it + j;
+          if (u % kProducers != pid) continue;
+          const int s = u % kStages;
+          if (!mbar_wait(&empty[s], ((u / kStages) & 1) ^ 1, budget)) {
+            atomicOr(P.err, ERR_WAIT_PRODUCER);
+            alive = false;
+            break;
           }
-          if (!alive) break;
+          int k0, n;
+          stage_kbs(S, I0, j, &k0, &n);
+          mbar_arrive_expect_tx(&full[s], S.halo ? bbox * n : bytes);
+          load_b(S, (S.halo && n < S.kpb) ? mapB1 : mapB, smem + kBOff + s * kBBytes, &full[s], I0, k0);
         }
+        if (!alive) break;
         if (!waited_pdl) {                       // the pseudo-image is the previous kernel's output
           pdl_wait();
           waited_pdl = true;
@@ -461,60 +530,85 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
         // Tap boxes and halo tiles share the A area: before it changes use,
         // the MMAs that read it must be done.  The issuer commits every stage
         // after its MMAs, halo tiles included, so the release of the last stage
-        // issued implies the rest (a wait costs about a hundred clocks even
-        // when the phase has long completed, so one wait, not one per slot).
+        // implies the rest.  This thread may get here before another producer
+        // has even issued the last stages, so it waits for the releases of the
+        // last kStages stages in order: each wait then finds its barrier's
+        // previous phase complete, and the phase parity cannot alias.
         const int mode = S.halo ? 2 : 1;
         if (a_mode != 0 && a_mode != mode && it > 0) {
-          if (!mbar_wait(&empty[(it - 1) % kStages], ((it - 1) / kStages) & 1, budget)) {
+          for (uint32_t x = it > (uint32_t)kStages ? it - kStages : 0u; x < it && alive; ++x) {
+            if (!mbar_wait(&empty[x % kStages], (x / kStages) & 1, budget)) {
+              atomicOr(P.err, ERR_WAIT_PRODUCER);
+              alive = false;
+            }
+          }
+          if (!alive) break;
+        }
+        a_mode = mode;
+        if (P.stamps && t0 == 0 && pid == 0) P.stamps[l] = global_ns();
+        if (S.halo) {
+          // Halo tiles in the order the MMAs use them: this CTA's items, chunk
+          // by chunk, tile k + kHalo in the slot of tile k once tile k's MMAs
+          // are done.  The layer's first tile goes out right after the
+          // dependency wait; tile k + 1 goes out with the trigger stage of
+          // chunk k (its 5th, or its last if shorter), from that stage's
+          // thread: that thread has just seen the release of the stage 5
+          // earlier, so chunk k - 1 is done (tile k + 1's slot is free) and
+          // the tile has a chunk of MMAs to land.
+          const int nch = (I0.kb1 - I0.kb0) / 9;       // chunks per item (the same for all)
+          const int n_halos = ((S.n_items - 1 - t0) / tstep + 1) * nch;
+          const uint32_t hbytes = S.tall ? (uint32_t)kHaloBytesTall : (uint32_t)kHaloBytes;
+          const int trig = S.spc < 5 ? S.spc - 1 : 4;
+          const uint32_t hc0 = hc;
+          // tile k of this layer (the threads take turns, so each works out
+          // the tile's item itself)
+          auto issue_halo = [&](int k) -> bool {
+            const uint32_t hk = hc0 + (uint32_t)k;
+            const int h = hk % kHalo;
+            if (!mbar_wait(&hempty[h], ((hk / kHalo) & 1) ^ 1, budget)) return false;
+            const int i = k / nch, c = k - i * nch;
+            const Item In = (i == 0) ? I0 : item_of(S, t0 + i * tstep, s_agents);
+            mbar_arrive_expect_tx(&hfull[h], hbytes);
+            load_halo(mapA, smem + h * kHaloSlot, &hfull[h], In, In.kb0 / 9 + c);
+            return true;
+          };
+          if (it % kProducers == pid && !issue_halo(0)) {
             atomicOr(P.err, ERR_WAIT_PRODUCER);
             break;
           }
-        }
-        a_mode = mode;
-        if (P.stamps && t0 == 0) P.stamps[l] = global_ns();
-        if (S.halo) {
+          int k = 0;                                    // chunk index in this layer
           for (int t = t0; t < S.n_items && alive; t += tstep) {
             const Item I = (t == t0) ? I0 : item_of(S, t, s_agents);
-            // The item's chunks: the first kHalo halo tiles go out at once;
-            // from then on, reaching chunk c issues chunk c + 1's halo tile
-            // into the slot of chunk c + 1 - kHalo (released when its MMAs are
-            // done), a chunk of MMAs ahead of its use.
-            const int c0 = I.kb0 / 9, nch = (I.kb1 - I.kb0) / 9;
-            int issued = 0;
-            for (int c = 0; c < nch && alive; ++c) {
-              while (issued < nch && (issued < kHalo ? c == 0 : issued == c + kHalo - 2)) {
-                const int h = hc % kHalo;
-                if (!mbar_wait(&hempty[h], ((hc / kHalo) & 1) ^ 1, budget)) {
-                  atomicOr(P.err, ERR_WAIT_PRODUCER);
-                  alive = false;
-                  break;
-                }
-                mbar_arrive_expect_tx(&hfull[h], (uint32_t)kHaloBytes);
-                load_halo(mapA, smem + h * kHaloSlot, &hfull[h], I, c0 + issued);
-                ++hc;
-                ++issued;
-              }
+            for (int c = 0; c < nch && alive; ++c, ++k) {
               for (int q = 0; q < S.spc && alive; ++q, ++it) {
+                if (it % kProducers != pid) continue;
                 const int j = c * S.spc + q;
-                if (t == t0 && j < npre) continue;               // weights already in flight
-                int k0, n;
-                stage_kbs(S, I, j, &k0, &n);
-                const int s = it % kStages;
-                if (!mbar_wait(&empty[s], ((it / kStages) & 1) ^ 1, budget)) {
+                if (!(t == t0 && j < npre)) {           // weights not already in flight
+                  int k0, n;
+                  stage_kbs(S, I, j, &k0, &n);
+                  const int s = it % kStages;
+                  if (!mbar_wait(&empty[s], ((it / kStages) & 1) ^ 1, budget)) {
+                    atomicOr(P.err, ERR_WAIT_PRODUCER);
+                    alive = false;
+                    break;
+                  }
+                  mbar_arrive_expect_tx(&full[s], bbox * n);
+                  load_b(S, n < S.kpb ? mapB1 : mapB, smem + kBOff + s * kBBytes, &full[s], I, k0);
+                }
+                if (q == trig && k + 1 < n_halos && !issue_halo(k + 1)) {
                   atomicOr(P.err, ERR_WAIT_PRODUCER);
                   alive = false;
                   break;
                 }
-                mbar_arrive_expect_tx(&full[s], bbox * n);
-                for (int i = 0; i < n; ++i)
-                  load_b(S, mapB, smem + kBOff + s * kBBytes + i * bbox, &full[s], I, k0 + i);
               }
             }
           }
+          hc = hc0 + (uint32_t)n_halos;
         } else {
           for (int t = t0; t < S.n_items && alive; t += tstep) {
             const Item I = (t == t0) ? I0 : item_of(S, t, s_agents);
             for (int kb = I.kb0; kb < I.kb1; ++kb, ++it) {
+              if (it % kProducers != pid) continue;
               const int s = it % kStages;
               uint8_t* dA = smem + s * kABytes;
               if (t == t0 && kb - I.kb0 < npre) {
@@ -562,12 +656,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
             break;
           }
           tc_fence_after();
-          const uint32_t d_tmem = tmem + acc * 128;
+          const uint32_t d_tmem = tmem + acc * kAccStride;
           if (S.halo) {
             // Chunk by chunk: wait for the halo tile, then the 9 taps fully
             // unrolled, so every descriptor offset is an immediate and the
             // MMAs issue back to back; a stage of kpb taps starts with a wait
-            // on its weight boxes and ends with a commit that frees it.
+            // on its weight boxes and ends with a commit that frees it.  A
+            // tall tile's lower row block (accumulator columns +128) takes the
+            // same weight box with the A rows TH halo rows further down.
+            const bool tall = S.tall != 0;
             const int nch = (I.kb1 - I.kb0) / 9;
             const int km = S.kpb - 1;
             const uint32_t bstep = (uint32_t)(S.bn * 8);        // one weight box, 16-byte units
@@ -580,27 +677,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
               }
               ++hc;
               const uint32_t a_lo = (uint32_t)smem_desc(smem0 + h * kHaloSlot, kHaloW * 128, 2u);
-              uint32_t b_lo = 0;
-              int s = 0;
-#pragma unroll
-              for (int tap = 0; tap < 9; ++tap) {
-                if ((tap & km) == 0) {
-                  s = it % kStages;
-                  if (!mbar_wait(&full[s], (it / kStages) & 1, budget)) {
-                    atomicOr(P.err, ERR_WAIT_MMA);
-                    alive = false;
-                    break;
-                  }
-                  tc_fence_after();
-                  b_lo = b_lo0 + (uint32_t)(s * (kBBytes >> 4));
-                }
-                mma_kblock(d_tmem, a_lo + (uint32_t)(((tap / 3) * kHaloW + tap % 3) * 8), a_hi_halo,
-                           b_lo + (uint32_t)(tap & km) * bstep, b_hi, idesc, (c > 0 || tap > 0) ? 1u : 0u,
-                           true);
-                if (((tap + 1) & km) == 0 || tap == 8) {
-                  umma_commit(&empty[s]);
-                  ++it;
-                }
+              const bool ok = tall ? halo_chunk_mma<true>(d_tmem, a_lo, a_hi_halo, b_lo0, b_hi, idesc, km, bstep,
+                                                          c > 0, full, empty, it, budget)
+                                   : halo_chunk_mma<false>(d_tmem, a_lo, a_hi_halo, b_lo0, b_hi, idesc, km, bstep,
+                                                           c > 0, full, empty, it, budget);
+              if (!ok) {
+                atomicOr(P.err, ERR_WAIT_MMA);
+                alive = false;
+                break;
               }
               umma_commit(&hempty[h]);
             }
@@ -649,7 +733,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
         }
         tc_fence_after();
         const float* bias = s_bias[acc];
-        const uint32_t taddr = tmem + acc * 128 + (static_cast<uint32_t>(qd * 32) << 16);
+        const uint32_t taddr = tmem + acc * kAccStride + (static_cast<uint32_t>(qd * 32) << 16);
         // This row's output pixel (the tile's row-th pixel; for a deconv one
         // sub-pixel position of its input pixel), written straight from
         // registers: channels [n0, n0 + bn) of a conv, [choff, choff + cout)
@@ -674,28 +758,42 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
         }
         // the previous item's bulk copies (DSMEM exchange) or tile stores
         // (deconv) must have read the shared memory they came from
-        if ((S.dsm || S.kind == DECONV) && row == 0) bulk_wait_read_all();
+        if ((S.dsm && row == 0) || (S.kind == DECONV && deconv_storer(row, S.bn))) bulk_wait_read_all();
         epilogue_sync();
         if (S.splits == 1) {
-          // up to 64 columns per round: issue all TMEM loads, wait once
-          for (int c0 = 0; c0 < S.bn; c0 += 64) {
-            const int ng = (S.bn - c0) / 16 < 4 ? (S.bn - c0) / 16 : 4;   // uniform
-            uint32_t r[4][16];
+          // up to 64 columns per round: issue all TMEM loads, wait once; a
+          // tall tile's lower row block (TH image rows further down) follows
+          // from accumulator columns +128
+          const int halves = S.tall ? 2 : 1;
+          for (int hh = 0; hh < halves; ++hh) {
+            T* o = orow;
+            if (hh > 0) {
+              const int px = I.x0 + row % TW, py = I.y0 + TH + row / TW;
+              o = (px < S.gw && py < S.gh)
+                      ? static_cast<T*>(S.out) + (size_t)I.agent * S.out_astride +
+                            ((size_t)py * S.ow + px) * S.ldc + S.choff + I.n0
+                      : nullptr;
+            }
+            const uint32_t ta = taddr + (uint32_t)(hh * 128);
+            for (int c0 = 0; c0 < S.bn; c0 += 64) {
+              const int ng = (S.bn - c0) / 16 < 4 ? (S.bn - c0) / 16 : 4;   // uniform
+              uint32_t r[4][16];
 #pragma unroll
-            for (int g = 0; g < 4; ++g)
-              if (g < ng) tmem_ld16_issue(taddr + c0 + 16 * g, r[g]);
-            tmem_ld_wait();
+              for (int g = 0; g < 4; ++g)
+                if (g < ng) tmem_ld16_issue(ta + c0 + 16 * g, r[g]);
+              tmem_ld_wait();
 #pragma unroll
-            for (int g = 0; g < 4; ++g) {
-              if (g < ng) {
-                tmem_reg_fence(r[g]);
-                float v[16];
+              for (int g = 0; g < 4; ++g) {
+                if (g < ng) {
+                  tmem_reg_fence(r[g]);
+                  float v[16];
 #pragma unroll
-                for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[g][i]);
-                if (S.kind == DECONV)
-                  stage16<T>(stage, row, c0 + 16 * g, v, bias + c0 + 16 * g);
-                else
-                  store16<T>(orow ? orow + c0 + 16 * g : nullptr, v, bias + c0 + 16 * g);
+                  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[g][i]);
+                  if (S.kind == DECONV)
+                    stage16<T>(stage, row, c0 + 16 * g, v, bias + c0 + 16 * g);
+                  else
+                    store16<T>(o ? o + c0 + 16 * g : nullptr, v, bias + c0 + 16 * g);
+                }
               }
             }
           }
@@ -840,14 +938,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
         if (S.kind == DECONV) {
           // A deconv row is 128 channels at a strided sub-pixel position:
           // one 5-D TMA box store per 64 channels beats 16 stores per thread.
+          // A thread's TMA operations complete one after another, so box g
+          // goes out from the first thread of epilogue warp g.
           fence_async_smem();
           epilogue_sync();
-          if (row == 0) {
+          if (deconv_storer(row, S.bn)) {
+            const int g = row / 32;
             const int sub = I.n0 / S.cout;
             const int sy = sub / S.s, sx = sub - sy * S.s;
             const CUtensorMap* mapC = &P.mapC[S.deconv_idx][I.agent];
-            for (int g = 0; g < S.bn / 64; ++g)
-              tma_store_5d(mapC, stage + g * BM * 128, S.choff + g * 64, sx, I.x0, sy, I.y0);
+            tma_store_5d(mapC, stage + g * BM * 128, S.choff + g * 64, sx, I.x0, sy, I.y0);
             bulk_commit();
           }
         }
@@ -858,12 +958,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
       // visible to this thread), so a consumer that acquires the counter
       // sees them.  (With TMA stores, waiting for their completion and a
       // full __threadfence here cost about a microsecond per layer.)
+      if (S.kind == DECONV && deconv_storer(row, S.bn)) {   // TMA stores: complete, then ordered
+        bulk_wait_all();
+        fence_async_global();
+      }
       epilogue_sync();
       if (row == 0) {
-        if (S.kind == DECONV) {                // TMA stores: complete, then ordered
-          bulk_wait_all();
-          fence_async_global();
-        }
         if (P.stamps) {
           const unsigned before = atom_add_release_gpu(&P.grid_bar[l], (unsigned)mine);
           // the CTA completing the layer's count stamps its end
@@ -946,6 +1046,10 @@ cudaError_t tmap_2d(CUtensorMap* m, const void* base, bool bf16, uint64_t inner,
 int conv_tile_w() { return TW; }
 int conv_tile_h() { return TH; }
 int conv_tile_m() { return BM; }
+int conv_m_tiles(const ConvLayer& L) {
+  const int th = L.tall ? kTallTH : TH;
+  return ((L.gw + TW - 1) / TW) * ((L.gh + th - 1) / th);
+}
 
 cudaError_t conv_make_maps(ConvLayer& L, bool bf16) {
   EncodeFn enc = encode_fn();
@@ -975,24 +1079,46 @@ cudaError_t conv_make_maps(ConvLayer& L, bool bf16) {
     cuuint64_t dims[4] = {C, W, H, NA};
     cuuint64_t strides[3] = {C * 2, W * C * 2, AS};
     const bool halo = conv_uses_halo(L);
+    if (L.tall && !halo) return cudaErrorInvalidValue;
     cuuint32_t box[4] = {(cuuint32_t)L.bk, (cuuint32_t)(halo ? kHaloW : TW),
-                         (cuuint32_t)(halo ? kHaloH : TH), 1};
+                         (cuuint32_t)(halo ? (L.tall ? kHaloHTall : kHaloH) : TH), 1};
     cuuint32_t es[4] = {1, 1, 1, 1};
     r = enc(&L.mapA, dt, 4, const_cast<void*>(L.in), dims, strides, box, es,
             CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   }
   if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
-  const cuuint64_t K = (cuuint64_t)((L.kind == DECONV ? 1 : 9) * L.cin);
-  const cuuint64_t rows = (cuuint64_t)((L.kind == DECONV ? L.s * L.s : 1) * L.cout);
-  cuuint64_t bdims[2] = {K, rows};
-  cuuint64_t bstr[1] = {K * 2};
-  cuuint32_t bbox[2] = {(cuuint32_t)L.bk, (cuuint32_t)L.bn};
-  cuuint32_t bes[2] = {1, 1};
-  r = enc(&L.mapB, dt, 2, const_cast<void*>(L.wpacked), bdims, bstr, bbox, bes,
-          CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+  if (L.kind == DECONV) {
+    const cuuint64_t K = (cuuint64_t)L.cin;
+    const cuuint64_t rows = (cuuint64_t)(L.s * L.s * L.cout);
+    cuuint64_t bdims[2] = {K, rows};
+    cuuint64_t bstr[1] = {K * 2};
+    cuuint32_t bbox[2] = {(cuuint32_t)L.bk, (cuuint32_t)L.bn};
+    cuuint32_t bes[2] = {1, 1};
+    r = enc(&L.mapB, dt, 2, const_cast<void*>(L.wpacked), bdims, bstr, bbox, bes,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+    L.mapB1 = L.mapB;
+  } else {
+    // tap-major weights [9][Cout][Cin] as (Cin, Cout, tap): mapB carries a
+    // halo layer's kpb taps per box (one tap otherwise), mapB1 one tap
+    const int kpb = conv_uses_halo(L) ? kStageTaps(L.bn) : 1;
+    if (kpb < 1) return cudaErrorInvalidValue;
+    cuuint64_t bdims[3] = {(cuuint64_t)L.cin, (cuuint64_t)L.cout, 9};
+    cuuint64_t bstr[2] = {(cuuint64_t)L.cin * 2, (cuuint64_t)L.cin * L.cout * 2};
+    cuuint32_t bes[3] = {1, 1, 1};
+    cuuint32_t bbox[3] = {(cuuint32_t)L.bk, (cuuint32_t)L.bn, (cuuint32_t)kpb};
+    r = enc(&L.mapB, dt, 3, const_cast<void*>(L.wpacked), bdims, bstr, bbox, bes,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+    bbox[2] = 1;
+    r = enc(&L.mapB1, dt, 3, const_cast<void*>(L.wpacked), bdims, bstr, bbox, bes,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+  }
   if (L.kind == DECONV) {
     // output store map of each agent: [in_h][s][in_w][s][ldc] view of its
     // output, so one sub-pixel position of a tile is one box of 64 channels
@@ -1048,6 +1174,7 @@ cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, int n_batch, uns
     LayerDesc& D = P->L[i];
     D.mapA = L.mapA;
     D.mapB = L.mapB;
+    D.mapB1 = L.mapB1;
     D.deconv_idx = -1;
     if (L.kind == DECONV) {
       if (n_deconv >= kMaxDeconv) return cudaErrorInvalidValue;
@@ -1065,8 +1192,10 @@ cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, int n_batch, uns
     D.bn = L.bn;
     D.bk = L.bk;
     D.splits = L.splits;
+    if (L.tall && (!conv_uses_halo(L) || L.splits != 1)) return cudaErrorInvalidValue;
     D.tiles_x = (L.gw + TW - 1) / TW;
-    D.m_tiles = D.tiles_x * ((L.gh + TH - 1) / TH);
+    D.m_tiles = conv_m_tiles(L);
+    D.tall = L.tall ? 1 : 0;
     D.n_tiles = L.n_tiles_n;
     D.choff = L.choff;
     D.wait_layers = L.wait_layers;

@@ -109,15 +109,19 @@ struct ConvLayer {
   int bn, bk;            // N tile (output channels per item), K chunk (channels)
   int n_tiles_n;         // N tiles
   int splits;            // split-K factor; 1 = none
+  int tall;              // halo layers without split-K: tiles of 8 x 32 pixels, two
+                         // 128-row MMAs per weight box (0: 8 x 16 pixels)
   int wait_layers;       // this layer reads outputs of layers [0, wait_layers)
   float* ws;             // split-K partials [batch][splits][m_tiles * n_tiles][128][bn] fp32
   int* counters;         // split-K arrivals per tile [batch][m_tiles * n_tiles], zero-initialised
   const void* in;        // device [agent][in_h][in_w][cin]
   void* out;             // device [agent][out_h][out_w][ldc]
-  const void* wpacked;   // device, K-major: conv [Cout][9][Cin]; deconv [s*s*Cout][Cin]
+  const void* wpacked;   // device, K-major: conv [9][Cout][Cin]; deconv [s*s*Cout][Cin]
   const float* bias;     // device [Cout]
   CUtensorMap mapA, mapB;         // input (tap boxes or halo tiles; outermost
-                                  // coordinate = agent), packed weights
+                                  // coordinate = agent), packed weights (a halo
+                                  // layer: boxes of a stage's taps)
+  CUtensorMap mapB1;              // packed weights, one tap per box
   CUtensorMap mapC[RTCC_MAX_AGENTS];  // deconvs: output store map of each agent
 };
 
@@ -130,15 +134,17 @@ inline bool conv_uses_halo(const ConvLayer& L) {
   return L.kind == CONV3_S1 && L.bk == 64 && L.splits >= 1 && (L.cin / 64) % L.splits == 0;
 }
 int conv_tile_w();
-int conv_tile_h();
+int conv_tile_h();                 // rows of a tile (a tall tile has twice as many)
 int conv_tile_m();
+// M tiles of layer L's grid with its tile shape
+int conv_m_tiles(const ConvLayer& L);
 
 // One layer of the persistent backbone kernel (kernel-parameter layout).
 constexpr int kMaxLayers = 20;
 constexpr int kMaxDeconv = 3;     // neck deconvs (one per block)
 constexpr int kMaxSplits = 4;     // split-K slices per tile (the reducing slice keeps one load per slice in flight)
 struct alignas(128) LayerDesc {   // CUtensorMap is 128-byte aligned
-  CUtensorMap mapA, mapB;
+  CUtensorMap mapA, mapB, mapB1;
   const float* bias;
   float* ws;
   int* counters;
@@ -149,6 +155,7 @@ struct alignas(128) LayerDesc {   // CUtensorMap is 128-byte aligned
   int cta_lo, cta_hi;            // the CTAs this layer's items are dealt to (round-robin)
   int wait_items;                // items of layer wait_layers - 1 (its counter's target)
   int halo;                      // 3x3 stride-1 with 64-channel k-blocks: A from halo tiles
+  int tall;                      // halo layers: tiles two MMA row blocks high (see ConvLayer)
   void* out;                     // output [agent][out_h][ow][ldc], channels from choff
   long long out_astride;         // elements between agents in `out`
   int ow, ldc, gw, gh;           // output row length, pixel stride, tile grid extent
