@@ -109,6 +109,16 @@ typedef enum {
                                     whose event gates the branch stream, instead
                                     of the branch's first kernel reading the
                                     pinned staging buffer (same results)       */
+#define RTCC_FLAG_MULTISCALE 256 /* the fusion placement of Sec. IV-A (needs a
+                                    neck): each branch ends at its backbone
+                                    blocks; after the join, every block's map
+                                    is fused across the present agents (the
+                                    configured max or ego-query attention, at
+                                    the block's channel count), the neck
+                                    (deconvs + concatenation) runs once on the
+                                    fused maps, then the head.  Without it the
+                                    branches run the neck and the 384-channel
+                                    maps are fused                            */
 
 /*
  * Network and workload description.  Supported: 1 <= n_agents <= 8;
@@ -345,7 +355,10 @@ rtcc_status rtcc_get_pillars(struct rtcc_ctx* ctx, int32_t agent,
  *   which = 1..n_blocks: output of block which-1 [H_b][W_b][C_b]
  *   which = 8: feature slot [H'][W'][C_feat]
  *   which = 9: fused map [H'][W'][C_feat] (agent ignored; needs
- *              RTCC_FLAG_KEEP_FUSED)
+ *              RTCC_FLAG_KEEP_FUSED, or with RTCC_FLAG_MULTISCALE the neck's
+ *              output on the fused blocks)
+ *   which = 10..9+n_blocks: RTCC_FLAG_MULTISCALE: fused map of block
+ *              which-10 [H_b][W_b][C_b] (agent ignored)
  *   which = 16 + i: output of the i-th 3x3 conv of the branch, counting
  *              through all blocks (needs RTCC_FLAG_KEEP_LAYERS)
  * *n_elems receives the tensor's element count. */

@@ -95,6 +95,15 @@ struct rtcc_ctx {
   std::vector<size_t> layer_elems;    // elements per agent
   void* block_out[RTCC_MAX_BLOCKS] = {};
   int block_w[RTCC_MAX_BLOCKS] = {}, block_h[RTCC_MAX_BLOCKS] = {};
+  // RTCC_FLAG_MULTISCALE: the branches end at their blocks; the post-join
+  // fuses each block's map across the agents, then runs the neck once
+  bool ms = false;
+  void* fblk[RTCC_MAX_BLOCKS] = {};   // fused block maps [H_b][W_b][C_b]
+  void* neck_out = nullptr;           // neck of the fused blocks [H'][W'][C_feat]
+  std::vector<ConvLayer> neck_layers; // its deconvs (one "agent")
+  BackboneParams* neck_p = nullptr;
+  unsigned* neck_bar = nullptr;       // [kMaxLayers + 1], zero between launches
+  int* d_one = nullptr;               // [RTCC_MAX_AGENTS] = {1, 0, ...}: the head's one input
   size_t img_elems = 0, feat_elems = 0;
   std::vector<ConvLayer> layers;      // the layer list (N tiles of a one-agent launch)
   BackboneParams* bbt[RTCC_MAX_AGENTS + 1] = {};  // launch parameters per batch size
@@ -236,6 +245,7 @@ rtcc_status validate_config(const rtcc_model_config& c) {
     if ((c.up_stride[b] != 0) != neck) return RTCC_E_ARG;
   }
   if (!neck && c.n_blocks != 1) return RTCC_E_ARG;
+  if ((c.flags & RTCC_FLAG_MULTISCALE) && !neck) return RTCC_E_ARG;
   if (neck) {
     if (c.up_ch != 128) return RTCC_E_ARG;
     // every deconv output must land on block 0's grid
@@ -507,7 +517,44 @@ rtcc_status build_backbone(rtcc_ctx* c) {
     w = ow;
     h = oh;
   }
-  if (neck) {
+  c->ms = (g.flags & RTCC_FLAG_MULTISCALE) != 0;
+  if (neck && c->ms) {
+    // the neck runs after the join, once, on the fused block maps
+    for (int bi = 0; bi < g.n_blocks; ++bi)
+      RS(dalloc(c, &c->fblk[bi], (size_t)c->block_w[bi] * c->block_h[bi] * g.block_ch[bi] * es));
+    RS(dalloc(c, &c->neck_out, c->feat_elems * es));
+    CK(cudaMemset(c->neck_out, 0, c->feat_elems * es));
+    for (int bi = 0; bi < g.n_blocks; ++bi) {
+      ConvLayer L{};
+      L.kind = DECONV;
+      L.n_agents = 1;
+      L.s = g.up_stride[bi];
+      L.cin = g.block_ch[bi];
+      L.cout = g.up_ch;
+      L.in_w = c->block_w[bi];
+      L.in_h = c->block_h[bi];
+      L.out_w = c->Wf;
+      L.out_h = c->Hf;
+      L.gw = L.in_w;
+      L.gh = L.in_h;
+      L.ldc = c->Cf;
+      L.choff = bi * g.up_ch;
+      L.bn = g.up_ch;
+      L.bk = (L.cin >= 64) ? 64 : 32;
+      L.n_tiles_n = L.s * L.s;
+      L.splits = 1;
+      L.in = c->fblk[bi];
+      L.in_astride = (long long)c->block_w[bi] * c->block_h[bi] * g.block_ch[bi];
+      L.out = c->neck_out;
+      L.out_astride = (long long)c->feat_elems;
+      L.wpacked = c->wbufs[wi];
+      L.bias = c->bbufs[wi];
+      L.wait_layers = 0;                              // the fused maps precede the launch
+      ++wi;
+      if (conv_make_maps(L, c->bf16) != cudaSuccess) return RTCC_E_CUDA;
+      c->neck_layers.push_back(L);
+    }
+  } else if (neck) {
     for (int bi = 0; bi < g.n_blocks; ++bi) {
       ConvLayer L{};
       L.kind = DECONV;
@@ -594,6 +641,18 @@ rtcc_status build_backbone(rtcc_ctx* c) {
   }
   c->launch_p = new (std::nothrow) BackboneParams;
   if (!c->launch_p) return RTCC_E_NOMEM;
+  if (c->ms) {
+    RS(dalloc(c, &c->neck_bar, (kMaxLayers + 1) * sizeof(unsigned)));
+    CK(cudaMemset(c->neck_bar, 0, (kMaxLayers + 1) * sizeof(unsigned)));
+    c->neck_p = new (std::nothrow) BackboneParams;
+    if (!c->neck_p) return RTCC_E_NOMEM;
+    if (backbone_fill(c->neck_layers, 1, c->neck_bar, c->d_err, nullptr, false, c->wait_budget, c->neck_p) !=
+        cudaSuccess)
+      return RTCC_E_ARG;
+    int one[RTCC_MAX_AGENTS] = {1};
+    RS(dalloc(c, &c->d_one, sizeof(one)));
+    CK(cudaMemcpy(c->d_one, one, sizeof(one), cudaMemcpyHostToDevice));
+  }
   return RTCC_OK;
 }
 
@@ -737,6 +796,25 @@ rtcc_status capture_branch(rtcc_ctx* c, int k) {
 
 rtcc_status capture_post(rtcc_ctx* c) {
   const bool tl = (c->cfg.flags & RTCC_FLAG_TIMELINE) != 0;
+  // multi-scale placement: fuse each block's outputs, run the neck once on the
+  // fused maps, then the head over that one map (the max "fusion" of a single
+  // input is the identity, so the tensor-core head kernel serves as the head)
+  FuseBlocksArgs fb{};
+  if (c->ms) {
+    fb.n = c->cfg.n_blocks;
+    for (int bi = 0; bi < fb.n; ++bi) {
+      fb.src[bi] = c->block_out[bi];
+      fb.cells[bi] = c->block_w[bi] * c->block_h[bi];
+      fb.ch[bi] = c->cfg.block_ch[bi];
+      fb.astride[bi] = (long long)fb.cells[bi] * fb.ch[bi];
+      fb.dst[bi] = c->fblk[bi];
+    }
+    fb.present = c->d_present;
+    fb.K = c->K;
+    fb.attention = c->cfg.fusion == RTCC_FUSE_ATTN;
+    fb.span = c->fuse_span;
+  }
+  const int K_head = c->ms ? 1 : c->K;
   FuseArgs fa{};
   fa.feats = c->d_feat_ptrs;
   fa.present = c->d_present;
@@ -755,30 +833,31 @@ rtcc_status capture_post(rtcc_ctx* c) {
   fa.span = c->fuse_span;
   // max fusion: tensor-core kernel (TMA-staged agent tiles, max in shared
   // memory, head as an N = 16 MMA); attention fusion: CUDA-core kernel
-  const int bkc = fuse_tc_chunk(c->Cf, c->K);
-  const bool use_tc = !fa.attention && bkc > 0;
+  const int bkc = fuse_tc_chunk(c->Cf, K_head);
+  const bool use_tc = (c->ms || !fa.attention) && bkc > 0;
+  if (c->ms && !use_tc) return RTCC_E_ARG;
   FuseTcParams tp{};
   if (use_tc) {
     const int swz = bkc * 2;                    // 128- or 64-byte rows
-    for (int k = 0; k < c->K; ++k)
-      CK(tmap_2d(&tp.feat[k], c->br[k].feat, c->bf16, (uint64_t)c->Cf, (uint64_t)fa.cells,
-                 (uint32_t)bkc, 128u, swz));
+    for (int k = 0; k < K_head; ++k)
+      CK(tmap_2d(&tp.feat[k], c->ms ? c->neck_out : c->br[k].feat, c->bf16, (uint64_t)c->Cf,
+                 (uint64_t)fa.cells, (uint32_t)bkc, 128u, swz));
     CK(tmap_2d(&tp.wmap, c->head_w16, c->bf16, (uint64_t)c->Cf, 16u, (uint32_t)bkc, 16u, swz));
-    tp.present = c->d_present;
-    tp.K = c->K;
+    tp.present = c->ms ? c->d_one : c->d_present;
+    tp.K = K_head;
     tp.C = c->Cf;
     tp.cells = fa.cells;
     tp.bkc = bkc;
-    tp.stages = fuse_tc_stages(c->Cf, c->K);
+    tp.stages = fuse_tc_stages(c->Cf, K_head);
     tp.head_b = c->head_b;
     tp.head_out = c->head_out;
-    tp.fused = c->fused;
+    tp.fused = c->ms ? nullptr : c->fused;
     tp.keys = c->keys;
     tp.hist0 = c->hist0;
     tp.cls_thresh = c->cfg.cls_thresh;
     tp.anchors = c->cfg.anchors;
     tp.err = c->d_err;
-    tp.span = c->fuse_span;
+    tp.span = c->ms ? nullptr : c->fuse_span;
   }
   DecodeArgs da{};
   da.head = c->head_out;
@@ -814,13 +893,20 @@ rtcc_status capture_post(rtcc_ctx* c) {
   cudaError_t e = cudaSuccess;
   if (tl) e = record_node(c->ev_post0, c->post);
   if (e == cudaSuccess && tl) e = record_node(c->ev_fuse0, c->post);
-  if (e == cudaSuccess) {
-    if (use_tc)
-      e = launch_fuse_max_head(tp, c->bf16, c->post);
-    else
-      e = launch_fuse_head(fa, c->bf16, c->post);
+  if (c->ms) {
+    if (e == cudaSuccess) e = launch_fuse_blocks(fb, c->bf16, c->post);
+    if (e == cudaSuccess && tl) e = record_node(c->ev_fuse1, c->post);
+    if (e == cudaSuccess) e = launch_backbone(*c->neck_p, c->bf16, c->post);
+    if (e == cudaSuccess) e = launch_fuse_max_head(tp, c->bf16, c->post);
+  } else {
+    if (e == cudaSuccess) {
+      if (use_tc)
+        e = launch_fuse_max_head(tp, c->bf16, c->post);
+      else
+        e = launch_fuse_head(fa, c->bf16, c->post);
+    }
+    if (e == cudaSuccess && tl) e = record_node(c->ev_fuse1, c->post);
   }
-  if (e == cudaSuccess && tl) e = record_node(c->ev_fuse1, c->post);
   if (e == cudaSuccess) e = launch_decode(da, c->post);
   if (e == cudaSuccess && c->dec_boxes) e = launch_nms(na, c->post);
   if (e == cudaSuccess && tl) e = record_node(c->ev_post1, c->post);
@@ -869,6 +955,7 @@ void free_all(rtcc_ctx* c) {
     c->bbt[n] = nullptr;
   }
   delete c->launch_p;
+  delete c->neck_p;
   c->launch_p = nullptr;
   if (c->bbst) cudaStreamDestroy(c->bbst);
   if (c->post) cudaStreamDestroy(c->post);
@@ -1587,10 +1674,17 @@ rtcc_status rtcc_get_tensor(rtcc_ctx* c, int32_t agent, int32_t which, uint16_t*
   const void* src = nullptr;
   size_t n = 0;
   if (which == 9) {
-    if (!c->fused) return RTCC_E_STATE;
+    const void* f = c->ms ? c->neck_out : c->fused;
+    if (!f) return RTCC_E_STATE;
     CK(cudaStreamSynchronize(c->post));
-    src = c->fused;
+    src = f;
     n = (size_t)c->Wf * c->Hf * c->Cf;
+  } else if (which >= 10 && which < 10 + c->cfg.n_blocks) {
+    if (!c->ms) return RTCC_E_STATE;
+    CK(cudaStreamSynchronize(c->post));
+    const int bi = which - 10;
+    src = c->fblk[bi];
+    n = (size_t)c->block_w[bi] * c->block_h[bi] * c->cfg.block_ch[bi];
   } else {
     if (agent < 0 || agent >= c->K) return RTCC_E_AGENT;
     Branch& b = c->br[agent];
@@ -1646,7 +1740,8 @@ int32_t rtcc_kernels_per_frame(rtcc_ctx* c, int32_t n_present) {
   // pillar chain per branch; the backbone launches of the last frame (one per
   // branch when none was batched); fusion, decode (and NMS)
   const int bb = c->n_launches > 0 ? c->n_launches : n_present;
-  return n_present * 5 + bb + 2 + (c->dec_boxes ? 1 : 0);
+  // multi-scale: block fusion and the neck's launch before the head
+  return n_present * 5 + bb + 2 + (c->dec_boxes ? 1 : 0) + (c->ms ? 2 : 0);
 }
 
 rtcc_status rtcc_test_unreachable_wait(rtcc_ctx* c) {

@@ -1,0 +1,215 @@
+// Cross-agent fusion of every backbone block's output, the first step of the
+// shared post-join subgraph when the multi-scale maps are fused before the
+// neck (the fusion/upsampling/concatenation placement of Sec. IV-A and the
+// agent-indexed slots of Sec. IV-D): for each block b and each of its BEV
+// cells, the present agents' C_b-channel vectors are fused -- per-channel max,
+// or scaled dot-product attention with the ego agent 0 as the query -- and
+// the fused vector is stored in the storage type.  The neck then runs once on
+// the fused maps.
+//
+// Each thread owns 8 channels (16 bytes) of one cell, so the C_b / 8 threads
+// of a cell read each agent's vector with one coalesced 16-byte load apiece
+// and a warp covers 32 * 8 / C_b consecutive cells.  The kernel is bound by
+// HBM bandwidth: every present agent's block outputs are read once and the
+// fused maps written once.  One launch covers all blocks (warp tasks are
+// numbered block after block).
+//   max:        F = max_k X_k elementwise (exact in the 16-bit domain; the
+//               block outputs are ReLU outputs, so a running max from +0
+//               equals the max over the present agents)
+//   attention:  s_k = <X_0, X_k> / sqrt(C_b), w = softmax over present k,
+//               F = sum_k w_k X_k   (fp32; the dot product is each thread's
+//               8 fused multiply-adds, then a butterfly over the cell's
+//               threads, so every thread holds the same s_k)
+// Every reduction has a fixed order: the result is bit-reproducible.
+#include <cmath>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace rtcc {
+
+namespace {
+
+constexpr unsigned kFull = 0xFFFFFFFFu;
+constexpr int kThreads = 256;
+
+template <typename T>
+__device__ __forceinline__ uint32_t max2(uint32_t a, uint32_t b);
+template <>
+__device__ __forceinline__ uint32_t max2<__half>(uint32_t a, uint32_t b) {
+  __half2 r = __hmax2(*reinterpret_cast<__half2*>(&a), *reinterpret_cast<__half2*>(&b));
+  return *reinterpret_cast<uint32_t*>(&r);
+}
+template <>
+__device__ __forceinline__ uint32_t max2<__nv_bfloat16>(uint32_t a, uint32_t b) {
+  __nv_bfloat162 r =
+      __hmax2(*reinterpret_cast<__nv_bfloat162*>(&a), *reinterpret_cast<__nv_bfloat162*>(&b));
+  return *reinterpret_cast<uint32_t*>(&r);
+}
+
+__device__ __forceinline__ uint4 ld16(const void* p) { return *reinterpret_cast<const uint4*>(p); }
+
+// One thread's 8 channels of one cell.  G = C / 8 threads share the cell
+// (G in {4, 8, 16, 32}); they are lanes [g0, g0 + G) of the warp.
+template <typename T, bool ATTN, int G>
+__device__ __forceinline__ uint4 fuse8(const T* src, long long astride, const unsigned pres, int K,
+                                       size_t off, float inv_sqrt_c) {
+  if (!ATTN) {
+    uint4 m = make_uint4(0u, 0u, 0u, 0u);
+    for (int k = 0; k < K; ++k) {
+      if (!((pres >> k) & 1u)) continue;
+      const uint4 r = ld16(src + (size_t)k * astride + off);
+      m.x = max2<T>(m.x, r.x);
+      m.y = max2<T>(m.y, r.y);
+      m.z = max2<T>(m.z, r.z);
+      m.w = max2<T>(m.w, r.w);
+    }
+    return m;
+  } else {
+    // two passes over the agents (scores, then the weighted sum, reloading
+    // each vector -- an L1 hit) keep one agent's vector live at a time
+    float x0[8];
+    {
+      const uint4 r = ld16(src + off);                // the ego agent 0 is present
+      const uint32_t w[4] = {r.x, r.y, r.z, r.w};
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float2 f = Store<T>::unpack2(w[i]);
+        x0[2 * i] = f.x;
+        x0[2 * i + 1] = f.y;
+      }
+    }
+    float s[RTCC_MAX_AGENTS];
+    float mx = -INFINITY;
+#pragma unroll
+    for (int k = 0; k < RTCC_MAX_AGENTS; ++k) {
+      s[k] = -INFINITY;
+      if (k < K && ((pres >> k) & 1u)) {
+        const uint4 r = ld16(src + (size_t)k * astride + off);
+        const uint32_t w[4] = {r.x, r.y, r.z, r.w};
+        float d = 0.f;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const float2 f = Store<T>::unpack2(w[i]);
+          d = fmaf(x0[2 * i], f.x, d);
+          d = fmaf(x0[2 * i + 1], f.y, d);
+        }
+#pragma unroll
+        for (int o = G / 2; o > 0; o >>= 1) d += __shfl_xor_sync(kFull, d, o);
+        s[k] = d * inv_sqrt_c;
+        mx = fmaxf(mx, s[k]);
+      }
+    }
+    float den = 0.f;
+#pragma unroll
+    for (int k = 0; k < RTCC_MAX_AGENTS; ++k) {
+      if (k < K && ((pres >> k) & 1u)) {
+        s[k] = expf(s[k] - mx);
+        den += s[k];
+      }
+    }
+    float F[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) F[j] = 0.f;
+#pragma unroll
+    for (int k = 0; k < RTCC_MAX_AGENTS; ++k) {
+      if (k < K && ((pres >> k) & 1u)) {
+        const float wk = s[k] / den;
+        const uint4 r = ld16(src + (size_t)k * astride + off);
+        const uint32_t w[4] = {r.x, r.y, r.z, r.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const float2 f = Store<T>::unpack2(w[i]);
+          F[2 * i] = fmaf(wk, f.x, F[2 * i]);
+          F[2 * i + 1] = fmaf(wk, f.y, F[2 * i + 1]);
+        }
+      }
+    }
+    uint4 o;
+    o.x = Store<T>::pack2(F[0], F[1]);
+    o.y = Store<T>::pack2(F[2], F[3]);
+    o.z = Store<T>::pack2(F[4], F[5]);
+    o.w = Store<T>::pack2(F[6], F[7]);
+    return o;
+  }
+}
+
+// Warp task w of block b: cells [w * 32 / G, (w + 1) * 32 / G) of that block.
+template <typename T, bool ATTN, int G>
+__device__ __forceinline__ void block_task(const FuseBlocksArgs& a, int b, int w, int lane, unsigned pres) {
+  constexpr int CPW = 32 / G;                       // cells per warp task
+  const int cell = w * CPW + lane / G;
+  const bool valid = cell < a.cells[b];
+  // lanes of a cell past the end still join the butterfly (their data is a
+  // clamped copy of the last cell and is not stored)
+  const int c = valid ? cell : a.cells[b] - 1;
+  const size_t off = (size_t)c * (8 * G) + (size_t)(lane % G) * 8;
+  const uint4 v = fuse8<T, ATTN, G>(static_cast<const T*>(a.src[b]), a.astride[b], pres, a.K, off,
+                                    a.inv_sqrt_c[b]);
+  if (valid) *reinterpret_cast<uint4*>(static_cast<T*>(a.dst[b]) + off) = v;
+}
+
+static_assert(RTCC_MAX_BLOCKS == 3, "the task numbering below covers three blocks");
+
+template <typename T, bool ATTN>
+__global__ void __launch_bounds__(kThreads, 3) k_fuse_blocks(const __grid_constant__ FuseBlocksArgs a) {
+  pdl_trigger();
+  pdl_wait();
+  span_begin(a.span);
+  unsigned pres = 0;
+  for (int k = 0; k < a.K; ++k) pres |= (a.present[k] ? 1u : 0u) << k;
+  const int lane = threadIdx.x & 31;
+  const int warps = (int)(gridDim.x * blockDim.x) >> 5;
+  // warp tasks of the blocks, numbered block after block
+  const int e0 = a.tasks[0];
+  const int e1 = e0 + (a.n > 1 ? a.tasks[1] : 0);
+  const int e2 = e1 + (a.n > 2 ? a.tasks[2] : 0);
+  for (int t = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5); t < e2; t += warps) {
+    const int b = t < e0 ? 0 : (t < e1 ? 1 : 2);
+    const int w = t - (b == 0 ? 0 : (b == 1 ? e0 : e1));
+    switch (a.ch[b]) {                               // warp-uniform
+      case 32: block_task<T, ATTN, 4>(a, b, w, lane, pres); break;
+      case 64: block_task<T, ATTN, 8>(a, b, w, lane, pres); break;
+      case 128: block_task<T, ATTN, 16>(a, b, w, lane, pres); break;
+      default: block_task<T, ATTN, 32>(a, b, w, lane, pres); break;
+    }
+  }
+  if (a.span) {
+    __syncthreads();
+    span_end(a.span);
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_fuse_blocks(FuseBlocksArgs a, bool bf16, cudaStream_t st) {
+  if (a.K < 1 || a.K > RTCC_MAX_AGENTS || a.n < 1 || a.n > RTCC_MAX_BLOCKS) return cudaErrorInvalidValue;
+  long long work = 0;
+  for (int b = 0; b < a.n; ++b) {
+    if (a.ch[b] != 32 && a.ch[b] != 64 && a.ch[b] != 128 && a.ch[b] != 256) return cudaErrorInvalidValue;
+    if (a.cells[b] < 1 || !a.src[b] || !a.dst[b] || a.astride[b] < (long long)a.cells[b] * a.ch[b])
+      return cudaErrorInvalidValue;
+    // 16-byte loads and stores: every base and the agent stride 16-byte aligned
+    if ((reinterpret_cast<uintptr_t>(a.src[b]) | reinterpret_cast<uintptr_t>(a.dst[b])) & 15u ||
+        (a.astride[b] * 2) % 16)
+      return cudaErrorInvalidValue;
+    const int cpw = 32 / (a.ch[b] / 8);
+    a.tasks[b] = (a.cells[b] + cpw - 1) / cpw;
+    a.inv_sqrt_c[b] = 1.0f / sqrtf((float)a.ch[b]);
+    work += a.tasks[b];
+  }
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const long long per_block = kThreads / 32;
+  long long blocks = (work + per_block - 1) / per_block;
+  if (blocks > 8LL * sms) blocks = 8LL * sms;       // grid-stride beyond 8 blocks per SM
+  if (blocks < 1) blocks = 1;
+  if (bf16)
+    return a.attention ? launch_pdl(k_fuse_blocks<__nv_bfloat16, true>, dim3((unsigned)blocks), dim3(kThreads), 0, st, a)
+                       : launch_pdl(k_fuse_blocks<__nv_bfloat16, false>, dim3((unsigned)blocks), dim3(kThreads), 0, st, a);
+  return a.attention ? launch_pdl(k_fuse_blocks<__half, true>, dim3((unsigned)blocks), dim3(kThreads), 0, st, a)
+                     : launch_pdl(k_fuse_blocks<__half, false>, dim3((unsigned)blocks), dim3(kThreads), 0, st, a);
+}
+
+}  // namespace rtcc

@@ -217,6 +217,24 @@ struct FuseArgs {
 };
 cudaError_t launch_fuse_head(const FuseArgs& a, bool bf16, cudaStream_t st);
 
+// Cross-agent fusion of the backbone blocks' outputs (fuse_blocks.cu): the
+// multi-scale placement, where each block's map is fused before the neck.
+struct FuseBlocksArgs {
+  const void* src[RTCC_MAX_BLOCKS];     // block b's outputs, agent-major [K][cells][C_b]
+  long long astride[RTCC_MAX_BLOCKS];   // elements between agents
+  void* dst[RTCC_MAX_BLOCKS];           // fused map of block b [cells][C_b]
+  int cells[RTCC_MAX_BLOCKS];           // cells of block b's grid
+  int ch[RTCC_MAX_BLOCKS];              // C_b: 32, 64, 128 or 256
+  int tasks[RTCC_MAX_BLOCKS];           // set by the launcher (warp tasks per block)
+  float inv_sqrt_c[RTCC_MAX_BLOCKS];    // set by the launcher
+  int n;                                // blocks
+  const int* present;                   // device [K] presence flags
+  int K;
+  int attention;                        // 0 = max, 1 = ego-query attention
+  unsigned long long* span;             // device [3] kernel span stamps, or null
+};
+cudaError_t launch_fuse_blocks(FuseBlocksArgs a, bool bf16, cudaStream_t st);
+
 // Max fusion + head on the tensor cores (fuse_tc.cu).
 constexpr int kFuseHeadOut = 16;
 struct FuseTcParams {

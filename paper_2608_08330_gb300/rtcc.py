@@ -29,7 +29,9 @@ FP16, BF16 = 0, 1
 WAITING, RELEASED, RUNNING, FINISHED, ABSENT = range(5)
 FLAG_TIMELINE, FLAG_KEEP_FUSED, FLAG_KEEP_LAYERS, FLAG_LAYER_TIMES = 1, 2, 4, 8
 FLAG_NO_CLUSTERS, FLAG_SHORT_WAITS, FLAG_NO_BATCH, FLAG_H2D_COPY = 16, 32, 64, 128
+FLAG_MULTISCALE = 256
 TENSOR_IMAGE, TENSOR_FEAT, TENSOR_FUSED, TENSOR_LAYER0 = 0, 8, 9, 16
+TENSOR_FUSED_BLOCK0 = 10
 
 
 class rtcc_model_config(C.Structure):
