@@ -795,6 +795,12 @@ def run_ours(args):
             others[name] = quad(tl[R.MODE_RTCC], tl[R.MODE_BARRIER])
             detail[f"paired_gain_{name}"] = paired_gain(tl[R.MODE_BARRIER], tl[R.MODE_RTCC])
         ab = {"pp3": release_ab(R, "pp3"), cfg.name: release_ab(R, cfg.name)}
+        # the paper's placement: block maps fused after the join, neck once
+        msc = {}
+        for name in ("pp3", "lr5", cfg.name):
+            tl = replay_leg(R, name, args.leg_frames // 3, GAP_CAP_MS, flags=R.FLAG_MULTISCALE)
+            msc[name] = quad(tl[R.MODE_RTCC], tl[R.MODE_BARRIER])
+        detail["multiscale"] = msc
         gv = gain_validation(R, synth.get_config("pp3"))
         detail["gain_validation"] = gv
         detail["layers"] = layer_spans(R, cfg, layer_table(cfg), tflops_peak)
@@ -821,6 +827,7 @@ def run_ours(args):
                           "timing": "kernel's global-timer span, 8-agent frames"}
         line["pfn_us"] = sig(np.mean(pf) * 1e3) if pf else None
         line["release_ab_e2e"] = {k: {kk: vv[0] for kk, vv in v.items()} for k, v in ab.items()}
+        line["multiscale_ms"] = msc
         line["gain_model"] = {"r": sig(gv["r"], 3), "mae_ms": sig(gv["mae_ms"], 3)}
         if args.detail:
             os.makedirs(os.path.dirname(os.path.abspath(args.detail)), exist_ok=True)
