@@ -54,7 +54,7 @@ METRIC = "complete-detection latency p50/p99 ms RTCC vs barrier; conv TFLOP/s, f
 # dram__bytes_read.sum + dram__bytes_write.sum per k_backbone launch from an
 # ncu capture of this build, keyed by the launch's agent count; None until
 # captured (and again once the kernel changes)
-BACKBONE_TRAFFIC = {}
+BACKBONE_TRAFFIC = {8: 540_403_456, 1: 27_808_000}   # profiles/backbone_stress8.md
 WORKLOAD = "stress8"
 DATA = ("synthetic: seeded uniform + Gaussian-cluster point clouds, He-normal fp32 weights "
         "rounded to fp16, seeded arrival traces (OPV2V and the trained OpenCOOD model are not "
@@ -754,7 +754,8 @@ def run_ours(args):
                      "unit": "TFLOP/s",
                      "frac": sig(enc_tflops / tflops_peak, 3) if enc_tflops else None,
                      "peak_kind": f"{peak_kind} bf16 burst (fp16: same nominal rate)",
-                     "traffic": traffic,
+                     "traffic": traffic, "traffic_launch": f"{K}-agent launch (one-agent: "
+                                                           f"{BACKBONE_TRAFFIC.get(1)} B)",
                      "over": "all backbone launches of the instrumented frames, sum of FLOPs / "
                              "sum of CUDA-event durations"},
         "e2e": {"value": e2e_value, "unit": "ms",
