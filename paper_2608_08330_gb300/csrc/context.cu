@@ -104,6 +104,7 @@ struct rtcc_ctx {
   BackboneParams* neck_p = nullptr;
   unsigned* neck_bar = nullptr;       // [kMaxLayers + 1], zero between launches
   int* d_one = nullptr;               // [RTCC_MAX_AGENTS] = {1, 0, ...}: the head's one input
+  int post_kernels = 0;               // kernels of the post-join graph
   size_t img_elems = 0, feat_elems = 0;
   std::vector<ConvLayer> layers;      // the layer list (N tiles of a one-agent launch)
   BackboneParams* bbt[RTCC_MAX_AGENTS + 1] = {};  // launch parameters per batch size
@@ -649,9 +650,6 @@ rtcc_status build_backbone(rtcc_ctx* c) {
     if (backbone_fill(c->neck_layers, 1, c->neck_bar, c->d_err, nullptr, false, c->wait_budget, c->neck_p) !=
         cudaSuccess)
       return RTCC_E_ARG;
-    int one[RTCC_MAX_AGENTS] = {1};
-    RS(dalloc(c, &c->d_one, sizeof(one)));
-    CK(cudaMemcpy(c->d_one, one, sizeof(one), cudaMemcpyHostToDevice));
   }
   return RTCC_OK;
 }
@@ -798,9 +796,24 @@ rtcc_status capture_post(rtcc_ctx* c) {
   const bool tl = (c->cfg.flags & RTCC_FLAG_TIMELINE) != 0;
   // multi-scale placement: fuse each block's outputs, run the neck once on the
   // fused maps, then the head over that one map (the max "fusion" of a single
-  // input is the identity, so the tensor-core head kernel serves as the head)
+  // input is the identity, so the tensor-core head kernel serves as the head).
+  // Single-scale attention takes the same two steps on the 384-channel slots:
+  // the bandwidth-bound fusion writes the fused map, the tensor-core kernel
+  // runs the head over it.
+  const bool attn1 = !c->ms && c->cfg.fusion == RTCC_FUSE_ATTN && fuse_tc_chunk(c->Cf, 1) > 0 && c->fused;
   FuseBlocksArgs fb{};
-  if (c->ms) {
+  if (attn1) {
+    fb.n = 1;
+    fb.src[0] = c->feat_all;
+    fb.cells[0] = c->Wf * c->Hf;
+    fb.ch[0] = c->Cf;
+    fb.astride[0] = (long long)c->feat_elems;
+    fb.dst[0] = c->fused;
+    fb.present = c->d_present;
+    fb.K = c->K;
+    fb.attention = 1;
+    fb.span = c->fuse_span;
+  } else if (c->ms) {
     fb.n = c->cfg.n_blocks;
     for (int bi = 0; bi < fb.n; ++bi) {
       fb.src[bi] = c->block_out[bi];
@@ -814,7 +827,8 @@ rtcc_status capture_post(rtcc_ctx* c) {
     fb.attention = c->cfg.fusion == RTCC_FUSE_ATTN;
     fb.span = c->fuse_span;
   }
-  const int K_head = c->ms ? 1 : c->K;
+  const bool two_step = c->ms || attn1;
+  const int K_head = two_step ? 1 : c->K;
   FuseArgs fa{};
   fa.feats = c->d_feat_ptrs;
   fa.present = c->d_present;
@@ -834,16 +848,17 @@ rtcc_status capture_post(rtcc_ctx* c) {
   // max fusion: tensor-core kernel (TMA-staged agent tiles, max in shared
   // memory, head as an N = 16 MMA); attention fusion: CUDA-core kernel
   const int bkc = fuse_tc_chunk(c->Cf, K_head);
-  const bool use_tc = (c->ms || !fa.attention) && bkc > 0;
-  if (c->ms && !use_tc) return RTCC_E_ARG;
+  const bool use_tc = (two_step || !fa.attention) && bkc > 0;
+  if (two_step && !use_tc) return RTCC_E_ARG;
   FuseTcParams tp{};
   if (use_tc) {
     const int swz = bkc * 2;                    // 128- or 64-byte rows
     for (int k = 0; k < K_head; ++k)
-      CK(tmap_2d(&tp.feat[k], c->ms ? c->neck_out : c->br[k].feat, c->bf16, (uint64_t)c->Cf,
+      CK(tmap_2d(&tp.feat[k], c->ms ? c->neck_out : (attn1 ? c->fused : c->br[k].feat), c->bf16,
+                 (uint64_t)c->Cf,
                  (uint64_t)fa.cells, (uint32_t)bkc, 128u, swz));
     CK(tmap_2d(&tp.wmap, c->head_w16, c->bf16, (uint64_t)c->Cf, 16u, (uint32_t)bkc, 16u, swz));
-    tp.present = c->ms ? c->d_one : c->d_present;
+    tp.present = two_step ? c->d_one : c->d_present;
     tp.K = K_head;
     tp.C = c->Cf;
     tp.cells = fa.cells;
@@ -851,13 +866,13 @@ rtcc_status capture_post(rtcc_ctx* c) {
     tp.stages = fuse_tc_stages(c->Cf, K_head);
     tp.head_b = c->head_b;
     tp.head_out = c->head_out;
-    tp.fused = c->ms ? nullptr : c->fused;
+    tp.fused = two_step ? nullptr : c->fused;
     tp.keys = c->keys;
     tp.hist0 = c->hist0;
     tp.cls_thresh = c->cfg.cls_thresh;
     tp.anchors = c->cfg.anchors;
     tp.err = c->d_err;
-    tp.span = c->ms ? nullptr : c->fuse_span;
+    tp.span = two_step ? nullptr : c->fuse_span;
   }
   DecodeArgs da{};
   da.head = c->head_out;
@@ -893,10 +908,10 @@ rtcc_status capture_post(rtcc_ctx* c) {
   cudaError_t e = cudaSuccess;
   if (tl) e = record_node(c->ev_post0, c->post);
   if (e == cudaSuccess && tl) e = record_node(c->ev_fuse0, c->post);
-  if (c->ms) {
+  if (two_step) {
     if (e == cudaSuccess) e = launch_fuse_blocks(fb, c->bf16, c->post);
     if (e == cudaSuccess && tl) e = record_node(c->ev_fuse1, c->post);
-    if (e == cudaSuccess) e = launch_backbone(*c->neck_p, c->bf16, c->post);
+    if (e == cudaSuccess && c->ms) e = launch_backbone(*c->neck_p, c->bf16, c->post);
     if (e == cudaSuccess) e = launch_fuse_max_head(tp, c->bf16, c->post);
   } else {
     if (e == cudaSuccess) {
@@ -910,6 +925,8 @@ rtcc_status capture_post(rtcc_ctx* c) {
   if (e == cudaSuccess) e = launch_decode(da, c->post);
   if (e == cudaSuccess && c->dec_boxes) e = launch_nms(na, c->post);
   if (e == cudaSuccess && tl) e = record_node(c->ev_post1, c->post);
+  // fusion(s) and head, decode, NMS
+  c->post_kernels = (two_step ? (c->ms ? 3 : 2) : 1) + 1 + (c->dec_boxes ? 1 : 0);
   cudaGraph_t graph = nullptr;
   cudaError_t e2 = cudaStreamEndCapture(c->post, &graph);
   if (e != cudaSuccess || e2 != cudaSuccess) {
@@ -1004,7 +1021,15 @@ rtcc_status init_impl(rtcc_ctx* c, const float* weights) {
   for (int k = 0; k < c->K; ++k) fp[k] = c->br[k].feat;
   CK(cudaMemcpy(c->d_feat_ptrs, fp, sizeof(fp), cudaMemcpyHostToDevice));
   RS(dalloc(c, &c->head_out, (size_t)cells_f * 16 * sizeof(float)));
-  if (g.flags & RTCC_FLAG_KEEP_FUSED) RS(dalloc(c, &c->fused, (size_t)cells_f * c->Cf * 2));
+  // attention fusion writes the fused map (the head then reads it), so it always
+  // has one; max fusion keeps it only for parity read-backs
+  if ((g.flags & RTCC_FLAG_KEEP_FUSED) || (g.fusion == RTCC_FUSE_ATTN && !c->ms))
+    RS(dalloc(c, &c->fused, (size_t)cells_f * c->Cf * 2));
+  {
+    int one[RTCC_MAX_AGENTS] = {1};
+    RS(dalloc(c, &c->d_one, sizeof(one)));
+    CK(cudaMemcpy(c->d_one, one, sizeof(one), cudaMemcpyHostToDevice));
+  }
   const size_t nkeys = decode_key_capacity(cells_f * g.anchors);
   RS(dalloc(c, &c->keys, nkeys * sizeof(uint32_t)));
   CK(cudaMemset(c->keys, 0xFF, nkeys * sizeof(uint32_t)));   // padding stays invalid
@@ -1740,8 +1765,7 @@ int32_t rtcc_kernels_per_frame(rtcc_ctx* c, int32_t n_present) {
   // pillar chain per branch; the backbone launches of the last frame (one per
   // branch when none was batched); fusion, decode (and NMS)
   const int bb = c->n_launches > 0 ? c->n_launches : n_present;
-  // multi-scale: block fusion and the neck's launch before the head
-  return n_present * 5 + bb + 2 + (c->dec_boxes ? 1 : 0) + (c->ms ? 2 : 0);
+  return n_present * 5 + bb + c->post_kernels;
 }
 
 rtcc_status rtcc_test_unreachable_wait(rtcc_ctx* c) {

@@ -49,34 +49,39 @@ __device__ __forceinline__ uint32_t max2<__nv_bfloat16>(uint32_t a, uint32_t b) 
 
 __device__ __forceinline__ uint4 ld16(const void* p) { return *reinterpret_cast<const uint4*>(p); }
 
-// One thread's 8 channels of one cell.  G = C / 8 threads share the cell
-// (G in {4, 8, 16, 32}); they are lanes [g0, g0 + G) of the warp.
-template <typename T, bool ATTN, int G>
-__device__ __forceinline__ uint4 fuse8(const T* src, long long astride, const unsigned pres, int K,
-                                       size_t off, float inv_sqrt_c) {
+// One thread's 8 * NV channels (NV 16-byte vectors) of one cell.  G threads
+// share the cell (C = 8 * NV * G); they are lanes [g0, g0 + G) of the warp.
+template <typename T, bool ATTN, int G, int NV>
+__device__ __forceinline__ void fuse_vec(const T* src, long long astride, const unsigned pres, int K,
+                                         size_t off, float inv_sqrt_c, uint4* out) {
   if (!ATTN) {
-    uint4 m = make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+    for (int v = 0; v < NV; ++v) out[v] = make_uint4(0u, 0u, 0u, 0u);
     for (int k = 0; k < K; ++k) {
       if (!((pres >> k) & 1u)) continue;
-      const uint4 r = ld16(src + (size_t)k * astride + off);
-      m.x = max2<T>(m.x, r.x);
-      m.y = max2<T>(m.y, r.y);
-      m.z = max2<T>(m.z, r.z);
-      m.w = max2<T>(m.w, r.w);
+#pragma unroll
+      for (int v = 0; v < NV; ++v) {
+        const uint4 r = ld16(src + (size_t)k * astride + off + 8 * v);
+        out[v].x = max2<T>(out[v].x, r.x);
+        out[v].y = max2<T>(out[v].y, r.y);
+        out[v].z = max2<T>(out[v].z, r.z);
+        out[v].w = max2<T>(out[v].w, r.w);
+      }
     }
-    return m;
   } else {
     // two passes over the agents (scores, then the weighted sum, reloading
     // each vector -- an L1 hit) keep one agent's vector live at a time
-    float x0[8];
-    {
-      const uint4 r = ld16(src + off);                // the ego agent 0 is present
+    constexpr int E = 8 * NV;
+    float x0[E];
+#pragma unroll
+    for (int v = 0; v < NV; ++v) {
+      const uint4 r = ld16(src + off + 8 * v);            // the ego agent 0 is present
       const uint32_t w[4] = {r.x, r.y, r.z, r.w};
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
         const float2 f = Store<T>::unpack2(w[i]);
-        x0[2 * i] = f.x;
-        x0[2 * i + 1] = f.y;
+        x0[8 * v + 2 * i] = f.x;
+        x0[8 * v + 2 * i + 1] = f.y;
       }
     }
     float s[RTCC_MAX_AGENTS];
@@ -85,14 +90,17 @@ __device__ __forceinline__ uint4 fuse8(const T* src, long long astride, const un
     for (int k = 0; k < RTCC_MAX_AGENTS; ++k) {
       s[k] = -INFINITY;
       if (k < K && ((pres >> k) & 1u)) {
-        const uint4 r = ld16(src + (size_t)k * astride + off);
-        const uint32_t w[4] = {r.x, r.y, r.z, r.w};
         float d = 0.f;
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const float2 f = Store<T>::unpack2(w[i]);
-          d = fmaf(x0[2 * i], f.x, d);
-          d = fmaf(x0[2 * i + 1], f.y, d);
+        for (int v = 0; v < NV; ++v) {
+          const uint4 r = ld16(src + (size_t)k * astride + off + 8 * v);
+          const uint32_t w[4] = {r.x, r.y, r.z, r.w};
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const float2 f = Store<T>::unpack2(w[i]);
+            d = fmaf(x0[8 * v + 2 * i], f.x, d);
+            d = fmaf(x0[8 * v + 2 * i + 1], f.y, d);
+          }
         }
 #pragma unroll
         for (int o = G / 2; o > 0; o >>= 1) d += __shfl_xor_sync(kFull, d, o);
@@ -108,34 +116,38 @@ __device__ __forceinline__ uint4 fuse8(const T* src, long long astride, const un
         den += s[k];
       }
     }
-    float F[8];
+    float F[E];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) F[j] = 0.f;
+    for (int j = 0; j < E; ++j) F[j] = 0.f;
 #pragma unroll
     for (int k = 0; k < RTCC_MAX_AGENTS; ++k) {
       if (k < K && ((pres >> k) & 1u)) {
         const float wk = s[k] / den;
-        const uint4 r = ld16(src + (size_t)k * astride + off);
-        const uint32_t w[4] = {r.x, r.y, r.z, r.w};
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const float2 f = Store<T>::unpack2(w[i]);
-          F[2 * i] = fmaf(wk, f.x, F[2 * i]);
-          F[2 * i + 1] = fmaf(wk, f.y, F[2 * i + 1]);
+        for (int v = 0; v < NV; ++v) {
+          const uint4 r = ld16(src + (size_t)k * astride + off + 8 * v);
+          const uint32_t w[4] = {r.x, r.y, r.z, r.w};
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const float2 f = Store<T>::unpack2(w[i]);
+            F[8 * v + 2 * i] = fmaf(wk, f.x, F[8 * v + 2 * i]);
+            F[8 * v + 2 * i + 1] = fmaf(wk, f.y, F[8 * v + 2 * i + 1]);
+          }
         }
       }
     }
-    uint4 o;
-    o.x = Store<T>::pack2(F[0], F[1]);
-    o.y = Store<T>::pack2(F[2], F[3]);
-    o.z = Store<T>::pack2(F[4], F[5]);
-    o.w = Store<T>::pack2(F[6], F[7]);
-    return o;
+#pragma unroll
+    for (int v = 0; v < NV; ++v) {
+      out[v].x = Store<T>::pack2(F[8 * v + 0], F[8 * v + 1]);
+      out[v].y = Store<T>::pack2(F[8 * v + 2], F[8 * v + 3]);
+      out[v].z = Store<T>::pack2(F[8 * v + 4], F[8 * v + 5]);
+      out[v].w = Store<T>::pack2(F[8 * v + 6], F[8 * v + 7]);
+    }
   }
 }
 
 // Warp task w of block b: cells [w * 32 / G, (w + 1) * 32 / G) of that block.
-template <typename T, bool ATTN, int G>
+template <typename T, bool ATTN, int G, int NV>
 __device__ __forceinline__ void block_task(const FuseBlocksArgs& a, int b, int w, int lane, unsigned pres) {
   constexpr int CPW = 32 / G;                       // cells per warp task
   const int cell = w * CPW + lane / G;
@@ -143,16 +155,21 @@ __device__ __forceinline__ void block_task(const FuseBlocksArgs& a, int b, int w
   // lanes of a cell past the end still join the butterfly (their data is a
   // clamped copy of the last cell and is not stored)
   const int c = valid ? cell : a.cells[b] - 1;
-  const size_t off = (size_t)c * (8 * G) + (size_t)(lane % G) * 8;
-  const uint4 v = fuse8<T, ATTN, G>(static_cast<const T*>(a.src[b]), a.astride[b], pres, a.K, off,
-                                    a.inv_sqrt_c[b]);
-  if (valid) *reinterpret_cast<uint4*>(static_cast<T*>(a.dst[b]) + off) = v;
+  const size_t off = (size_t)c * (8 * NV * G) + (size_t)(lane % G) * (8 * NV);
+  uint4 v[NV];
+  fuse_vec<T, ATTN, G, NV>(static_cast<const T*>(a.src[b]), a.astride[b], pres, a.K, off, a.inv_sqrt_c[b], v);
+  if (valid) {
+#pragma unroll
+    for (int i = 0; i < NV; ++i) reinterpret_cast<uint4*>(static_cast<T*>(a.dst[b]) + off)[i] = v[i];
+  }
 }
 
 static_assert(RTCC_MAX_BLOCKS == 3, "the task numbering below covers three blocks");
 
-template <typename T, bool ATTN>
-__global__ void __launch_bounds__(kThreads, 3) k_fuse_blocks(const __grid_constant__ FuseBlocksArgs a) {
+// WIDE: one 384-channel map (the single-scale 384-channel slots; 16 threads of
+// 24 channels per cell); otherwise block maps of 32 to 256 channels.
+template <typename T, bool ATTN, bool WIDE>
+__global__ void __launch_bounds__(kThreads, WIDE ? 2 : 3) k_fuse_blocks(const __grid_constant__ FuseBlocksArgs a) {
   pdl_trigger();
   pdl_wait();
   span_begin(a.span);
@@ -167,11 +184,15 @@ __global__ void __launch_bounds__(kThreads, 3) k_fuse_blocks(const __grid_consta
   for (int t = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5); t < e2; t += warps) {
     const int b = t < e0 ? 0 : (t < e1 ? 1 : 2);
     const int w = t - (b == 0 ? 0 : (b == 1 ? e0 : e1));
-    switch (a.ch[b]) {                               // warp-uniform
-      case 32: block_task<T, ATTN, 4>(a, b, w, lane, pres); break;
-      case 64: block_task<T, ATTN, 8>(a, b, w, lane, pres); break;
-      case 128: block_task<T, ATTN, 16>(a, b, w, lane, pres); break;
-      default: block_task<T, ATTN, 32>(a, b, w, lane, pres); break;
+    if (WIDE) {
+      block_task<T, ATTN, 16, 3>(a, b, w, lane, pres);
+    } else {
+      switch (a.ch[b]) {                             // warp-uniform
+        case 32: block_task<T, ATTN, 4, 1>(a, b, w, lane, pres); break;
+        case 64: block_task<T, ATTN, 8, 1>(a, b, w, lane, pres); break;
+        case 128: block_task<T, ATTN, 16, 1>(a, b, w, lane, pres); break;
+        default: block_task<T, ATTN, 32, 1>(a, b, w, lane, pres); break;
+      }
     }
   }
   if (a.span) {
@@ -185,15 +206,18 @@ __global__ void __launch_bounds__(kThreads, 3) k_fuse_blocks(const __grid_consta
 cudaError_t launch_fuse_blocks(FuseBlocksArgs a, bool bf16, cudaStream_t st) {
   if (a.K < 1 || a.K > RTCC_MAX_AGENTS || a.n < 1 || a.n > RTCC_MAX_BLOCKS) return cudaErrorInvalidValue;
   long long work = 0;
+  const bool wide = a.ch[0] == 384;
+  if (wide && a.n != 1) return cudaErrorInvalidValue;
   for (int b = 0; b < a.n; ++b) {
-    if (a.ch[b] != 32 && a.ch[b] != 64 && a.ch[b] != 128 && a.ch[b] != 256) return cudaErrorInvalidValue;
+    if (!wide && a.ch[b] != 32 && a.ch[b] != 64 && a.ch[b] != 128 && a.ch[b] != 256)
+      return cudaErrorInvalidValue;
     if (a.cells[b] < 1 || !a.src[b] || !a.dst[b] || a.astride[b] < (long long)a.cells[b] * a.ch[b])
       return cudaErrorInvalidValue;
     // 16-byte loads and stores: every base and the agent stride 16-byte aligned
     if ((reinterpret_cast<uintptr_t>(a.src[b]) | reinterpret_cast<uintptr_t>(a.dst[b])) & 15u ||
         (a.astride[b] * 2) % 16)
       return cudaErrorInvalidValue;
-    const int cpw = 32 / (a.ch[b] / 8);
+    const int cpw = wide ? 2 : 32 / (a.ch[b] / 8);   // cells per warp task
     a.tasks[b] = (a.cells[b] + cpw - 1) / cpw;
     a.inv_sqrt_c[b] = 1.0f / sqrtf((float)a.ch[b]);
     work += a.tasks[b];
@@ -205,11 +229,19 @@ cudaError_t launch_fuse_blocks(FuseBlocksArgs a, bool bf16, cudaStream_t st) {
   long long blocks = (work + per_block - 1) / per_block;
   if (blocks > 8LL * sms) blocks = 8LL * sms;       // grid-stride beyond 8 blocks per SM
   if (blocks < 1) blocks = 1;
-  if (bf16)
-    return a.attention ? launch_pdl(k_fuse_blocks<__nv_bfloat16, true>, dim3((unsigned)blocks), dim3(kThreads), 0, st, a)
-                       : launch_pdl(k_fuse_blocks<__nv_bfloat16, false>, dim3((unsigned)blocks), dim3(kThreads), 0, st, a);
-  return a.attention ? launch_pdl(k_fuse_blocks<__half, true>, dim3((unsigned)blocks), dim3(kThreads), 0, st, a)
-                     : launch_pdl(k_fuse_blocks<__half, false>, dim3((unsigned)blocks), dim3(kThreads), 0, st, a);
+  const dim3 g((unsigned)blocks), t(kThreads);
+  if (bf16) {
+    if (wide)
+      return a.attention ? launch_pdl(k_fuse_blocks<__nv_bfloat16, true, true>, g, t, 0, st, a)
+                         : launch_pdl(k_fuse_blocks<__nv_bfloat16, false, true>, g, t, 0, st, a);
+    return a.attention ? launch_pdl(k_fuse_blocks<__nv_bfloat16, true, false>, g, t, 0, st, a)
+                       : launch_pdl(k_fuse_blocks<__nv_bfloat16, false, false>, g, t, 0, st, a);
+  }
+  if (wide)
+    return a.attention ? launch_pdl(k_fuse_blocks<__half, true, true>, g, t, 0, st, a)
+                       : launch_pdl(k_fuse_blocks<__half, false, true>, g, t, 0, st, a);
+  return a.attention ? launch_pdl(k_fuse_blocks<__half, true, false>, g, t, 0, st, a)
+                     : launch_pdl(k_fuse_blocks<__half, false, false>, g, t, 0, st, a);
 }
 
 }  // namespace rtcc
