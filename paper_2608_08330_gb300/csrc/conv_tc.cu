@@ -1220,24 +1220,25 @@ cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, int n_batch, uns
   P->grid = any_dsm ? grid_cl : grid_sm;
   // Item ranges.  Every layer's items are dealt round-robin over all CTAs,
   // except the deconvs of the shallower blocks (those that do not read the
-  // deepest block): when the conv layers leave at least 8 CTAs without items,
-  // those CTAs take the early deconvs, which then run alongside the deeper
-  // conv blocks instead of after them.  A layer waits for the items of the
-  // one layer it reads.
-  int main_max = 0, last_conv = -1;
-  for (int i = 0; i < P->n_layers; ++i) {
-    const LayerDesc& D = P->L[i];
-    if (D.kind != DECONV) {
-      main_max = std::max(main_max, n_batch * D.ipa);
-      last_conv = i;
-    }
-  }
-  const bool background = P->grid - main_max >= 8;
+  // deepest block): when the conv layers that can run at the same time as
+  // such a deconv (those after the layer it reads) leave at least 8 CTAs
+  // without items, those CTAs take the deconv, which then runs alongside the
+  // deeper conv blocks instead of after them (a CTA with no items in a layer
+  // skips it without waiting).  A layer waits for the items of the one layer
+  // it reads.
+  int last_conv = -1;
+  for (int i = 0; i < P->n_layers; ++i)
+    if (P->L[i].kind != DECONV) last_conv = i;
   for (int i = 0; i < P->n_layers; ++i) {
     LayerDesc& D = P->L[i];
     D.cta_lo = 0;
     D.cta_hi = P->grid;
-    if (background && D.kind == DECONV && D.wait_layers - 1 != last_conv) D.cta_lo = main_max;
+    if (D.kind == DECONV && D.wait_layers >= 1 && D.wait_layers - 1 != last_conv) {
+      int conc_max = 0;                            // conv items beside this deconv
+      for (int j = D.wait_layers; j < P->n_layers; ++j)
+        if (P->L[j].kind != DECONV) conc_max = std::max(conc_max, n_batch * P->L[j].ipa);
+      if (P->grid - conc_max >= 8) D.cta_lo = conc_max;
+    }
     if (D.wait_layers > P->n_layers || D.wait_layers > (int)i) return cudaErrorInvalidValue;
     D.wait_items = 0;
     if (D.wait_layers > 0) {
