@@ -50,6 +50,7 @@ enum : int {
   ERR_WAIT_EPILOGUE = 4,
   ERR_BOUNDS = 8,
   ERR_WAIT_FUSE = 16,
+  ERR_WAIT_PILLAR = 32,
 };
 
 // Upper bound on any in-kernel wait, in SM clock cycles (about 1 s at the

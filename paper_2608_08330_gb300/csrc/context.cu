@@ -47,7 +47,7 @@ struct Branch {
   float* splitk_ws = nullptr;      // split-K partials of this branch's own launches
   int* splitk_cnt = nullptr;       // split-K per-tile arrival counters
   unsigned* grid_bar = nullptr;      // inside frame_zero: per-layer counters + exit count
-  void* frame_zero = nullptr;         // [kFrameZeroBytes] cleared at the start of every branch graph
+  void* frame_zero = nullptr;         // [kFrameZeroBytes] cleared by every pass's first pillar kernel
   unsigned long long* stamps = nullptr;   // RTCC_FLAG_LAYER_TIMES: layer starts, then ends
   BackboneParams* bb = nullptr;    // backbone kernel parameters of this agent alone
   cudaStream_t st = nullptr;
@@ -223,6 +223,8 @@ rtcc_status validate_config(const rtcc_model_config& c) {
   if (c.n_agents < 1 || c.n_agents > RTCC_MAX_AGENTS) return RTCC_E_ARG;
   if (c.grid_w < 1 || c.grid_h < 1 || c.grid_w > 4096 || c.grid_h > 4096) return RTCC_E_ARG;
   if (!(c.pillar > 0.f) || !(c.x_max > c.x_min) || !(c.y_max > c.y_min) || !(c.z_max > c.z_min))
+    return RTCC_E_ARG;
+  if (!grid_coords_ok(c.x_min, c.y_min, c.z_min, c.z_max, c.pillar, c.grid_w, c.grid_h))
     return RTCC_E_ARG;
   if (c.max_pillars < 1 || c.max_pts < 1 || c.max_pts > 32) return RTCC_E_ARG;
   if (!pow2_in(c.pfn_ch, {32, 64})) return RTCC_E_ARG;
@@ -671,18 +673,25 @@ rtcc_status build_branch(rtcc_ctx* c, int k) {
   p.P = c->P;
   p.N = c->N;
   p.C = c->Cp;
-  RS(dalloc(c, &p.cell_of, (size_t)c->cap * 4));
+  const size_t tiles = (size_t)scan_tiles(c->cap);
+  RS(dalloc(c, &p.cell_of, scan_pad(c->cap) * 4));
+  RS(dalloc(c, &p.slot_of, scan_pad(c->cap) * 4));
   RS(dalloc(c, &p.cnt_cell, (size_t)cells * 4));
   RS(dalloc(c, &p.first_cell, (size_t)cells * 4));
-  RS(dalloc(c, &p.c2p, (size_t)cells * 4));
-  RS(dalloc(c, &p.blocksum, (size_t)scan_blocks(c->cap) * sizeof(int2)));
-  RS(dalloc(c, &p.items, (size_t)scan_blocks(c->cap) * kScanTile * sizeof(int2)));
-  RS(dalloc(c, &p.pcnt_raw, (size_t)c->P * 4));
-  RS(dalloc(c, &p.poff, (size_t)c->P * 4));
-  RS(dalloc(c, &p.cursor, (size_t)c->P * 4));
-  RS(dalloc(c, &p.list, (size_t)c->cap * 4));
+  RS(dalloc(c, &p.cell_loc, (size_t)cells * sizeof(int2)));
+  RS(dalloc(c, &p.tile_agg, tiles * kAggStride * sizeof(unsigned long long)));
+  RS(dalloc(c, &p.pillar_rec, (size_t)c->P * sizeof(int4)));
+  RS(dalloc(c, &p.touched, (size_t)(c->cap > 0 ? c->cap : 1) * 4));
+  RS(dalloc(c, &p.ntouched, 4));
+  RS(dalloc(c, &p.list, (size_t)(c->cap > 0 ? c->cap : 1) * 4));
+  RS(dalloc(c, &p.bucket, (size_t)c->P * c->N * sizeof(float4)));
   RS(dalloc(c, &p.np_prev, 4));
   CK(cudaMemset(p.np_prev, 0, 4));
+  // valid cells and empty pillars from the start (read only after a wait ran out)
+  CK(cudaMemset(p.pillar_rec, 0, (size_t)c->P * sizeof(int4)));
+  CK(cudaMemset(p.touched, 0, (size_t)(c->cap > 0 ? c->cap : 1) * 4));
+  CK(cudaMemset(p.cell_loc, 0x7F, (size_t)cells * sizeof(int2)));
+  p.err = c->d_err;
   p.clear_all = 0;                              // image and cell2pillar start cleared below
   p.present_flag = c->d_present + k;
   if (g.flags & RTCC_FLAG_TIMELINE) {
@@ -690,12 +699,15 @@ rtcc_status build_branch(rtcc_ctx* c, int k) {
     CK(cudaMemset(p.pfn_span, 0, 3 * sizeof(unsigned long long)));
   }
   RS(dalloc(c, &p.pillar_cell, (size_t)c->P * 4));
+  CK(cudaMemset(p.pillar_cell, 0, (size_t)c->P * 4));
   RS(dalloc(c, &p.pcount, (size_t)c->P * 4));
-  // words cleared at the start of every branch graph (one memset): the pillar
-  // stats [8] and the backbone's per-layer arrival counters and exit count
+  // words the first pillar kernel of every pass clears: the pillar stats [8]
+  // and the backbone's per-layer arrival counters and exit count
   RS(dalloc(c, &b.frame_zero, kFrameZeroBytes));
   CK(cudaMemset(b.frame_zero, 0, kFrameZeroBytes));
   p.stats = reinterpret_cast<int*>(b.frame_zero);
+  p.zero_words = p.stats;                       // cleared by the pass's first kernel
+  p.n_zero = (int)(kFrameZeroBytes / sizeof(int));
   RS(dalloc(c, &p.cell2pillar, (size_t)cells * 4));
   CK(cudaMemset(p.cnt_cell, 0, (size_t)cells * 4));
   CK(cudaMemset(p.first_cell, 0x7F, (size_t)cells * 4));
@@ -754,10 +766,10 @@ rtcc_status capture_branch_graph(rtcc_ctx* c, int k, const PillarBufs& pb, bool 
   CK(cudaStreamBeginCapture(b.st, cudaStreamCaptureModeRelaxed));
   cudaError_t e = cudaSuccess;
   if (tl) e = record_node(b.ev_start, b.st);
-  // one memset of the per-frame words, then kernels only, so that the pillar
-  // chain and the backbone are programmatic dependent launches of each other
-  if (e == cudaSuccess) e = cudaMemsetAsync(b.frame_zero, 0, kFrameZeroBytes, b.st);
-  if (e == cudaSuccess) e = launch_pillarise(pb, gg, c->pfn_w, c->pfn_b, c->bf16, c->d_err, b.st);
+  // kernels only (the first one clears the per-frame words), so that the
+  // pillar chain and the backbone are programmatic dependent launches of each
+  // other
+  if (e == cudaSuccess) e = launch_pillarise(pb, gg, c->pfn_w, c->pfn_b, c->bf16, b.st);
   if (e == cudaSuccess && tl) e = record_node(b.ev_bb0, b.st);
   if (e == cudaSuccess && with_bb) e = launch_backbone(*b.bb, c->bf16, b.st);
   if (e == cudaSuccess && tl) e = record_node(b.ev_bb1, b.st);
@@ -1560,6 +1572,16 @@ rtcc_status rtcc_wait_detection(rtcc_ctx* c, int32_t timeout_ms, rtcc_box* out, 
       if (c->br[k].splitk_cnt) CK(cudaMemset(c->br[k].splitk_cnt, 0, c->splitk_cnt_bytes));
     if (c->batch_cnt) CK(cudaMemset(c->batch_cnt, 0, (size_t)c->K * c->splitk_cnt_bytes));
     CK(cudaMemset(c->batch_bar, 0, (kMaxLayers + 1) * sizeof(unsigned)));
+    // the pillar passes' per-cell state and their image cells, as at allocation
+    const size_t cells = (size_t)c->W * c->H;
+    for (int k = 0; k < c->K; ++k) {
+      const PillarBufs& p = c->br[k].pb;
+      CK(cudaMemset(p.cnt_cell, 0, cells * 4));
+      CK(cudaMemset(p.first_cell, 0x7F, cells * 4));
+      CK(cudaMemset(p.cell2pillar, 0xFF, cells * 4));
+      CK(cudaMemset(p.np_prev, 0, 4));
+      CK(cudaMemset(p.image, 0, (size_t)c->img_elems * 2));
+    }
     return RTCC_E_DEVICE;
   }
   return RTCC_OK;

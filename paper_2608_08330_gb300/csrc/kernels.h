@@ -35,6 +35,9 @@ inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
 struct GridGeom {
   float x_min, y_min, z_min, z_max, v;
   int W, H;
+  // fixed-point scales of the PFN's means (powers of two, set by
+  // launch_pillarise): 32 x v x qxy and 32 x (z_max - z_min) x qz <= 2^30
+  float qxy, qz, qxy_inv, qz_inv;
 };
 
 // Buffers of one pillarisation + PFN + scatter pass.  `cap` is the payload
@@ -43,23 +46,30 @@ struct PillarBufs {
   const float4* pts;     // [cap] device payload (x, y, z, intensity)
   const int* n_hdr;      // device: number of valid points
   // scratch
-  int* cell_of;          // [cap]   cell of each point, -1 out of range
+  int* cell_of;          // [scan_pad(cap)] cell of each point, -1 out of range
+  int* slot_of;          // [scan_pad(cap)] the point's slot in its cell's list
   int* cnt_cell;         // [H*W]   points per cell (0 between passes)
   int* first_cell;       // [H*W]   first point index per cell (kFirstInit between passes)
-  int* c2p;              // [H*W]   pillar id of a cell (valid where cnt_cell > 0)
-  int2* items;           // [cap]   per point (first-point flag, its cell's count)
-  int2* blocksum;        // [nblk]  per-tile (#first points, #points of their cells)
-  int* pcnt_raw;         // [P]     points of the pillar's cell before the N_max cap
-  int* poff;             // [P]     offset of the pillar's point list
-  int* cursor;           // [P]     fill cursor
-  int* list;             // [cap]   point indices grouped by pillar
+  int2* cell_loc;        // [H*W]   per cell the pass opened: (tile << 12 | pillar rank
+                         //         in the tile, list offset in the tile)
+  unsigned long long* tile_agg;   // [scan_tiles(cap) * kAggStride] the scan's published tile
+                                  // aggregates, one per 128-byte line
+  int4* pillar_rec;      // [P]     (cell, points before the N_max cap, list offset,
+                         //         column | row << 16)
+  int* touched;          // [cap]   cell of every pillar id of the pass, kept or not
+  int* ntouched;         // [1]     pillar ids of the pass
+  int* list;             // [cap]   point indices grouped by pillar (pillars over N_max points)
+  float4* bucket;        // [P][N]  the points of each pillar of at most N_max points
   int* np_prev;          // [1]     pillars the previous pass wrote into image and
                          //         cell2pillar (0 at allocation)
+  int* err;              // optional: error word (a scan wait ran out: bit 32)
   // outputs
   int* pillar_cell;      // [P]
   int* pcount;           // [P]     kept points
   int* stats;            // [8]     n, in_range, n_pillars, kept, 0, 0, ncap drops,
                          //         points of kept pillars before the N_max cap
+  int* zero_words;       // [n_zero] words the pass's first kernel clears; begins with
+  int n_zero;            //         the 8 stats words (zero_words == stats, n_zero >= 8)
   int* cell2pillar;      // [H*W]     -1 where no kept pillar
   void* image;           // [H][W][C] storage type, zeros where no kept pillar
   int* present_flag;     // optional: set to 1 by the pass (the agent's slot is filled)
@@ -78,13 +88,32 @@ struct PillarBufs {
 };
 
 constexpr int kFirstInit = 0x7F7F7F7F;   // memset byte 0x7F
-constexpr int kScanTile = 1024;          // points per scan block
-inline int scan_blocks(int cap) { return (cap + kScanTile - 1) / kScanTile; }
+// The scan takes tiles of 4 points per thread, 256 to 1024 threads.
+constexpr int kScanTileMin = 1024;
+constexpr int kAggStride = 16;           // words between two tiles' aggregates (one line each)
+constexpr int kScanPadUnit = 4096;
+// Most tiles a pass over cap points has; points the per-point scratch holds.
+inline int scan_tiles(int cap) { return cap > 0 ? (cap + kScanTileMin - 1) / kScanTileMin : 1; }
+inline size_t scan_pad(int cap) {   // whole tiles of any size up to 4096 points
+  return ((size_t)(cap > 0 ? cap : 1) + kScanPadUnit - 1) / kScanPadUnit * kScanPadUnit +
+         kScanPadUnit;
+}
+// Grid bounds the PFN's fixed-point means accept: every bound within 2^20
+// pillar edges of 0 (and z within 2^20 z-ranges), so that float32 rounding
+// keeps a point within one edge of its pillar's centre.
+inline bool grid_coords_ok(double x_min, double y_min, double z_min, double z_max, double v,
+                           int W, int H) {
+  const double lim = v * 1048576.0, zlim = (z_max - z_min) * 1048576.0;
+  auto in = [](double a, double l) { return a >= -l && a <= l; };
+  return in(x_min, lim) && in(x_min + W * v, lim) && in(y_min, lim) && in(y_min + H * v, lim) &&
+         in(z_min, zlim) && in(z_max, zlim);
+}
 
-// Enqueue the 5 pillar kernels (cells, block sums, scan, fill, PFN; the PFN
-// writes each pillar's vector into the BEV pseudo-image).
+// Enqueue the 3 pillar kernels (cells; scan + list fill; PFN, which writes
+// each pillar's vector into the BEV pseudo-image).  The first kernel clears
+// b.zero_words, so the caller needs no memset per pass.
 cudaError_t launch_pillarise(const PillarBufs& b, const GridGeom& g, const float* pfn_w,
-                             const float* pfn_b, bool bf16, int* err, cudaStream_t st);
+                             const float* pfn_b, bool bf16, cudaStream_t st);
 
 // ---------------------------------------------------------------------------
 // implicit-GEMM convolution on tcgen05 (3x3 stride 1/2 and deconv k = s)

@@ -8,8 +8,8 @@
 // this entry point takes its scratch from one fixed array in device global
 // memory that the library reserves when it is loaded, instead of calling any
 // allocator.  The array is sized for grids up to 65,536 cells, payloads up to
-// 131,072 points, 16,384 pillars and 64 PFN channels (about 3.1 MB, held on
-// every GPU that loads the library until the process exits).
+// 131,072 points, 16,384 pillars of up to 32 points and 64 PFN channels (about
+// 11.8 MB, held on every GPU that loads the library until the process exits).
 //
 // The kernels are the ones rtcc_payload_complete runs (launch_pillarise); only
 // the scratch pointers differ.  All calls share the one array: a call clears
@@ -29,24 +29,26 @@ constexpr int kMaxCells = 65536;
 constexpr int kMaxPoints = 131072;
 constexpr int kMaxPillars = 16384;
 constexpr int kMaxCh = 64;
-constexpr int kMaxScanBlocks = (kMaxPoints + kScanTile - 1) / kScanTile;
+constexpr int kMaxPts = 32;
+constexpr int kMaxTiles = (kMaxPoints + kScanTileMin - 1) / kScanTileMin;
+constexpr size_t kPad = (kMaxPoints + kScanPadUnit - 1) / kScanPadUnit * kScanPadUnit + kScanPadUnit;
 
 constexpr size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
-// byte offsets of the regions inside the static array (each 256-byte aligned)
 constexpr size_t kOffN = 0;
 constexpr size_t kOffCellOf = align256(kOffN + 16);
-constexpr size_t kOffList = align256(kOffCellOf + 4ull * kMaxPoints);
-constexpr size_t kOffCnt = align256(kOffList + 4ull * kMaxPoints);
+constexpr size_t kOffSlot = align256(kOffCellOf + 4ull * kPad);
+constexpr size_t kOffList = align256(kOffSlot + 4ull * kPad);
+constexpr size_t kOffTouched = align256(kOffList + 4ull * kMaxPoints);
+constexpr size_t kOffBucket = align256(kOffTouched + 4ull * kMaxPoints);
+constexpr size_t kOffCnt = align256(kOffBucket + 16ull * kMaxPillars * kMaxPts);
 constexpr size_t kOffFirst = align256(kOffCnt + 4ull * kMaxCells);
-constexpr size_t kOffC2P = align256(kOffFirst + 4ull * kMaxCells);
-constexpr size_t kOffBlock = align256(kOffC2P + 4ull * kMaxCells);
-constexpr size_t kOffItems = align256(kOffBlock + 8ull * kMaxScanBlocks);
-constexpr size_t kOffRaw = align256(kOffItems + 8ull * kMaxScanBlocks * kScanTile);
-constexpr size_t kOffPoff = align256(kOffRaw + 4ull * kMaxPillars);
-constexpr size_t kOffCursor = align256(kOffPoff + 4ull * kMaxPillars);
-constexpr size_t kOffNp = align256(kOffCursor + 4ull * kMaxPillars);
-constexpr size_t kStaticBytes = align256(kOffNp + 16);
+constexpr size_t kOffLoc = align256(kOffFirst + 4ull * kMaxCells);
+constexpr size_t kOffAgg = align256(kOffLoc + 8ull * kMaxCells);
+constexpr size_t kOffPrec = align256(kOffAgg + 8ull * kMaxTiles * kAggStride);
+constexpr size_t kOffNp = align256(kOffPrec + 16ull * kMaxPillars);
+constexpr size_t kOffNt = align256(kOffNp + 16);
+constexpr size_t kStaticBytes = align256(kOffNt + 16);
 
 static __device__ __align__(256) unsigned char g_pillar_scratch[kStaticBytes];
 
@@ -98,10 +100,13 @@ extern "C" rtcc_status rtcc_pillarise_noalloc(const rtcc_model_config* cfg, cons
   if (cfg->grid_w < 1 || cfg->grid_h < 1 || cells > kMaxCells) return RTCC_E_ARG;
   if (n_points < 0 || n_points > kMaxPoints) return RTCC_E_ARG;
   if (cfg->max_pillars < 1 || cfg->max_pillars > kMaxPillars) return RTCC_E_ARG;
-  if (cfg->max_pts < 1 || cfg->max_pts > 32) return RTCC_E_ARG;
+  if (cfg->max_pts < 1 || cfg->max_pts > kMaxPts) return RTCC_E_ARG;
   if (cfg->pfn_ch != 32 && cfg->pfn_ch != kMaxCh) return RTCC_E_ARG;
   if (cfg->dtype != RTCC_FP16 && cfg->dtype != RTCC_BF16) return RTCC_E_ARG;
   if (!(cfg->pillar > 0.f)) return RTCC_E_ARG;
+  if (!grid_coords_ok(cfg->x_min, cfg->y_min, cfg->z_min, cfg->z_max, cfg->pillar, cfg->grid_w,
+                      cfg->grid_h))
+    return RTCC_E_ARG;
   // The kernels read the points as float4 and clear the image with 16-byte
   // stores; a sub-view that is not so aligned is refused here instead of
   // faulting on the device.
@@ -119,22 +124,25 @@ extern "C" rtcc_status rtcc_pillarise_noalloc(const rtcc_model_config* cfg, cons
   b.pts = reinterpret_cast<const float4*>(d_points);
   b.n_hdr = reinterpret_cast<const int*>(base + kOffN);
   b.cell_of = reinterpret_cast<int*>(base + kOffCellOf);
+  b.slot_of = reinterpret_cast<int*>(base + kOffSlot);
   b.cnt_cell = reinterpret_cast<int*>(base + kOffCnt);
   b.first_cell = reinterpret_cast<int*>(base + kOffFirst);
-  b.c2p = reinterpret_cast<int*>(base + kOffC2P);
-  b.blocksum = reinterpret_cast<int2*>(base + kOffBlock);
-  b.items = reinterpret_cast<int2*>(base + kOffItems);
-  b.pcnt_raw = reinterpret_cast<int*>(base + kOffRaw);
-  b.poff = reinterpret_cast<int*>(base + kOffPoff);
-  b.cursor = reinterpret_cast<int*>(base + kOffCursor);
+  b.cell_loc = reinterpret_cast<int2*>(base + kOffLoc);
+  b.tile_agg = reinterpret_cast<unsigned long long*>(base + kOffAgg);
+  b.pillar_rec = reinterpret_cast<int4*>(base + kOffPrec);
+  b.touched = reinterpret_cast<int*>(base + kOffTouched);
+  b.ntouched = reinterpret_cast<int*>(base + kOffNt);
   b.list = reinterpret_cast<int*>(base + kOffList);
+  b.bucket = reinterpret_cast<float4*>(base + kOffBucket);
   b.np_prev = reinterpret_cast<int*>(base + kOffNp);
   b.pillar_cell = d_pillar_cell;
   b.pcount = d_count;
   b.stats = d_stats;
+  b.zero_words = d_stats;                       // the first kernel clears the stats
+  b.n_zero = 8;
   b.cell2pillar = d_cell2pillar;
   b.image = d_image;
-  b.cap = n_points > 0 ? n_points : 1;
+  b.cap = n_points;
   b.P = cfg->max_pillars;
   b.N = cfg->max_pts;
   b.C = cfg->pfn_ch;
@@ -153,7 +161,7 @@ extern "C" rtcc_status rtcc_pillarise_noalloc(const rtcc_model_config* cfg, cons
     return RTCC_E_CUDA;
   GridGeom g{cfg->x_min, cfg->y_min, cfg->z_min, cfg->z_max, cfg->pillar, cfg->grid_w,
              cfg->grid_h};
-  if (launch_pillarise(b, g, d_pfn_w, d_pfn_b, cfg->dtype == RTCC_BF16, nullptr, st) !=
+  if (launch_pillarise(b, g, d_pfn_w, d_pfn_b, cfg->dtype == RTCC_BF16, st) !=
       cudaSuccess)
     return RTCC_E_CUDA;
   return RTCC_OK;
