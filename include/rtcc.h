@@ -208,7 +208,12 @@ typedef struct {
  * the K branch graphs plus the post-join graph, and (unless
  * RTCC_FLAG_NO_BATCH) starts one host thread, the dispatcher of batched
  * backbone launches (see rtcc_payload_complete), which rtcc_destroy joins.
- * RTCC_E_ARG for an unsupported config or a blob of the wrong length.
+ * RTCC_E_ARG for an unsupported config or a blob of the wrong length.  A
+ * grid whose x or y bounds (x_min, x_min + grid_w * pillar, and the same in
+ * y) lie more than 2^20 pillar edges from 0, or whose z bounds lie more than
+ * 2^20 times (z_max - z_min) from 0, is unsupported: the PFN forms the means
+ * as fixed-point sums of the points' offsets from their pillar, which needs
+ * float32 to place each point within one edge of its pillar's centre.
  */
 rtcc_status rtcc_init(const rtcc_model_config* cfg, const float* weights,
                       size_t n_floats, struct rtcc_ctx** out);
@@ -377,9 +382,10 @@ rtcc_status rtcc_get_tensor(struct rtcc_ctx* ctx, int32_t agent, int32_t which,
  * loops that must not risk the device synchronisation an allocation can
  * trigger.  This call allocates nothing: its scratch is one fixed array in
  * device memory that the library reserves on every GPU that loads it (about
- * 3.1 MB, kept until the process exits).  The array bounds the sizes:
+ * 11.8 MB, kept until the process exits).  The array bounds the sizes:
  * grid_w * grid_h <= 65536 cells, n_points <= 131072, max_pillars <= 16384,
- * pfn_ch in {32, 64}, max_pts <= 32; larger requests return RTCC_E_ARG.
+ * pfn_ch in {32, 64}, max_pts <= 32; larger requests, and grid bounds that
+ * rtcc_init rejects, return RTCC_E_ARG.
  *
  * Uses from cfg: grid_w/h, x_min, y_min, z_min, z_max, pillar, max_pillars,
  * max_pts, pfn_ch, dtype.  Inputs (device, caller-owned): d_points float32

@@ -59,6 +59,33 @@ def test_init_rejects_bad_config_without_touching_gpu(R):
     assert R.load().rtcc_init(None, w, 4, ctypes.byref(out)) == R.E_ARG
 
 
+def test_init_rejects_grid_bounds_far_from_origin(R):
+    # the PFN's fixed-point means need every grid bound within 2^20 pillar
+    # edges of 0 (z: within 2^20 z-ranges); 0.4 m pillars allow 419,430 m
+    import synth
+    tiny = synth.get_config("tiny")
+    blob = synth.weight_blob(synth.weights_for(tiny))
+    wp = blob.ctypes.data_as(ctypes.POINTER(ctypes.c_float))
+    lib = R.load()
+    out = ctypes.c_void_p()
+    # the blob has the right length: the plain config gets past validation
+    # (no GPU here: it fails later, or builds a context where there is one)
+    s = lib.rtcc_init(ctypes.byref(R.model_config(tiny)), wp, blob.size, ctypes.byref(out))
+    assert s != R.E_ARG
+    if s == R.OK:
+        lib.rtcc_destroy(out)
+    for field, value in (("x_min", 5.0e5), ("y_min", -4.3e5), ("z_min", 1.0e7)):
+        cfg = R.model_config(tiny)
+        setattr(cfg, field, value)
+        if field == "x_min":
+            cfg.x_max = value + cfg.grid_w * cfg.pillar
+        if field == "y_min":
+            cfg.y_max = value + cfg.grid_h * cfg.pillar
+        if field == "z_min":                      # a 4 m range 10,000 km up
+            cfg.z_max = value + 4.0
+        assert lib.rtcc_init(ctypes.byref(cfg), wp, blob.size, ctypes.byref(out)) == R.E_ARG, field
+
+
 def test_nms_arguments_are_checked_before_any_gpu_work(R):
     import numpy as np
     import synth
