@@ -869,6 +869,10 @@ rtcc_status capture_post(rtcc_ctx* c) {
       CK(tmap_2d(&tp.feat[k], c->ms ? c->neck_out : (attn1 ? c->fused : c->br[k].feat), c->bf16,
                  (uint64_t)c->Cf,
                  (uint64_t)fa.cells, (uint32_t)bkc, 128u, swz));
+    // the K slots are consecutive in feat_all (K_head = 1: the one fused map)
+    CK(tmap_3d(&tp.feat_all, c->ms ? c->neck_out : (attn1 ? c->fused : c->feat_all), c->bf16,
+               (uint64_t)c->Cf, (uint64_t)fa.cells, (uint64_t)K_head, (uint32_t)bkc, 128u,
+               (uint32_t)K_head, swz));
     CK(tmap_2d(&tp.wmap, c->head_w16, c->bf16, (uint64_t)c->Cf, 16u, (uint32_t)bkc, 16u, swz));
     tp.present = two_step ? c->d_one : c->d_present;
     tp.K = K_head;

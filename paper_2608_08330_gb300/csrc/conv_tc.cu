@@ -1043,6 +1043,26 @@ cudaError_t tmap_2d(CUtensorMap* m, const void* base, bool bf16, uint64_t inner,
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
+cudaError_t tmap_3d(CUtensorMap* m, const void* base, bool bf16, uint64_t inner, uint64_t mid,
+                    uint64_t outer, uint32_t box_inner, uint32_t box_mid, uint32_t box_outer,
+                    int swizzle_bytes) {
+  EncodeFn enc = encode_fn();
+  if (!enc) return cudaErrorNotSupported;
+  const CUtensorMapDataType dt =
+      bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT16;
+  const CUtensorMapSwizzle sw = swizzle_bytes == 128  ? CU_TENSOR_MAP_SWIZZLE_128B
+                                : swizzle_bytes == 64 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                                      : CU_TENSOR_MAP_SWIZZLE_NONE;
+  cuuint64_t dims[3] = {inner, mid, outer};
+  cuuint64_t strides[2] = {inner * 2, inner * mid * 2};
+  cuuint32_t box[3] = {box_inner, box_mid, box_outer};
+  cuuint32_t es[3] = {1, 1, 1};
+  const CUresult r = enc(m, dt, 3, const_cast<void*>(base), dims, strides, box, es,
+                         CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
 int conv_tile_w() { return TW; }
 int conv_tile_h() { return TH; }
 int conv_tile_m() { return BM; }

@@ -7,8 +7,10 @@
 //
 // The head is a GEMM with M = cells, N = 16, K = C.  One work item is a tile
 // of 128 consecutive cells.  For each 64- (or 32-) channel chunk of the tile,
-// TMA loads the chunk of every present agent's slot into one pipeline stage,
-// all with the same 128-byte (64-byte) swizzle; because the max is taken
+// TMA loads the chunk of every present agent's slot into one pipeline stage
+// (one 3-D box over all K consecutive slots when every agent is present, one
+// box per present agent otherwise), all with the same 128-byte (64-byte)
+// swizzle; because the max is taken
 // position by position, the max of the swizzled agent tiles is the swizzled
 // fused tile, i.e. directly the A operand of tcgen05.mma.  B is the head
 // weight matrix [16][C] (K-major, loaded once per CTA).  The accumulator is 16
@@ -36,11 +38,15 @@ constexpr int kThreads = 320;
 constexpr int kWorkers = kThreads - 64;        // warps 2..9 take the max; warps 2..5 the epilogue
 constexpr int kTile = 128;                     // cells per work item (MMA M)
 constexpr int kMaxStages = 8;
-constexpr int kStageArea = 176 * 1024;         // agent-chunk stages
 constexpr int kMaxC = 512;
-constexpr int kFBytes = kTile * 64 * 2;        // one fused chunk (bkc <= 64)
+// The agent-chunk stages and the two fused chunks (the MMA's A operand, 128
+// rows of bkc channels each) share one area, so 32-channel chunks leave room
+// for more stages.
+constexpr int kArea = 208 * 1024;
+__host__ __device__ constexpr int fused_bytes(int bkc) { return kTile * bkc * 2; }
+__host__ __device__ constexpr int stage_area(int bkc) { return kArea - 2 * fused_bytes(bkc); }
 constexpr int kWBytes = kFuseHeadOut * kMaxC * 2;
-constexpr int kSmem = kStageArea + 2 * kFBytes + kWBytes + 1024 + 256;
+constexpr int kSmem = kArea + kWBytes + 1024 + 256;
 static_assert(kSmem <= 227 * 1024, "shared memory budget");
 
 template <typename T>
@@ -117,8 +123,9 @@ __global__ void __launch_bounds__(kThreads, 1) k_fuse_max_head(const __grid_cons
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint8_t* fbuf = smem + kStageArea;           // [2] fused chunks (the MMA's A operand)
-  uint8_t* wsm = fbuf + 2 * kFBytes;           // head weights [C / bkc][16][bkc]
+  const int fbytes = fused_bytes(P.bkc);
+  uint8_t* fbuf = smem + stage_area(P.bkc);    // [2] fused chunks (the MMA's A operand)
+  uint8_t* wsm = smem + kArea;                 // head weights [C / bkc][16][bkc]
   uint64_t* full = reinterpret_cast<uint64_t*>(wsm + kWBytes);   // [kMaxStages] agent chunks landed
   uint64_t* empty = full + kMaxStages;         // [kMaxStages] workers have read the stage
   uint64_t* fready = empty + kMaxStages;       // [2] fused chunk written
@@ -183,7 +190,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_fuse_max_head(const __grid_cons
   if (warp == 0) {
     if (lane == 0) {
       // ---------------- TMA producer: agent chunks -> stages ----------------
-      for (int k = 0; k < Kp; ++k) tma_prefetch_desc(&P.feat[s_list[k]]);
+      if (Kp == P.K)
+        tma_prefetch_desc(&P.feat_all);
+      else
+        for (int k = 0; k < Kp; ++k) tma_prefetch_desc(&P.feat[s_list[k]]);
       uint32_t it = 0;
       bool alive = true;
       for (int t = blockIdx.x; t < tiles && alive; t += gridDim.x) {
@@ -195,9 +205,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_fuse_max_head(const __grid_cons
             break;
           }
           mbar_arrive_expect_tx(&full[s], (uint32_t)(Kp * slot_bytes));
-          for (int i = 0; i < Kp; ++i)
-            tma_load_2d(smem + s * stage_bytes + i * slot_bytes, &P.feat[s_list[i]], &full[s],
-                        j * bkc, t * kTile);
+          if (Kp == P.K) {
+            // every slot present: one box of all K agents' chunks (a thread's
+            // boxes complete one after another, whatever their size)
+            tma_load_3d(smem + s * stage_bytes, &P.feat_all, &full[s], j * bkc, t * kTile, 0);
+          } else {
+            for (int i = 0; i < Kp; ++i)
+              tma_load_2d(smem + s * stage_bytes + i * slot_bytes, &P.feat[s_list[i]], &full[s],
+                          j * bkc, t * kTile);
+          }
         }
       }
     }
@@ -227,7 +243,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fuse_max_head(const __grid_cons
             break;
           }
           tc_fence_after();
-          const uint64_t ad = smem_desc(f0 + b * kFBytes, sbo, swz);
+          const uint64_t ad = smem_desc(f0 + b * fbytes, sbo, swz);
           const uint64_t bd = smem_desc(w0 + j * kFuseHeadOut * bkc * 2, sbo, swz);
           for (int kk = 0; kk < bkc / 16; ++kk)      // K advance: 32 bytes = +2
             umma_f16(d_tmem, ad + 2 * kk, bd + 2 * kk, idesc, (j > 0 || kk > 0) ? 1u : 0u);
@@ -263,7 +279,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fuse_max_head(const __grid_cons
           alive = false;
         }
         const uint4* st = reinterpret_cast<const uint4*>(smem + s * stage_bytes);
-        uint4* fb = reinterpret_cast<uint4*>(fbuf + b * kFBytes);
+        uint4* fb = reinterpret_cast<uint4*>(fbuf + b * fbytes);
         max_chunk_any<T>(st, fb, nvec, wt, Kp);
         if (fused) {
           // debug copy of the fused features, unswizzled to [cell][C]
@@ -328,14 +344,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_fuse_max_head(const __grid_cons
 int fuse_tc_chunk(int C, int K) {
   if (C % 32 != 0 || C > kMaxC || K < 1 || K > RTCC_MAX_AGENTS) return 0;
   // 64-channel chunks while at least 3 stages of K agent chunks fit, else 32
-  if (C % 64 == 0 && 3 * K * kTile * 64 * 2 <= kStageArea) return 64;
-  return 2 * K * kTile * 32 * 2 <= kStageArea ? 32 : 0;
+  if (C % 64 == 0 && 3 * K * kTile * 64 * 2 <= stage_area(64)) return 64;
+  return 2 * K * kTile * 32 * 2 <= stage_area(32) ? 32 : 0;
 }
 
 int fuse_tc_stages(int C, int K) {
   const int bkc = fuse_tc_chunk(C, K);
   if (bkc == 0) return 0;
-  const int n = kStageArea / (K * kTile * bkc * 2);
+  const int n = stage_area(bkc) / (K * kTile * bkc * 2);
   return n < kMaxStages ? n : kMaxStages;
 }
 

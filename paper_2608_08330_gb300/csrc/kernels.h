@@ -268,6 +268,7 @@ cudaError_t launch_fuse_blocks(FuseBlocksArgs a, bool bf16, cudaStream_t st);
 constexpr int kFuseHeadOut = 16;
 struct FuseTcParams {
   CUtensorMap feat[RTCC_MAX_AGENTS];  // agent k's slot [cells][C], box (bkc, 128), swizzled
+  CUtensorMap feat_all;               // the K slots as one [K][cells][C] tensor, box (bkc, 128, K)
   CUtensorMap wmap;                   // head weights [16][C] in the storage type, box (bkc, 16)
   const int* present;                 // device [K]
   int K, C, cells, bkc, stages;
@@ -292,6 +293,10 @@ cudaError_t launch_fuse_max_head(const FuseTcParams& p, bool bf16, cudaStream_t 
 // bytes); OOB elements read as zero.
 cudaError_t tmap_2d(CUtensorMap* m, const void* base, bool bf16, uint64_t inner, uint64_t outer,
                     uint32_t box_inner, uint32_t box_outer, int swizzle_bytes);
+// The same for a 3-D tensor [outer][mid][inner], dense.
+cudaError_t tmap_3d(CUtensorMap* m, const void* base, bool bf16, uint64_t inner, uint64_t mid,
+                    uint64_t outer, uint32_t box_inner, uint32_t box_mid, uint32_t box_outer,
+                    int swizzle_bytes);
 // Head weight permutation expected by the fusion kernel (host side).
 void permute_head_weights(const float* w /*[16][C]*/, int C, float* out /*[16*C]*/);
 
