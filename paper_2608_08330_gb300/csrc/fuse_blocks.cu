@@ -18,8 +18,9 @@
 //               equals the max over the present agents)
 //   attention:  s_k = <X_0, X_k> / sqrt(C_b), w = softmax over present k,
 //               F = sum_k w_k X_k   (fp32; the dot product is each thread's
-//               8 fused multiply-adds, then a butterfly over the cell's
-//               threads, so every thread holds the same s_k)
+//               fused multiply-adds, then a butterfly over the cell's
+//               threads, so every thread holds the same s_k; the softmax is
+//               taken online in one pass over the agents)
 // Every reduction has a fixed order: the result is bit-reproducible.
 #include <cmath>
 
@@ -69,79 +70,80 @@ __device__ __forceinline__ void fuse_vec(const T* src, long long astride, const 
       }
     }
   } else {
-    // two passes over the agents (scores, then the weighted sum, reloading
-    // each vector -- an L1 hit) keep one agent's vector live at a time
+    // one pass over the present agents in index order, softmax online: a
+    // running maximum m of the scores, the denominator and the weighted sum
+    // rescaled by exp(m_old - m_new) when m grows (the ego agent 0, always
+    // present, starts them).  The ego vector stays packed (16-bit pairs) for
+    // the dot products, so each agent's vector is read once and few
+    // registers stay live.
     constexpr int E = 8 * NV;
-    float x0[E];
+    uint32_t q[4 * NV];
 #pragma unroll
     for (int v = 0; v < NV; ++v) {
-      const uint4 r = ld16(src + off + 8 * v);            // the ego agent 0 is present
-      const uint32_t w[4] = {r.x, r.y, r.z, r.w};
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const float2 f = Store<T>::unpack2(w[i]);
-        x0[8 * v + 2 * i] = f.x;
-        x0[8 * v + 2 * i + 1] = f.y;
-      }
+      const uint4 r = ld16(src + off + 8 * v);
+      q[4 * v] = r.x;
+      q[4 * v + 1] = r.y;
+      q[4 * v + 2] = r.z;
+      q[4 * v + 3] = r.w;
     }
-    float s[RTCC_MAX_AGENTS];
-    float mx = -INFINITY;
+    float F[E], m = 0.f, den = 0.f;
 #pragma unroll
     for (int k = 0; k < RTCC_MAX_AGENTS; ++k) {
-      s[k] = -INFINITY;
       if (k < K && ((pres >> k) & 1u)) {
+        uint32_t x[4 * NV];
+        if (k == 0) {
+#pragma unroll
+          for (int i = 0; i < 4 * NV; ++i) x[i] = q[i];
+        } else {
+#pragma unroll
+          for (int v = 0; v < NV; ++v) {
+            const uint4 r = ld16(src + (size_t)k * astride + off + 8 * v);
+            x[4 * v] = r.x;
+            x[4 * v + 1] = r.y;
+            x[4 * v + 2] = r.z;
+            x[4 * v + 3] = r.w;
+          }
+        }
         float d = 0.f;
 #pragma unroll
-        for (int v = 0; v < NV; ++v) {
-          const uint4 r = ld16(src + (size_t)k * astride + off + 8 * v);
-          const uint32_t w[4] = {r.x, r.y, r.z, r.w};
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            const float2 f = Store<T>::unpack2(w[i]);
-            d = fmaf(x0[8 * v + 2 * i], f.x, d);
-            d = fmaf(x0[8 * v + 2 * i + 1], f.y, d);
-          }
+        for (int i = 0; i < 4 * NV; ++i) {
+          const float2 a = Store<T>::unpack2(q[i]), b = Store<T>::unpack2(x[i]);
+          d = fmaf(a.x, b.x, d);
+          d = fmaf(a.y, b.y, d);
         }
 #pragma unroll
         for (int o = G / 2; o > 0; o >>= 1) d += __shfl_xor_sync(kFull, d, o);
-        s[k] = d * inv_sqrt_c;
-        mx = fmaxf(mx, s[k]);
-      }
-    }
-    float den = 0.f;
+        const float sk = d * inv_sqrt_c;
+        if (k == 0) {
+          m = sk;
+          den = 1.f;
 #pragma unroll
-    for (int k = 0; k < RTCC_MAX_AGENTS; ++k) {
-      if (k < K && ((pres >> k) & 1u)) {
-        s[k] = expf(s[k] - mx);
-        den += s[k];
-      }
-    }
-    float F[E];
+          for (int i = 0; i < 4 * NV; ++i) {
+            const float2 b = Store<T>::unpack2(x[i]);
+            F[2 * i] = b.x;
+            F[2 * i + 1] = b.y;
+          }
+        } else {
+          const float mn = fmaxf(m, sk);
+          const float sc = expf(m - mn), wk = expf(sk - mn);
+          m = mn;
+          den = fmaf(den, sc, wk);
 #pragma unroll
-    for (int j = 0; j < E; ++j) F[j] = 0.f;
-#pragma unroll
-    for (int k = 0; k < RTCC_MAX_AGENTS; ++k) {
-      if (k < K && ((pres >> k) & 1u)) {
-        const float wk = s[k] / den;
-#pragma unroll
-        for (int v = 0; v < NV; ++v) {
-          const uint4 r = ld16(src + (size_t)k * astride + off + 8 * v);
-          const uint32_t w[4] = {r.x, r.y, r.z, r.w};
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            const float2 f = Store<T>::unpack2(w[i]);
-            F[8 * v + 2 * i] = fmaf(wk, f.x, F[8 * v + 2 * i]);
-            F[8 * v + 2 * i + 1] = fmaf(wk, f.y, F[8 * v + 2 * i + 1]);
+          for (int i = 0; i < 4 * NV; ++i) {
+            const float2 b = Store<T>::unpack2(x[i]);
+            F[2 * i] = fmaf(F[2 * i], sc, wk * b.x);
+            F[2 * i + 1] = fmaf(F[2 * i + 1], sc, wk * b.y);
           }
         }
       }
     }
+    const float inv = 1.f / den;
 #pragma unroll
     for (int v = 0; v < NV; ++v) {
-      out[v].x = Store<T>::pack2(F[8 * v + 0], F[8 * v + 1]);
-      out[v].y = Store<T>::pack2(F[8 * v + 2], F[8 * v + 3]);
-      out[v].z = Store<T>::pack2(F[8 * v + 4], F[8 * v + 5]);
-      out[v].w = Store<T>::pack2(F[8 * v + 6], F[8 * v + 7]);
+      out[v].x = Store<T>::pack2(F[8 * v + 0] * inv, F[8 * v + 1] * inv);
+      out[v].y = Store<T>::pack2(F[8 * v + 2] * inv, F[8 * v + 3] * inv);
+      out[v].z = Store<T>::pack2(F[8 * v + 4] * inv, F[8 * v + 5] * inv);
+      out[v].w = Store<T>::pack2(F[8 * v + 6] * inv, F[8 * v + 7] * inv);
     }
   }
 }
@@ -169,7 +171,7 @@ static_assert(RTCC_MAX_BLOCKS == 3, "the task numbering below covers three block
 // WIDE: one 384-channel map (the single-scale 384-channel slots; 16 threads of
 // 24 channels per cell); otherwise block maps of 32 to 256 channels.
 template <typename T, bool ATTN, bool WIDE>
-__global__ void __launch_bounds__(kThreads, WIDE ? 2 : 3) k_fuse_blocks(const __grid_constant__ FuseBlocksArgs a) {
+__global__ void __launch_bounds__(kThreads, 3) k_fuse_blocks(const __grid_constant__ FuseBlocksArgs a) {
   pdl_trigger();
   pdl_wait();
   span_begin(a.span);
