@@ -146,10 +146,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_fuse_max_head(const __grid_cons
   const int nst = P.stages;
   const int tiles = (P.cells + kTile - 1) / kTile;
 
+  // One agent and no debug copy: the max is the staged chunk itself, so the
+  // MMA reads the stage directly and its commit releases the stage.
+  const bool direct = P.K == 1 && P.fused == nullptr;
   if (warp == 0 && lane == 0) {
     for (int s = 0; s < nst; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], kWorkers);
+      mbar_init(&empty[s], direct ? 1 : kWorkers);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&fready[b], kWorkers);
@@ -236,18 +239,19 @@ __global__ void __launch_bounds__(kThreads, 1) k_fuse_max_head(const __grid_cons
         tc_fence_after();
         const uint32_t d_tmem = tmem + acc * kFuseHeadOut;
         for (int j = 0; j < nch; ++j, ++it) {
-          const int b = it & 1;
-          if (!mbar_wait(&fready[b], (it >> 1) & 1)) {
+          const int b = it & 1, s = it % nst;
+          if (direct ? !mbar_wait(&full[s], (it / nst) & 1) : !mbar_wait(&fready[b], (it >> 1) & 1)) {
             atomicOr(P.err, ERR_WAIT_FUSE);
             alive = false;
             break;
           }
           tc_fence_after();
-          const uint64_t ad = smem_desc(f0 + b * fbytes, sbo, swz);
+          const uint64_t ad = direct ? smem_desc(smem_u32(smem) + s * stage_bytes, sbo, swz)
+                                     : smem_desc(f0 + b * fbytes, sbo, swz);
           const uint64_t bd = smem_desc(w0 + j * kFuseHeadOut * bkc * 2, sbo, swz);
           for (int kk = 0; kk < bkc / 16; ++kk)      // K advance: 32 bytes = +2
             umma_f16(d_tmem, ad + 2 * kk, bd + 2 * kk, idesc, (j > 0 || kk > 0) ? 1u : 0u);
-          umma_commit(&fempty[b]);
+          umma_commit(direct ? &empty[s] : &fempty[b]);
         }
         umma_commit(&accfull[acc]);
       }
@@ -267,7 +271,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_fuse_max_head(const __grid_cons
     uint32_t it = 0, tc = 0;
     bool alive = true;
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++tc) {
-      for (int j = 0; j < nch; ++j, ++it) {
+      for (int j = 0; j < nch && !direct; ++j, ++it) {
         const int s = it % nst, b = it & 1;
         if (alive && !mbar_wait(&full[s], (it / nst) & 1)) {
           atomicOr(P.err, ERR_WAIT_FUSE);
