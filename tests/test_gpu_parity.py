@@ -174,6 +174,29 @@ def test_caps_bind_bit_exact(R):
     R.rtcc_destroy(ctx)
 
 
+def test_large_payload_scan_takes_several_tiles_per_block(R):
+    # 1.6 million points per branch: the pillar scan runs 4,096-point tiles,
+    # more tiles than the cooperative grid has blocks, so each block takes
+    # several in order; pillars, drops and every later stage as in any frame
+    cfg = dataclasses.replace(synth.get_config("tiny"), max_pillars=2048, max_pts=16)
+    rng = np.random.default_rng(5)
+    pts = []
+    for n in (1_600_000, 700_001):
+        p = np.zeros((n, 4), dtype=np.float32)
+        p[:, 0] = rng.uniform(-14.0, 14.0, n)
+        p[:, 1] = rng.uniform(-14.0, 14.0, n)
+        p[:, 2] = rng.uniform(-3.2, 1.2, n)
+        p[:, 3] = rng.uniform(0.0, 1.0, n)
+        pts.append(p)
+    ctx, w = U.make_ctx(cfg, max_points=1_600_000)
+    try:
+        for fid, mode in ((1, R.MODE_RTCC), (2, R.MODE_BARRIER)):
+            U.run_frame(ctx, cfg, pts, [0.0, 1.0], mode, frame_id=fid)
+            _check_frame(R, ctx, cfg, w, pts)
+    finally:
+        R.rtcc_destroy(ctx)
+
+
 def test_empty_and_out_of_range_payloads(R):
     cfg = synth.get_config("tiny")
     ctx, w = U.make_ctx(cfg)
