@@ -169,9 +169,12 @@ __device__ __forceinline__ void block_task(const FuseBlocksArgs& a, int b, int w
 static_assert(RTCC_MAX_BLOCKS == 3, "the task numbering below covers three blocks");
 
 // WIDE: one 384-channel map (the single-scale 384-channel slots; 16 threads of
-// 24 channels per cell); otherwise block maps of 32 to 256 channels.
+// 24 channels per cell); otherwise block maps of 32 to 256 channels.  The max
+// of the block maps runs 5 blocks per SM (more loads in flight: stress8's
+// three maps 12.8 -> 10.7 us against 3 blocks); attention keeps 3 (80
+// registers).
 template <typename T, bool ATTN, bool WIDE>
-__global__ void __launch_bounds__(kThreads, 3) k_fuse_blocks(const __grid_constant__ FuseBlocksArgs a) {
+__global__ void __launch_bounds__(kThreads, (ATTN || WIDE) ? 3 : 5) k_fuse_blocks(const __grid_constant__ FuseBlocksArgs a) {
   pdl_trigger();
   pdl_wait();
   span_begin(a.span);
