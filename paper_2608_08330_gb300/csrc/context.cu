@@ -125,6 +125,7 @@ struct rtcc_ctx {
   int launch_size[RTCC_MAX_AGENTS] = {};
   int launch_word[RTCC_MAX_AGENTS] = {};
   std::vector<int> pending;           // released agents whose backbone waits for a batch
+  std::atomic<double> t_hold{0.0};    // host time of the last release that left a batch open
   std::thread disp;                   // dispatcher of deferred batches
   std::condition_variable cv;
   bool stop = false;
@@ -1247,25 +1248,33 @@ rtcc_status launch_post(rtcc_ctx* c) {
 // Dispatch what an event made ready; launch the post-join once every branch
 // is resolved.  `t_entry` is the host time the event call began.
 //
-// Batching (unless RTCC_FLAG_NO_BATCH): a branch released while the GPU is
-// free starts at once with its own backbone; one released while a backbone
-// is still running enqueues only its pillar chain and waits in `pending`.
-// When the running backbone ends, the dispatcher thread launches one backbone
-// over every pending agent.  Agents released by one event (Barrier's release
-// of all branches at A) form one batch.  Once the last branch is resolved no
-// later release can join a batch, so whatever is pending is launched at once,
-// queued behind the running backbone, followed by the post-join.
+// Batching (unless RTCC_FLAG_NO_BATCH): a release that does not resolve the
+// last branch enqueues only its pillar chain and waits in `pending`; the
+// dispatcher thread launches one backbone over every pending agent once the
+// backbone in flight (if any) has ended and no release has come for kHoldMs.
+// Completions reported close together (several agents completing at one
+// instant, reported by one call each) so share one launch, and a lone branch
+// loses only the hold beyond its pillar chain, which the backbone waits for
+// anyway.  Agents released by one event (Barrier's release of all branches at
+// A) form one batch.  The release that resolves the last branch launches at
+// once: with nothing pending and the GPU free, as its own branch graph;
+// otherwise with whatever is pending, queued behind the running backbone;
+// the post-join follows.
 rtcc_status after_event(rtcc_ctx* c, const std::vector<int>& released, double t_entry) {
   const bool batching = (c->cfg.flags & RTCC_FLAG_NO_BATCH) == 0;
   const bool last = c->ctrl.join_ready();
   if (!batching) {
     for (int k : released) RS(launch_full(c, k));
-  } else if (released.size() == 1 && c->pending.empty() && !backbone_busy(c)) {
+  } else if (released.size() == 1 && last && c->pending.empty() && !backbone_busy(c)) {
     RS(launch_full(c, released[0]));
   } else if (!released.empty()) {
     for (int k : released) RS(launch_pill(c, k));
-    if (released.size() > 1 || last || !backbone_busy(c)) RS(launch_batch(c));
-    else c->cv.notify_all();
+    if (released.size() > 1 || last) {
+      RS(launch_batch(c));
+    } else {
+      c->t_hold.store(now_ms(), std::memory_order_relaxed);
+      c->cv.notify_all();
+    }
   }
   if (last && !c->post_launched) {
     if (!c->pending.empty()) RS(launch_batch(c));
@@ -1275,8 +1284,14 @@ rtcc_status after_event(rtcc_ctx* c, const std::vector<int>& released, double t_
   return RTCC_OK;
 }
 
-// Launches the pending batch once the backbone in flight has ended (see
-// after_event).  Waits for the end on the launch's done word in pinned host
+// Gathering window of a batch: a release leaves its batch open this long for
+// the next one.  It covers the host's gap between completions reported back
+// to back, and stays near the pillar chain's own length (about 20 us), which
+// the backbone waits for in any case.
+constexpr double kHoldMs = 0.04;
+
+// Launches the pending batch once the backbone in flight has ended and the
+// hold has run out (see after_event).  Waits for the end on the launch's done word in pinned host
 // memory, without the context mutex.
 void dispatcher_main(rtcc_ctx* c) {
   cudaSetDevice(c->dev);
@@ -1291,9 +1306,13 @@ void dispatcher_main(rtcc_ctx* c) {
       // a launch that never reports its end (it failed) stops holding the batch back
       if ((it & 1023u) == 0 && now_ms() - t0 > 2000.0) break;
     }
+    while (now_ms() - c->t_hold.load(std::memory_order_relaxed) < kHoldMs) {
+    }
     lk.lock();
     if (c->stop) break;
-    if (!c->pending.empty() && c->inflight == w) {
+    // a release that came in meanwhile reopens the hold (the loop comes back)
+    if (!c->pending.empty() && c->inflight == w &&
+        now_ms() - c->t_hold.load(std::memory_order_relaxed) >= kHoldMs) {
       if (launch_batch(c) != RTCC_OK) c->disp_err = true;
     }
   }

@@ -10,6 +10,7 @@ Stages are also checked in isolation (the oracle's next stage applied to the
 GPU's own input of that stage) so that a kernel is judged on its own error.
 """
 import dataclasses
+import time
 
 import numpy as np
 import pytest
@@ -138,13 +139,56 @@ def test_tiny_end_to_end(R):
     assert info.n_dispatched == 2 and info.gpu_backbone_ms[0] > 0 and info.gpu_fusion_ms > 0
     # the fusion kernel's own global-timer span sits inside its event-node span
     assert 0 < info.gpu_fusion_kernel_ms <= info.gpu_fusion_ms + 1e-3
-    # agent 0 runs as its own branch graph; agent 1, released while agent 0's
-    # backbone runs, may run its backbone as a separate launch (no branch span)
-    assert info.gpu_branch_ms[0] > 0 and all(info.gpu_pfn_kernel_ms[k] > 0 for k in range(2))
+    # completions reported back to back share a backbone launch (or, if the
+    # host was slow, agent 0 ran alone and agent 1 as its own branch graph)
+    assert all(info.gpu_pfn_kernel_ms[k] > 0 for k in range(2))
     assert all(info.gpu_pfn_kernel_ms[k] < info.gpu_branch_ms[k] for k in range(2)
                if info.gpu_branch_ms[k] > 0)
     assert sum(info.backbone_batch[j] for j in range(info.n_backbone_launches)) == 2
     R.rtcc_destroy(ctx)
+
+
+def test_release_hold_gathers_a_burst_and_lets_a_lone_branch_go(R):
+    # A release that does not resolve the last branch leaves its backbone
+    # batch open for a short hold.  Completions reported back to back then
+    # share one backbone launch; a branch released alone gets its own launch
+    # once the hold runs out, and the last branch, released onto a free GPU,
+    # runs as its own branch graph (pillar chain and backbone in one graph).
+    # The outputs are the same bytes either way (Sec. III-C: the schedule
+    # changes when work runs, not what it computes).
+    cfg = synth.get_config("tiny")
+    ctx, _ = U.make_ctx(cfg)
+    try:
+        pts = [synth.points_for(cfg, 0, k) for k in range(cfg.n_agents)]
+        U.run_frame(ctx, cfg, pts, [0.0, 0.0], R.MODE_BARRIER, frame_id=1)
+        ref = R.rtcc_get_head(ctx, cfg.feat_h, cfg.feat_w).tobytes()
+        info = R.rtcc_get_frame_info(ctx)
+        assert list(info.backbone_batch)[:info.n_backbone_launches] == [2]
+        # back to back: one launch (a host stall past the hold splits it, so
+        # the burst gets a few tries)
+        burst = []
+        for f in range(3):
+            U.run_frame(ctx, cfg, pts, [0.0, 0.0], R.MODE_RTCC, frame_id=2 + f)
+            assert R.rtcc_get_head(ctx, cfg.feat_h, cfg.feat_w).tobytes() == ref
+            info = R.rtcc_get_frame_info(ctx)
+            burst.append(list(info.backbone_batch)[:info.n_backbone_launches])
+        assert [2] in burst, burst
+        # 20 ms apart: agent 0's backbone runs alone after the hold and has
+        # ended when agent 1 arrives
+        assert R.rtcc_frame_begin(ctx, 9, 0.0) == R.OK
+        assert R.rtcc_payload_complete(ctx, 0, pts[0], 0.0) == R.OK
+        time.sleep(0.02)
+        assert R.rtcc_payload_complete(ctx, 1, pts[1], 20.0) == R.OK
+        s, _, _ = R.rtcc_wait_detection(ctx, 60000)
+        assert s == R.OK, R.rtcc_status_str(s)
+        assert R.rtcc_get_head(ctx, cfg.feat_h, cfg.feat_w).tobytes() == ref
+        info = R.rtcc_get_frame_info(ctx)
+        assert list(info.backbone_batch)[:info.n_backbone_launches] == [1, 1]
+        assert list(info.dispatch_order)[:2] == [0, 1]
+        assert info.gpu_branch_ms[0] < 0 < info.gpu_branch_ms[1]
+        assert info.gpu_backbone_ms[0] > 0 and info.gpu_backbone_ms[1] > 0
+    finally:
+        R.rtcc_destroy(ctx)
 
 
 def test_pointpillars_small_grid_ragged_tiles(R):
