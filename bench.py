@@ -54,7 +54,7 @@ METRIC = "complete-detection latency p50/p99 ms RTCC vs barrier; conv TFLOP/s, f
 # dram__bytes_read.sum + dram__bytes_write.sum per k_backbone launch from an
 # ncu capture of this build, keyed by the launch's agent count; None until
 # captured (and again once the kernel changes)
-BACKBONE_TRAFFIC = {8: 540_403_456, 1: 27_808_000}   # profiles/backbone_stress8.md
+BACKBONE_TRAFFIC = {8: 542_687_232, 1: 28_923_392}   # profiles/backbone_stress8.md
 WORKLOAD = "stress8"
 DATA = ("synthetic: seeded uniform + Gaussian-cluster point clouds, He-normal fp32 weights "
         "rounded to fp16, seeded arrival traces (OPV2V and the trained OpenCOOD model are not "

@@ -399,39 +399,49 @@ constexpr size_t kFrameZeroBytes = 8 * sizeof(int) + (kMaxLayers + 1) * sizeof(u
 // fixed (they decide the fp32 summation order, so they are the same for every
 // batch size and a branch's result does not depend on the launch that ran
 // it; the N tile only decides which channels an item computes, and the tile
-// height which pixels).  Cost model: rounds of items over the grid times
+// shape which pixels).  Cost model: rounds of items over the grid times
 // k-blocks per item times a k-block's MMA time at that N tile (measured:
 // 45, 48 and 64 clocks per K = 16 MMA at N = 32, 64, 128); a tall tile
 // (halo layers without split-K: two 128-row MMAs on every weight box) costs
 // kTallCost short k-blocks per k-block -- more than one because it does
 // twice the MMAs, less than two because it halves the weight boxes per FLOP,
-// which bound a short k-block once every CTA has several items.  Ties go to
-// the narrower tile, then to the short one (more, shorter items).
+// which bound a short k-block once every CTA has several items.  The tile
+// may also be laid the other way round (a halo layer's tiles transposed, a
+// tap-box layer's 16 x 8 instead of 8 x 16): the same work per item, but a
+// different item count where the image's sides are not multiples of the
+// tile's (352 x 100 in 8 x 16 tiles: 308 items, 3 rounds on 152 CTAs;
+// transposed, 286).  Ties go to the short, then the narrower tile, then the
+// first orientation.
 constexpr double kTallCost = 1.6;
 double kblock_cost(int bn) { return bn >= 128 ? 1.0 : bn >= 64 ? 0.75 : 0.70; }
-void pick_tile_batch(const ConvLayer& L0, int sp, int grid, int batch, bool need64, int* bn_out,
-                     int* tall_out) {
+void pick_tile_batch(const ConvLayer L0, int sp, int grid, int batch, bool need64, ConvLayer* out) {
   double best = 1e30;
-  *bn_out = std::min(L0.cout, 64);
-  *tall_out = 0;
+  out->bn = std::min(L0.cout, 64);
+  out->tall = out->tr = out->wide = 0;
   const int total_kb = 9 * (L0.cin / L0.bk);
   for (int tall = 0; tall <= 1; ++tall) {
-    ConvLayer L = L0;
-    L.tall = tall;
-    L.splits = sp;
-    if (tall && (sp != 1 || !conv_uses_halo(L))) continue;
-    const int m_tiles = conv_m_tiles(L);
     for (int bn : {32, 64, 128}) {
-      if (bn > L.cout || L.cout % bn) continue;
+      if (bn > L0.cout || L0.cout % bn) continue;
       if (need64 && bn != 64) continue;
-      const int items = batch * m_tiles * (L.cout / bn) * sp;
-      const int rounds = (items + grid - 1) / grid;
-      const double cost =
-          rounds * (double)((total_kb + sp - 1) / sp) * kblock_cost(bn) * (tall ? kTallCost : 1.0);
-      if (cost < best - 1e-9) {
-        best = cost;
-        *bn_out = bn;
-        *tall_out = tall;
+      for (int orient = 0; orient <= 1; ++orient) {
+        ConvLayer L = L0;
+        L.splits = sp;
+        L.tall = tall;
+        const bool halo = conv_uses_halo(L);
+        L.tr = orient && halo;
+        L.wide = orient && !halo;
+        if (!conv_shape_ok(L)) continue;
+        const int items = batch * conv_m_tiles(L) * (L.cout / bn) * sp;
+        const int rounds = (items + grid - 1) / grid;
+        const double cost =
+            rounds * (double)((total_kb + sp - 1) / sp) * kblock_cost(bn) * (tall ? kTallCost : 1.0);
+        if (cost < best - 1e-9) {
+          best = cost;
+          out->bn = bn;
+          out->tall = L.tall;
+          out->tr = L.tr;
+          out->wide = L.wide;
+        }
       }
     }
   }
@@ -629,7 +639,7 @@ rtcc_status build_backbone(rtcc_ctx* c) {
         // a split layer whose items fit the clustered grid keeps the DSMEM
         // exchange (64-wide tiles); otherwise it reduces through global memory
         const bool dsm_fit = L.splits > 1 && nb * m_tiles * (L.cout / 64) * L.splits <= grid;
-        pick_tile_batch(L, L.splits, grid, nb, dsm_fit, &L.bn, &L.tall);
+        pick_tile_batch(L, L.splits, grid, nb, dsm_fit, &L);
         L.n_tiles_n = L.cout / L.bn;
       }
       L.ws = c->batch_ws;

@@ -52,6 +52,8 @@ namespace {
 constexpr int TW = 8;                        // tile width in pixels: one 8-row MMA atom per image row
 constexpr int TH = 16;                       // tile height
 constexpr int kTallTH = 2 * TH;              // height of a tall tile: two MMA row blocks
+constexpr int kWideTW = 2 * TW;              // wide tile of a tap-box layer: 16 x 8 pixels,
+constexpr int kWideTH = TH / 2;              // two MMA atoms per image row (BM rows all the same)
 constexpr int BM = TW * TH;                  // 128 = MMA M
 // warps: 0 TMA producer, 1 MMA issuer, 2..5 epilogue, 6..7 more TMA producers
 constexpr int kThreads = 256;
@@ -169,6 +171,9 @@ struct LayerScalars {
   int halo;                // A from halo tiles; k-blocks chunk-major (kb = 9 chunk + tap)
   int tall;                // halo layers: tiles of TW x kTallTH pixels (two MMA row blocks
                            // sharing every weight box) instead of TW x TH
+  int tw_log2, th;         // tile width (a power of two) and height in tile coordinates
+  int tr;                  // tile coordinates transposed: tile x runs along the image's
+                           // rows (H), tile y along W (halo layers)
   int kpb;                 // k-blocks per pipeline stage: halo layers put the weight boxes of
                            // kBBytes / (bn * 128) taps into one stage, others 1 (A + B)
   int spc;                 // halo layers: stages per 64-channel chunk (a stage never spans
@@ -203,6 +208,9 @@ __device__ __forceinline__ LayerScalars layer_scalars(const LayerDesc& D, int n_
   S.wait_items = D.wait_items;
   S.halo = D.halo;
   S.tall = D.tall;
+  S.tw_log2 = __ffs(D.tw) - 1;
+  S.th = D.th;
+  S.tr = D.tr;
   S.out = D.out;
   S.out_astride = D.out_astride;
   S.ipa = D.ipa;
@@ -246,8 +254,8 @@ __device__ __forceinline__ Item item_of(const LayerScalars& S, int t, const int*
   it.tile = t / S.splits;
   const int mt = it.tile % S.m_tiles;
   const int nt = it.tile / S.m_tiles;
-  it.x0 = (mt % S.tiles_x) * TW;
-  it.y0 = (mt / S.tiles_x) * (S.tall ? kTallTH : TH);
+  it.x0 = (mt % S.tiles_x) << S.tw_log2;
+  it.y0 = (mt / S.tiles_x) * (S.tall ? kTallTH : S.th);
   it.n0 = nt * S.bn;
   it.kb0 = (it.z * S.total_kb) / S.splits;
   it.kb1 = ((it.z + 1) * S.total_kb) / S.splits;
@@ -369,8 +377,10 @@ __device__ __forceinline__ void mma_kblock(uint32_t d_tmem, uint32_t a_lo, uint3
 // back to back; a stage of kpb taps (km = kpb - 1) starts with a wait on its
 // weight box and ends with a commit that frees it.  TALL: the tile's lower
 // row block (accumulator columns +128) takes the same weight box with the A
-// rows TH halo rows further down.  False if a wait runs out.
-template <bool TALL>
+// rows TH halo rows further down.  TR: the halo tile is stored in transposed
+// tile coordinates (tile x along the image's H), so image tap (dy, dx)
+// starts dx halo rows and dy atoms-rows in.  False if a wait runs out.
+template <bool TALL, bool TR>
 __device__ __forceinline__ bool halo_chunk_mma(uint32_t d_tmem, uint32_t a_lo, uint32_t a_hi, uint32_t b_lo0,
                                                uint32_t b_hi, uint32_t idesc, int km, uint32_t bstep,
                                                bool accumulate, uint64_t* full, uint64_t* empty, uint32_t& it,
@@ -385,7 +395,8 @@ __device__ __forceinline__ bool halo_chunk_mma(uint32_t d_tmem, uint32_t a_lo, u
       tc_fence_after();
       b_lo = b_lo0 + (uint32_t)(s * (kBBytes >> 4));
     }
-    const uint32_t a_tap = a_lo + (uint32_t)(((tap / 3) * kHaloW + tap % 3) * 8);
+    const int tap_y = TR ? tap % 3 : tap / 3, tap_x = TR ? tap / 3 : tap % 3;
+    const uint32_t a_tap = a_lo + (uint32_t)((tap_y * kHaloW + tap_x) * 8);
     const uint32_t b_tap = b_lo + (uint32_t)(tap & km) * bstep;
     const uint32_t accum = (accumulate || tap > 0) ? 1u : 0u;
     mma_kblock(d_tmem, a_tap, a_hi, b_tap, b_hi, idesc, accum, true);
@@ -677,10 +688,16 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
               }
               ++hc;
               const uint32_t a_lo = (uint32_t)smem_desc(smem0 + h * kHaloSlot, kHaloW * 128, 2u);
-              const bool ok = tall ? halo_chunk_mma<true>(d_tmem, a_lo, a_hi_halo, b_lo0, b_hi, idesc, km, bstep,
-                                                          c > 0, full, empty, it, budget)
-                                   : halo_chunk_mma<false>(d_tmem, a_lo, a_hi_halo, b_lo0, b_hi, idesc, km, bstep,
-                                                           c > 0, full, empty, it, budget);
+              const bool acc_in = c > 0;
+              const bool ok =
+                  tall ? (S.tr ? halo_chunk_mma<true, true>(d_tmem, a_lo, a_hi_halo, b_lo0, b_hi, idesc, km, bstep,
+                                                            acc_in, full, empty, it, budget)
+                               : halo_chunk_mma<true, false>(d_tmem, a_lo, a_hi_halo, b_lo0, b_hi, idesc, km,
+                                                             bstep, acc_in, full, empty, it, budget))
+                       : (S.tr ? halo_chunk_mma<false, true>(d_tmem, a_lo, a_hi_halo, b_lo0, b_hi, idesc, km,
+                                                             bstep, acc_in, full, empty, it, budget)
+                               : halo_chunk_mma<false, false>(d_tmem, a_lo, a_hi_halo, b_lo0, b_hi, idesc, km,
+                                                              bstep, acc_in, full, empty, it, budget));
               if (!ok) {
                 atomicOr(P.err, ERR_WAIT_MMA);
                 alive = false;
@@ -740,7 +757,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
         // of a deconv.  Null outside the image (ragged tiles).
         T* orow = nullptr;
         {
-          const int px = I.x0 + row % TW, py = I.y0 + row / TW;
+          const int px = I.x0 + (row & ((1 << S.tw_log2) - 1)), py = I.y0 + (row >> S.tw_log2);
           if (px < S.gw && py < S.gh) {
             size_t pix;
             int c0;
@@ -750,7 +767,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
               pix = (size_t)(py * S.s + sy) * S.ow + (size_t)(px * S.s + sx);
               c0 = S.choff;
             } else {
-              pix = (size_t)py * S.ow + px;
+              pix = S.tr ? (size_t)px * S.ow + py : (size_t)py * S.ow + px;
               c0 = S.choff + I.n0;
             }
             orow = static_cast<T*>(S.out) + (size_t)I.agent * S.out_astride + pix * S.ldc + c0;
@@ -768,10 +785,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_backbone(const __grid_constant_
           for (int hh = 0; hh < halves; ++hh) {
             T* o = orow;
             if (hh > 0) {
+              // tall tiles are TW wide
               const int px = I.x0 + row % TW, py = I.y0 + TH + row / TW;
+              const size_t pix = S.tr ? (size_t)px * S.ow + py : (size_t)py * S.ow + px;
               o = (px < S.gw && py < S.gh)
-                      ? static_cast<T*>(S.out) + (size_t)I.agent * S.out_astride +
-                            ((size_t)py * S.ow + px) * S.ldc + S.choff + I.n0
+                      ? static_cast<T*>(S.out) + (size_t)I.agent * S.out_astride + pix * S.ldc + S.choff + I.n0
                       : nullptr;
             }
             const uint32_t ta = taddr + (uint32_t)(hh * 128);
@@ -1066,9 +1084,25 @@ cudaError_t tmap_3d(CUtensorMap* m, const void* base, bool bf16, uint64_t inner,
 int conv_tile_w() { return TW; }
 int conv_tile_h() { return TH; }
 int conv_tile_m() { return BM; }
+// The tile grid of layer L: tile width and height, and the extent the tiles
+// cover in tile coordinates (the image's W x H, or H x W when transposed).
+static void tile_grid(const ConvLayer& L, int* tw, int* th, int* gx, int* gy) {
+  *tw = L.wide ? kWideTW : TW;
+  *th = L.tall ? kTallTH : L.wide ? kWideTH : TH;
+  *gx = L.tr ? L.gh : L.gw;
+  *gy = L.tr ? L.gw : L.gh;
+}
 int conv_m_tiles(const ConvLayer& L) {
-  const int th = L.tall ? kTallTH : TH;
-  return ((L.gw + TW - 1) / TW) * ((L.gh + th - 1) / th);
+  int tw, th, gx, gy;
+  tile_grid(L, &tw, &th, &gx, &gy);
+  return ((gx + tw - 1) / tw) * ((gy + th - 1) / th);
+}
+bool conv_shape_ok(const ConvLayer& L) {
+  const bool halo = conv_uses_halo(L);
+  if (L.tall && (!halo || L.splits != 1)) return false;
+  if (L.tr && (!halo || L.splits != 1 || L.wide)) return false;
+  if (L.wide && (L.kind == DECONV || halo || L.splits != 1)) return false;
+  return true;
 }
 
 cudaError_t conv_make_maps(ConvLayer& L, bool bf16) {
@@ -1086,22 +1120,25 @@ cudaError_t conv_make_maps(ConvLayer& L, bool bf16) {
       (L.kind == DECONV && L.out_astride < (long long)L.out_w * L.out_h * L.ldc))
     return cudaErrorInvalidValue;
   CUresult r;
+  if (!conv_shape_ok(L)) return cudaErrorInvalidValue;
+  const cuuint32_t tw = (cuuint32_t)(L.wide ? kWideTW : TW), th = (cuuint32_t)(L.wide ? kWideTH : TH);
   if (L.kind == CONV3_S2) {
     if ((L.in_w & 1) || (L.in_h & 1)) return cudaErrorInvalidValue;
     cuuint64_t dims[5] = {2 * C, W / 2, 2, H / 2, NA};
     cuuint64_t strides[4] = {2 * C * 2, W * C * 2, 2 * W * C * 2, AS};
-    cuuint32_t box[5] = {(cuuint32_t)L.bk, (cuuint32_t)TW, 1, (cuuint32_t)TH, 1};
+    cuuint32_t box[5] = {(cuuint32_t)L.bk, tw, 1, th, 1};
     cuuint32_t es[5] = {1, 1, 1, 1, 1};
     r = enc(&L.mapA, dt, 5, const_cast<void*>(L.in), dims, strides, box, es,
             CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   } else {
-    cuuint64_t dims[4] = {C, W, H, NA};
-    cuuint64_t strides[3] = {C * 2, W * C * 2, AS};
+    // transposed halo layers walk the image with H as the tile's x: the same
+    // NHWC tensor described with its two pixel dimensions swapped
+    cuuint64_t dims[4] = {C, L.tr ? H : W, L.tr ? W : H, NA};
+    cuuint64_t strides[3] = {L.tr ? W * C * 2 : C * 2, L.tr ? C * 2 : W * C * 2, AS};
     const bool halo = conv_uses_halo(L);
-    if (L.tall && !halo) return cudaErrorInvalidValue;
-    cuuint32_t box[4] = {(cuuint32_t)L.bk, (cuuint32_t)(halo ? kHaloW : TW),
-                         (cuuint32_t)(halo ? (L.tall ? kHaloHTall : kHaloH) : TH), 1};
+    cuuint32_t box[4] = {(cuuint32_t)L.bk, (cuuint32_t)(halo ? kHaloW : tw),
+                         (cuuint32_t)(halo ? (L.tall ? kHaloHTall : kHaloH) : th), 1};
     cuuint32_t es[4] = {1, 1, 1, 1};
     r = enc(&L.mapA, dt, 4, const_cast<void*>(L.in), dims, strides, box, es,
             CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
@@ -1212,10 +1249,15 @@ cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, int n_batch, uns
     D.bn = L.bn;
     D.bk = L.bk;
     D.splits = L.splits;
-    if (L.tall && (!conv_uses_halo(L) || L.splits != 1)) return cudaErrorInvalidValue;
-    D.tiles_x = (L.gw + TW - 1) / TW;
+    if (!conv_shape_ok(L)) return cudaErrorInvalidValue;
+    int tw, th, gx, gy;
+    tile_grid(L, &tw, &th, &gx, &gy);
+    D.tiles_x = (gx + tw - 1) / tw;
     D.m_tiles = conv_m_tiles(L);
     D.tall = L.tall ? 1 : 0;
+    D.tw = tw;
+    D.th = L.wide ? kWideTH : TH;
+    D.tr = L.tr ? 1 : 0;
     D.n_tiles = L.n_tiles_n;
     D.choff = L.choff;
     D.wait_layers = L.wait_layers;
@@ -1224,8 +1266,8 @@ cudaError_t backbone_fill(const std::vector<ConvLayer>& layers, int n_batch, uns
     D.ipa = D.m_tiles * D.n_tiles * L.splits;
     D.ow = L.out_w;
     D.ldc = L.ldc;
-    D.gw = L.gw;
-    D.gh = L.gh;
+    D.gw = gx;
+    D.gh = gy;
     D.halo = conv_uses_halo(L) ? 1 : 0;
     // a split of a 64-wide tile into 2 or kMaxSplits slices, one item per
     // CTA, reduces its slices through distributed shared memory within a

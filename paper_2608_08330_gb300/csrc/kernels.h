@@ -140,6 +140,9 @@ struct ConvLayer {
   int splits;            // split-K factor; 1 = none
   int tall;              // halo layers without split-K: tiles of 8 x 32 pixels, two
                          // 128-row MMAs per weight box (0: 8 x 16 pixels)
+  int tr;                // halo layers without split-K: tiles walk the image transposed,
+                         // 8 pixels along H by 16 (tall: 32) along W
+  int wide;              // tap-box convs without split-K: tiles of 16 x 8 pixels
   int wait_layers;       // this layer reads outputs of layers [0, wait_layers)
   float* ws;             // split-K partials [batch][splits][m_tiles * n_tiles][128][bn] fp32
   int* counters;         // split-K arrivals per tile [batch][m_tiles * n_tiles], zero-initialised
@@ -167,6 +170,8 @@ int conv_tile_h();                 // rows of a tile (a tall tile has twice as m
 int conv_tile_m();
 // M tiles of layer L's grid with its tile shape
 int conv_m_tiles(const ConvLayer& L);
+// Whether L's tile shape flags (tall, tr, wide) fit its kind and split.
+bool conv_shape_ok(const ConvLayer& L);
 
 // One layer of the persistent backbone kernel (kernel-parameter layout).
 constexpr int kMaxLayers = 20;
@@ -185,6 +190,8 @@ struct alignas(128) LayerDesc {   // CUtensorMap is 128-byte aligned
   int wait_items;                // items of layer wait_layers - 1 (its counter's target)
   int halo;                      // 3x3 stride-1 with 64-channel k-blocks: A from halo tiles
   int tall;                      // halo layers: tiles two MMA row blocks high (see ConvLayer)
+  int tw, th;                    // tile width and height (one MMA row block) in pixels
+  int tr;                        // tile x along the image's H (see ConvLayer)
   void* out;                     // output [agent][out_h][ow][ldc], channels from choff
   long long out_astride;         // elements between agents in `out`
   int ow, ldc, gw, gh;           // output row length, pixel stride, tile grid extent
