@@ -259,15 +259,17 @@ rtcc_status rtcc_frame_begin(struct rtcc_ctx* ctx, uint64_t frame_id, double t0_
  * stay unchanged until rtcc_wait_detection returns for this frame; when it is
  * the staging buffer no host copy is made.
  *
- * Launches (Sec. III-B's single encoder stream, kept busy): a branch released
- * while no backbone runs starts at once, pillar chain and backbone.  One
- * released while another branch's backbone still runs starts its pillar chain
- * at once; its backbone is held and, when the running backbone ends, the
- * dispatcher thread launches one backbone over every branch held meanwhile.
- * Branches released by one event (Barrier at A) share one launch, and the
- * event that resolves the last branch launches whatever is held at once.
- * Every branch writes its own slot and its result does not depend on the
- * launch that ran it, so RTCC and Barrier outputs stay byte-identical.
+ * Launches (Sec. III-B's single encoder stream, kept busy): a released branch
+ * starts its pillar chain before return.  Unless it resolves the last branch,
+ * its backbone is held: the dispatcher thread launches one backbone over every
+ * held branch once the backbone in flight (if any) has ended and no release
+ * has come for 40 us, so completions reported close together share a launch.
+ * Branches released by one event (Barrier at A) share one launch.  The event
+ * that resolves the last branch launches at once: alone onto a free GPU as
+ * the branch's own graph (pillar chain and backbone), else together with
+ * whatever is held.  Every branch writes its own slot and its result does not
+ * depend on the launch that ran it, so RTCC and Barrier outputs stay
+ * byte-identical.
  */
 rtcc_status rtcc_payload_complete(struct rtcc_ctx* ctx, int32_t agent,
                                   const float* host_points, int32_t n_points,
