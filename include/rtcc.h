@@ -483,6 +483,40 @@ rtcc_status rtcc_uplink_simulate(int32_t n_agents, int32_t n_rb, int32_t t_max,
                                  int32_t* n_slots_used);
 
 /* ------------------------------------------------------------------------ */
+/* Backbone tile plan (host only; no counterpart in the paper)              */
+/* ------------------------------------------------------------------------ */
+
+/* How one 3x3 conv layer of the backbone is cut into work items. */
+typedef struct {
+  int32_t splits;       /* K slices per tile (split-K); fixed for every batch
+                           size, since they decide the fp32 summation order  */
+  int32_t bn;           /* output channels per item (32, 64 or 128)          */
+  int32_t tall;         /* 1: tiles of 8 x 32 pixels (two 128-row MMAs per
+                           weight box), else 8 x 16 (or 16 x 8 when wide)   */
+  int32_t transposed;   /* 1: the tiles' 8-pixel side runs along the image's
+                           rows (H) instead of W                            */
+  int32_t wide;         /* 1: tiles of 16 x 8 pixels (stride-2 and other
+                           layers that load one box per tap)                */
+  int32_t m_tiles;      /* pixel tiles covering one agent's output          */
+  int32_t items;        /* work items of the launch:
+                           n_batch x m_tiles x (cout / bn) x splits         */
+} rtcc_conv_plan;
+
+/*
+ * The tile choice rtcc_init makes for one 3x3 conv layer (pad 1) of a
+ * backbone launch over n_batch agents on `grid` CTAs: kind 0 = stride 1,
+ * 1 = stride 2; cin, cout its channels; out_w x out_h its output.  The K
+ * slices come from the one-agent cost model, the N tile and tile shape from
+ * the cost model at n_batch (rounds of items over the grid x k-blocks per
+ * item x the k-block's MMA time).  Pure host arithmetic: no device, no
+ * context.  RTCC_E_ARG unless kind is 0 or 1, cin is a power of two in
+ * 32..256, cout is a multiple of 32 in 32..256, the extents and grid are
+ * positive and 1 <= n_batch <= RTCC_MAX_AGENTS; `out` is caller-owned.
+ */
+rtcc_status rtcc_plan_conv(int32_t kind, int32_t cin, int32_t cout, int32_t out_w, int32_t out_h,
+                           int32_t grid, int32_t n_batch, rtcc_conv_plan* out);
+
+/* ------------------------------------------------------------------------ */
 /* Misc                                                                     */
 /* ------------------------------------------------------------------------ */
 

@@ -447,6 +447,27 @@ void pick_tile_batch(const ConvLayer L0, int sp, int grid, int batch, bool need6
   }
 }
 
+// The K slices of conv layer L (its split-K factor, with its K chunk and a
+// first N tile) from the one-agent model; they stay the same for every batch
+// size.  L's kind, channels and output extent (gw x gh) must be set.
+void choose_split(ConvLayer& L, int grid) {
+  const int m_tiles = ((L.gw + conv_tile_w() - 1) / conv_tile_w()) * ((L.gh + conv_tile_h() - 1) / conv_tile_h());
+  L.bk = (L.cin >= 64) ? 64 : 32;
+  pick_tile(m_tiles, L.cout, 9 * (L.cin / L.bk), grid, &L.bn, &L.splits);
+  L.n_tiles_n = L.cout / L.bn;
+}
+
+// The N tile and tile shape of conv layer L (K slices already chosen) in a
+// launch over nb agents.  A split layer whose items fit the clustered grid
+// keeps the DSMEM exchange (64-wide tiles); otherwise it reduces through
+// global memory.
+void choose_tiles(ConvLayer& L, int grid, int nb) {
+  const int m_tiles = conv_m_tiles(L);
+  const bool dsm_fit = L.splits > 1 && nb * m_tiles * (L.cout / 64) * L.splits <= grid;
+  pick_tile_batch(L, L.splits, grid, nb, dsm_fit, &L);
+  L.n_tiles_n = L.cout / L.bn;
+}
+
 // The backbone's layer list over the agent-major tensors of all K agents, and
 // the launch parameters for every batch size.
 rtcc_status build_backbone(rtcc_ctx* c) {
@@ -493,11 +514,7 @@ rtcc_status build_backbone(rtcc_ctx* c) {
       L.gh = oh;
       L.ldc = co;
       L.choff = 0;
-      const int m_tiles = ((ow + conv_tile_w() - 1) / conv_tile_w()) *
-                          ((oh + conv_tile_h() - 1) / conv_tile_h());
-      L.bk = (cin >= 64) ? 64 : 32;
-      pick_tile(m_tiles, co, 9 * (cin / L.bk), grid, &L.bn, &L.splits);
-      L.n_tiles_n = co / L.bn;
+      choose_split(L, grid);
       L.in = in;
       L.in_astride = in_as;
       const bool last = (bi == g.n_blocks - 1) && (li == g.block_layers[bi] - 1);
@@ -634,14 +651,7 @@ rtcc_status build_backbone(rtcc_ctx* c) {
   for (int nb = 1; nb <= K; ++nb) {
     std::vector<ConvLayer> Lb = c->layers;
     for (ConvLayer& L : Lb) {
-      if (L.kind != DECONV) {
-        const int m_tiles = conv_m_tiles(L);           // short tiles (the one-agent K slices)
-        // a split layer whose items fit the clustered grid keeps the DSMEM
-        // exchange (64-wide tiles); otherwise it reduces through global memory
-        const bool dsm_fit = L.splits > 1 && nb * m_tiles * (L.cout / 64) * L.splits <= grid;
-        pick_tile_batch(L, L.splits, grid, nb, dsm_fit, &L);
-        L.n_tiles_n = L.cout / L.bn;
-      }
+      if (L.kind != DECONV) choose_tiles(L, grid, nb);
       L.ws = c->batch_ws;
       L.counters = c->batch_cnt;
       if (conv_make_maps(L, c->bf16) != cudaSuccess) return RTCC_E_CUDA;
@@ -1624,6 +1634,30 @@ rtcc_status rtcc_get_frame_info(rtcc_ctx* c, rtcc_frame_info* info) {
   if (!c || !info) return RTCC_E_ARG;
   std::lock_guard<std::mutex> lk(c->mu);
   *info = c->info;
+  return RTCC_OK;
+}
+
+rtcc_status rtcc_plan_conv(int32_t kind, int32_t cin, int32_t cout, int32_t out_w, int32_t out_h,
+                           int32_t grid, int32_t n_batch, rtcc_conv_plan* out) {
+  if (!out || (kind != 0 && kind != 1) || cin < 32 || cin > 256 || cout < 32 || cout > 256 ||
+      cin % 32 || cout % 32 || (cin & (cin - 1)) || out_w < 1 || out_h < 1 || grid < 1 ||
+      n_batch < 1 || n_batch > RTCC_MAX_AGENTS)
+    return RTCC_E_ARG;
+  ConvLayer L{};
+  L.kind = kind == 1 ? CONV3_S2 : CONV3_S1;
+  L.cin = cin;
+  L.cout = cout;
+  L.gw = out_w;
+  L.gh = out_h;
+  choose_split(L, grid);
+  choose_tiles(L, grid, n_batch);
+  out->splits = L.splits;
+  out->bn = L.bn;
+  out->tall = L.tall;
+  out->transposed = L.tr;
+  out->wide = L.wide;
+  out->m_tiles = conv_m_tiles(L);
+  out->items = n_batch * out->m_tiles * (cout / L.bn) * L.splits;
   return RTCC_OK;
 }
 

@@ -68,6 +68,12 @@ class rtcc_frame_info(C.Structure):
     ]
 
 
+class rtcc_conv_plan(C.Structure):
+    _fields_ = [("splits", C.c_int32), ("bn", C.c_int32), ("tall", C.c_int32),
+                ("transposed", C.c_int32), ("wide", C.c_int32), ("m_tiles", C.c_int32),
+                ("items", C.c_int32)]
+
+
 BOX_DTYPE = np.dtype([("x", "<f4"), ("y", "<f4"), ("z", "<f4"), ("l", "<f4"), ("w", "<f4"),
                       ("h", "<f4"), ("yaw", "<f4"), ("score", "<f4"), ("anchor", "<i4")])
 
@@ -142,6 +148,8 @@ def load(path: Optional[str] = None) -> C.CDLL:
         "rtcc_uplink_simulate": (S, [C.c_int32, C.c_int32, C.c_int32, C.c_void_p, C.c_void_p,
                                      C.c_void_p, C.c_double, C.c_int32, C.c_void_p, C.c_void_p,
                                      C.POINTER(C.c_int32)]),
+        "rtcc_plan_conv": (S, [C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_int32, C.c_int32,
+                               C.c_int32, C.POINTER(rtcc_conv_plan)]),
         "rtcc_pillarise_noalloc": (S, [C.POINTER(rtcc_model_config), C.c_void_p, C.c_int32,
                                        C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
                                        C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]),
@@ -377,6 +385,15 @@ def rtcc_uplink_simulate(payload_bits, first_slot, rates: np.ndarray, slot_s: fl
                                      None if wt is None else _ptr(wt), _ptr(out), C.byref(used)),
          "rtcc_uplink_simulate")
     return out, used.value
+
+
+def rtcc_plan_conv(kind: int, cin: int, cout: int, out_w: int, out_h: int, grid: int,
+                   n_batch: int) -> dict:
+    """The backbone's tile choice for one 3x3 conv layer (see rtcc.h)."""
+    p = rtcc_conv_plan()
+    _chk(load().rtcc_plan_conv(int(kind), int(cin), int(cout), int(out_w), int(out_h), int(grid),
+                               int(n_batch), C.byref(p)), "rtcc_plan_conv")
+    return {f: int(getattr(p, f)) for f, _ in rtcc_conv_plan._fields_}
 
 
 def rtcc_test_unreachable_wait(ctx) -> int:
