@@ -1292,8 +1292,10 @@ rtcc_status after_event(rtcc_ctx* c, const std::vector<int>& released, double t_
     if (released.size() > 1 || last) {
       RS(launch_batch(c));
     } else {
-      c->t_hold.store(now_ms(), std::memory_order_relaxed);
+      // the hold starts after the wake-up call, which can take microseconds;
+      // the dispatcher reads it only once this call has released the mutex
       c->cv.notify_all();
+      c->t_hold.store(now_ms(), std::memory_order_relaxed);
     }
   }
   if (last && !c->post_launched) {

@@ -164,15 +164,29 @@ def test_release_hold_gathers_a_burst_and_lets_a_lone_branch_go(R):
         ref = R.rtcc_get_head(ctx, cfg.feat_h, cfg.feat_w).tobytes()
         info = R.rtcc_get_frame_info(ctx)
         assert list(info.backbone_batch)[:info.n_backbone_launches] == [2]
-        # back to back: one launch (a host stall past the hold splits it, so
-        # the burst gets a few tries)
+        # back to back (resident payloads, so the calls are short): the second
+        # completion joins the first one's launch when it comes within the
+        # hold.  A slow host can miss the hold, so the library's release stamps
+        # decide what to expect: a second release less than 30 us after the
+        # first was inside the hold and must have shared the launch
+        for k in range(cfg.n_agents):
+            assert R.rtcc_stage_resident(ctx, k, pts[k]) == R.OK
         burst = []
-        for f in range(3):
-            U.run_frame(ctx, cfg, pts, [0.0, 0.0], R.MODE_RTCC, frame_id=2 + f)
+        for f in range(5):
+            assert R.rtcc_set_mode(ctx, R.MODE_RTCC) == R.OK
+            assert R.rtcc_frame_begin(ctx, 2 + f, 0.0) == R.OK
+            for k in range(cfg.n_agents):
+                assert R.rtcc_payload_resident(ctx, k, 0.0) == R.OK
+            s, _, _ = R.rtcc_wait_detection(ctx, 60000)
+            assert s == R.OK, R.rtcc_status_str(s)
             assert R.rtcc_get_head(ctx, cfg.feat_h, cfg.feat_w).tobytes() == ref
             info = R.rtcc_get_frame_info(ctx)
-            burst.append(list(info.backbone_batch)[:info.n_backbone_launches])
-        assert [2] in burst, burst
+            sizes = list(info.backbone_batch)[:info.n_backbone_launches]
+            gap_us = (info.t_release_ms[1] - info.t_release_ms[0]) * 1e3
+            burst.append((sizes, round(gap_us, 1)))
+            assert sizes in ([2], [1, 1]), burst
+            if gap_us < 30.0:
+                assert sizes == [2], burst
         # 20 ms apart: agent 0's backbone runs alone after the hold and has
         # ended when agent 1 arrives
         assert R.rtcc_frame_begin(ctx, 9, 0.0) == R.OK
