@@ -52,8 +52,8 @@ namespace {
 constexpr int TW = 8;                        // tile width in pixels: one 8-row MMA atom per image row
 constexpr int TH = 16;                       // tile height
 constexpr int kTallTH = 2 * TH;              // height of a tall tile: two MMA row blocks
-constexpr int kWideTW = 2 * TW;              // wide tile of a tap-box layer: 16 x 8 pixels,
-constexpr int kWideTH = TH / 2;              // two MMA atoms per image row (BM rows all the same)
+constexpr int kWideTW = 2 * TW;              // wide tile of a tap-box layer: 16 x 8 = BM pixels,
+constexpr int kWideTH = TH / 2;              // two MMA atoms per image row of its dense boxes
 constexpr int BM = TW * TH;                  // 128 = MMA M
 // warps: 0 TMA producer, 1 MMA issuer, 2..5 epilogue, 6..7 more TMA producers
 constexpr int kThreads = 256;
@@ -378,8 +378,9 @@ __device__ __forceinline__ void mma_kblock(uint32_t d_tmem, uint32_t a_lo, uint3
 // weight box and ends with a commit that frees it.  TALL: the tile's lower
 // row block (accumulator columns +128) takes the same weight box with the A
 // rows TH halo rows further down.  TR: the halo tile is stored in transposed
-// tile coordinates (tile x along the image's H), so image tap (dy, dx)
-// starts dx halo rows and dy atoms-rows in.  False if a wait runs out.
+// tile coordinates (tile x along the image's H), so image tap (dy, dx) starts
+// dx * kHaloW + dy rows into it instead of dy * kHaloW + dx.  False if a wait
+// runs out.
 template <bool TALL, bool TR>
 __device__ __forceinline__ bool halo_chunk_mma(uint32_t d_tmem, uint32_t a_lo, uint32_t a_hi, uint32_t b_lo0,
                                                uint32_t b_hi, uint32_t idesc, int km, uint32_t bstep,
