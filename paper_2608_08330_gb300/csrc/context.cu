@@ -1313,8 +1313,8 @@ rtcc_status after_event(rtcc_ctx* c, const std::vector<int>& released, double t_
 constexpr double kHoldMs = 0.04;
 
 // Launches the pending batch once the backbone in flight has ended and the
-// hold has run out (see after_event).  Waits for the end on the launch's done word in pinned host
-// memory, without the context mutex.
+// hold has run out (see after_event).  Waits for the end on the launch's done
+// word in pinned host memory, without the context mutex.
 void dispatcher_main(rtcc_ctx* c) {
   cudaSetDevice(c->dev);
   std::unique_lock<std::mutex> lk(c->mu);
