@@ -707,6 +707,10 @@ def run_ours(args):
         for resident in (True, False):
             key = ("" if resident else "e2e_") + f"{cfg.name}_{spread}"
             lat[key] = quad(tails(spread, resident, R.MODE_RTCC), tails(spread, resident, R.MODE_BARRIER))
+    # all-simultaneous RTCC frames whose branches shared one backbone launch
+    # (the dispatcher's hold gathered the burst)
+    one = [len(r["launches"]) == 1 for (sp, res, m, r) in rec if sp == "zero" and m == R.MODE_RTCC]
+    lat["rtcc_zero_one_launch"] = round(sum(one) / len(one), 3) if one else None
     value = pct(tails("lognormal", True, R.MODE_RTCC), 50)
     e2e_value = pct(tails("lognormal", False, R.MODE_RTCC), 50)
     if dist is not None:
